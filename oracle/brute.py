@@ -1,0 +1,51 @@
+"""Pure-Python brute force of the CompressKV selection for tiny prompts.
+
+TEST INFRASTRUCTURE ONLY (same rule as ``compresskv_oracle``).  It restates
+Sec. 3.3 (window scoring, pooling, top-N retention) with explicit loops,
+``math.exp`` and ``math.fsum`` over Python floats, and a full sort for the
+top-k, so that the numpy oracle can be checked against an implementation
+that shares none of its code.  Meant for prompts of at most a few dozen
+tokens.
+"""
+from __future__ import annotations
+
+import math
+
+
+def brute_unit(q_heads, k_unit, window, pool_width, budget, scale):
+    """q_heads: list over SRH heads of W lists of d floats; k_unit: L lists of
+    d floats.  Returns (raw, pooled, indices) as Python lists."""
+    L = len(k_unit)
+    W = window
+    if budget < W:
+        raise ValueError("budget smaller than window")
+    if L <= W:
+        return [], [], list(range(L))
+    n = L - W
+    raw = [0.0] * n
+    terms = [[] for _ in range(n)]
+    for head in q_heads:
+        for w in range(W):
+            p = L - W + w
+            logits = []
+            for j in range(p + 1):
+                logits.append(scale * math.fsum(a * b for a, b in zip(head[w], k_unit[j])))
+            top = max(logits)
+            exps = [math.exp(x - top) for x in logits]
+            z = math.fsum(exps)
+            for j in range(n):
+                terms[j].append(exps[j] / z)
+    for j in range(n):
+        raw[j] = math.fsum(terms[j])
+    r = (pool_width - 1) // 2
+    pooled = []
+    for j in range(n):
+        acc = []
+        for t in range(-r, r + 1):
+            if 0 <= j + t < n:
+                acc.append(raw[j + t])
+        pooled.append(math.fsum(acc) / pool_width)
+    k = min(budget, L) - W
+    ranked = sorted(range(n), key=lambda j: (-pooled[j], j))
+    chosen = sorted(ranked[:k])
+    return raw, pooled, chosen + list(range(n, L))
