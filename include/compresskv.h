@@ -1,0 +1,191 @@
+/*
+ * compresskv.h -- C ABI of the CompressKV prefill-end KV-cache compression
+ * path on one GB300 (sm_103a).
+ *
+ * The method (CompressKV, Sec. 3.3 "Token Selection Driven by Semantic
+ * Retrieval Heads", with the SnapKV-style local setting of Sec. 4
+ * "Implementation Details"): for every sequence s and GQA KV group g of a
+ * layer (a *unit*),
+ *   1. score each prefix token j < n = L_s - W by the causal softmax
+ *      attention of the last W prompt queries of the group's Semantic
+ *      Retrieval Heads (SRH; the SRH mask is an input, identified offline per
+ *      Sec. 3.2), summed over the window queries and the SRH heads;
+ *   2. smooth the scores with 1-D average pooling of width P over tokens;
+ *   3. keep the k = min(B, L_s) - W prefix tokens with the largest pooled
+ *      score (ties to the lower position) plus the W window tokens, where B is
+ *      the layer's budget from the offline layer-wise allocation (Sec. 3.4);
+ *   4. gather the retained K and V rows into a contiguous compressed cache.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - All tensor arguments are DEVICE pointers unless marked "host".  The
+ *   caller allocates and frees every buffer, including the workspace; the
+ *   library allocates no device memory, keeps no per-call global state and
+ *   never synchronises the stream (except compresskv_read_device_status).
+ * - Work is enqueued on `stream` (a cudaStream_t, NULL = legacy default).
+ *   Entry points return after enqueueing; results are ready when the stream
+ *   reaches them.  Argument errors are detected on the host before anything
+ *   is enqueued; launch failures return CKV_ERR_CUDA.  Errors found by a
+ *   kernel (a bounded wait that ran out, an index out of range passed to
+ *   compresskv_gather) are written to the status word at the start of the
+ *   workspace and read with compresskv_read_device_status.
+ * - Sequences are packed: sequence s owns rows cu_seqlens[s] ..
+ *   cu_seqlens[s+1]-1 of K and V (host array of batch+1 ints, first entry 0).
+ *   L_s = cu_seqlens[s+1] - cu_seqlens[s], n_s = max(L_s - W, 0).
+ * - K, V: [T][num_kv_heads][head_dim] elements of `dtype`, head_dim contiguous,
+ *   element strides kv_token_stride / kv_head_stride (multiples of 8, base
+ *   16-byte aligned).  V shares K's strides.
+ * - Window queries q_win: element (s, h, w, :) at
+ *   q_win + s*q_batch_stride + h*q_head_stride + w*q_win_stride, head_dim
+ *   contiguous; row w is the query of prompt position L_s - W + w.
+ *   Strides are multiples of 8 elements, base 16-byte aligned.  Q and K are
+ *   taken as given (post-RoPE); no RoPE is applied.
+ * - GQA grouping: query head h belongs to KV group h / (num_q_heads /
+ *   num_kv_heads).
+ * - Prefix-score layout ("score layout"): float [num_kv_heads][P_total],
+ *   P_total = sum_s n_s, sequence s at offset cu_prefix[s] = sum_{s'<s} n_s'.
+ * - Output layout: kept_s = min(budget_s, L_s) tokens per sequence,
+ *   cu_out[s] = sum_{s'<s} kept_s', O_total = cu_out[batch];
+ *   indices: int32 [num_kv_heads][O_total], positions within the sequence in
+ *   ascending order (the W window positions are the last W entries of a
+ *   compressed sequence); k_out / v_out: [O_total][num_kv_heads][head_dim]
+ *   contiguous, in the input dtype, bit-exact copies of the retained rows.
+ * - Scores are the sum over SRH heads and window queries (the paper averages
+ *   the head vectors; within a unit the head count is fixed, so the ranking
+ *   is the same).
+ */
+#ifndef COMPRESSKV_H_
+#define COMPRESSKV_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes returned by every entry point (and stored by kernels in the
+ * workspace status word). */
+enum {
+  CKV_OK = 0,
+  CKV_ERR_INVALID_ARG = -1,     /* null pointer, bad shape/stride/alignment */
+  CKV_ERR_UNSUPPORTED = -2,     /* valid but outside what the kernels take (see limits) */
+  CKV_ERR_BUDGET = -3,          /* a budget smaller than the window W */
+  CKV_ERR_EMPTY_SRH_GROUP = -4, /* a KV group with no SRH head but a sequence to score */
+  CKV_ERR_WORKSPACE = -5,       /* workspace null or smaller than compresskv_workspace_size */
+  CKV_ERR_CUDA = -6,            /* a CUDA runtime call or kernel launch failed */
+  CKV_ERR_DEVICE_TIMEOUT = -7,  /* a kernel's bounded wait ran out (device status only) */
+  CKV_ERR_DEVICE_INDEX = -8     /* compresskv_gather got an index outside its sequence */
+};
+
+enum { CKV_DTYPE_F16 = 0, CKV_DTYPE_BF16 = 1 };
+enum { CKV_POOL_AVG = 0 };
+
+/* Kernel kinds reported through ckv_trace. */
+enum {
+  CKV_KERNEL_SCORE_STATS = 1,   /* scoring pass 1: per-query softmax max / normaliser */
+  CKV_KERNEL_SCORE_ACCUM = 2,   /* scoring pass 2: normalised attention summed per token */
+  CKV_KERNEL_SELECT = 3,        /* pooling + top-k + window append */
+  CKV_KERNEL_GATHER = 4         /* retained K/V rows -> compressed cache */
+};
+
+/* Optional launch trace.  When ckv_problem.trace is non-null every kernel
+ * launch is bracketed by two caller-created CUDA events (cudaEvent_t handles
+ * in `events`, 2 per launch) recorded on the call's stream, and its kind is
+ * stored in `kinds`.  Inside a stream capture the events are recorded as
+ * external event nodes.  Once `count` reaches `capacity` further launches
+ * are only counted.  The caller zeroes `count` and `launches`. */
+typedef struct ckv_trace {
+  void** events;       /* [2*capacity] cudaEvent_t */
+  int32_t* kinds;      /* [capacity] host */
+  int32_t capacity;
+  int32_t count;       /* launches recorded so far */
+  int64_t launches;    /* kernels launched so far */
+} ckv_trace;
+
+/* One layer's problem description (host memory). */
+typedef struct ckv_problem {
+  int32_t batch;            /* sequences, 1..512 */
+  int32_t num_q_heads;      /* H_q, 1..256, a multiple of num_kv_heads */
+  int32_t num_kv_heads;     /* H_kv, 1..64 */
+  int32_t head_dim;         /* d; 128 */
+  int32_t window;           /* W >= 1, the observation window (Sec. 4) */
+  int32_t pool_width;       /* P, odd, 1..63, average pooling width (Sec. 4) */
+  int32_t dtype;            /* CKV_DTYPE_F16 | CKV_DTYPE_BF16 for Q, K and V */
+  int32_t pool_kind;        /* CKV_POOL_AVG */
+  float scale;              /* softmax scale; 0 selects 1/sqrt(head_dim) */
+  int32_t reserved;         /* must be 0 */
+  const int32_t* cu_seqlens;/* host [batch+1] */
+  int64_t kv_token_stride;  /* elements between consecutive tokens of K/V */
+  int64_t kv_head_stride;   /* elements between KV heads of K/V */
+  int64_t q_batch_stride;   /* elements, window queries */
+  int64_t q_head_stride;
+  int64_t q_win_stride;
+  ckv_trace* trace;         /* optional launch trace, NULL for none */
+} ckv_problem;
+
+/* Bytes of device workspace the calls below need for problem `p` (depends
+ * on the shapes and cu_seqlens only; an upper bound over every SRH mask).
+ * Returns 0 if `p` is invalid. */
+size_t compresskv_workspace_size(const ckv_problem* p);
+
+/* Zero the workspace status word (enqueued on `stream`).  Call once after
+ * allocating a workspace, and after reading a non-zero device status. */
+int compresskv_workspace_init(void* workspace, size_t workspace_bytes, void* stream);
+
+/* Host-only: per-sequence offsets of the prefix scores (cu_prefix, [batch+1])
+ * and of the compressed output (cu_out, [batch+1]) for the given host
+ * budgets ([batch]).  Either output may be NULL.  Returns CKV_ERR_BUDGET if a
+ * budget is below W. */
+int compresskv_output_layout(const ckv_problem* p, const int32_t* budgets,
+                             int32_t* cu_prefix, int32_t* cu_out);
+
+/* Step 1 (Sec. 3.3): raw prefix scores.
+ * srh_mask: host uint8 [num_q_heads], non-zero = SRH head of this layer.
+ * raw_scores: device float, score layout, written for every prefix token.
+ * Per unit, |S_g| * W must not exceed 256 query rows (CKV_ERR_UNSUPPORTED). */
+int compresskv_score(const ckv_problem* p, const void* q_win, const void* k,
+                     const uint8_t* srh_mask, float* raw_scores,
+                     void* workspace, size_t workspace_bytes, void* stream);
+
+/* Steps 2-3 (Sec. 3.3, Sec. 4): average pooling of width P, top-k of the
+ * pooled prefix scores, window append.
+ * budgets: host int32 [batch] (per sequence, including the W window tokens).
+ * indices: device int32 [num_kv_heads][O_total] (output layout).
+ * cu_out: host int32 [batch+1], written.
+ * pooled_scores: optional device float in score layout (NULL for none). */
+int compresskv_select(const ckv_problem* p, const float* raw_scores,
+                      const int32_t* budgets, int32_t* indices, int32_t* cu_out,
+                      float* pooled_scores, void* workspace, size_t workspace_bytes,
+                      void* stream);
+
+/* Step 4 (Sec. 3.3): copy the retained K/V rows.
+ * indices / cu_out as produced by compresskv_select (cu_out on the host);
+ * an index outside [0, L_s) is skipped and reported as CKV_ERR_DEVICE_INDEX
+ * in the device status of `workspace` (which may be NULL to skip
+ * reporting). */
+int compresskv_gather(const ckv_problem* p, const int32_t* indices, const int32_t* cu_out,
+                      const void* k, const void* v, void* k_out, void* v_out,
+                      void* workspace, void* stream);
+
+/* Steps 1-4 fused for one layer: score, select, gather.
+ * raw_scores / pooled_scores are optional outputs (NULL: kept in the
+ * workspace).  cu_out: host int32 [batch+1], written. */
+int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const void* k,
+                              const void* v, const uint8_t* srh_mask, const int32_t* budgets,
+                              int32_t* indices, int32_t* cu_out, void* k_out, void* v_out,
+                              float* raw_scores, float* pooled_scores,
+                              void* workspace, size_t workspace_bytes, void* stream);
+
+/* Synchronise `stream`, copy the workspace status word to *status and return
+ * CKV_OK (or CKV_ERR_CUDA if the copy fails). */
+int compresskv_read_device_status(const void* workspace, void* stream, int32_t* status);
+
+/* Static text for a status code. */
+const char* compresskv_status_string(int status);
+
+#ifdef __cplusplus
+}  /* extern "C" */
+#endif
+
+#endif  /* COMPRESSKV_H_ */

@@ -81,10 +81,11 @@ def window_attention(q_rows: np.ndarray, k_unit: np.ndarray, scale: float) -> np
     k = np.asarray(k_unit, dtype=np.float64)
     W = q.shape[0]
     L = k.shape[0]
+    Z = (q @ k.T) * scale                      # [W, L] logits
     A = np.zeros((W, L), dtype=np.float64)
     for w in range(W):
-        p = L - W + w
-        z = (k[: p + 1] @ q[w]) * scale
+        p = L - W + w                          # causal: keys 0..p only
+        z = Z[w, : p + 1]
         e = np.exp(z - z.max())
         A[w, : p + 1] = e / e.sum()
     return A

@@ -1,0 +1,284 @@
+"""ctypes binding of libcompresskv (include/compresskv.h).
+
+Argument marshalling only: every step of the compression path runs in the
+library's CUDA kernels.  PyTorch supplies device memory and streams.  There
+is no fallback: if the library is missing or fails to load, importing the
+binding raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from ctypes import POINTER, c_float, c_int32, c_int64, c_size_t, c_void_p
+
+import numpy as np
+import torch
+
+from . import _build
+
+CKV_OK = 0
+CKV_ERR_INVALID_ARG = -1
+CKV_ERR_UNSUPPORTED = -2
+CKV_ERR_BUDGET = -3
+CKV_ERR_EMPTY_SRH_GROUP = -4
+CKV_ERR_WORKSPACE = -5
+CKV_ERR_CUDA = -6
+CKV_ERR_DEVICE_TIMEOUT = -7
+CKV_ERR_DEVICE_INDEX = -8
+CKV_DTYPE_F16 = 0
+CKV_DTYPE_BF16 = 1
+CKV_POOL_AVG = 0
+KERNEL_KINDS = {1: "score_stats", 2: "score_accum", 3: "select", 4: "gather"}
+
+EXPORTED = (
+    "compresskv_workspace_size",
+    "compresskv_workspace_init",
+    "compresskv_output_layout",
+    "compresskv_score",
+    "compresskv_select",
+    "compresskv_gather",
+    "compresskv_compress_layer",
+    "compresskv_read_device_status",
+    "compresskv_status_string",
+)
+
+
+class CkvTrace(ctypes.Structure):
+    _fields_ = [("events", POINTER(c_void_p)), ("kinds", POINTER(c_int32)),
+                ("capacity", c_int32), ("count", c_int32), ("launches", c_int64)]
+
+
+class CkvProblem(ctypes.Structure):
+    _fields_ = [("batch", c_int32), ("num_q_heads", c_int32), ("num_kv_heads", c_int32),
+                ("head_dim", c_int32), ("window", c_int32), ("pool_width", c_int32),
+                ("dtype", c_int32), ("pool_kind", c_int32), ("scale", c_float),
+                ("reserved", c_int32), ("cu_seqlens", POINTER(c_int32)),
+                ("kv_token_stride", c_int64), ("kv_head_stride", c_int64),
+                ("q_batch_stride", c_int64), ("q_head_stride", c_int64),
+                ("q_win_stride", c_int64), ("trace", POINTER(CkvTrace))]
+
+
+class CompressKVError(RuntimeError):
+    def __init__(self, code: int, what: str):
+        super().__init__(f"{what}: {status_string(code)} ({code})")
+        self.code = code
+
+
+_LIB = None
+
+
+def library_path() -> str:
+    return _build.LIB_PATH
+
+
+def load(build_if_missing: bool = True) -> ctypes.CDLL:
+    """Load libcompresskv (building it first if it is absent or stale)."""
+    global _LIB
+    if _LIB is not None:
+        return _LIB
+    path = library_path()
+    if build_if_missing and _build.needs_build():
+        _build.build()
+    if not os.path.exists(path):
+        raise RuntimeError(f"libcompresskv not built ({path}); run __graft_entry__.build()")
+    lib = ctypes.CDLL(path)
+    vp, pp = c_void_p, POINTER(CkvProblem)
+    i32p = POINTER(c_int32)
+    sig = {
+        "compresskv_workspace_size": (c_size_t, [pp]),
+        "compresskv_workspace_init": (c_int32, [vp, c_size_t, vp]),
+        "compresskv_output_layout": (c_int32, [pp, i32p, i32p, i32p]),
+        "compresskv_score": (c_int32, [pp, vp, vp, vp, vp, vp, c_size_t, vp]),
+        "compresskv_select": (c_int32, [pp, vp, i32p, vp, i32p, vp, vp, c_size_t, vp]),
+        "compresskv_gather": (c_int32, [pp, vp, i32p, vp, vp, vp, vp, vp, vp]),
+        "compresskv_compress_layer": (c_int32, [pp, vp, vp, vp, vp, i32p, vp, i32p, vp, vp,
+                                                 vp, vp, vp, c_size_t, vp]),
+        "compresskv_read_device_status": (c_int32, [vp, vp, i32p]),
+        "compresskv_status_string": (ctypes.c_char_p, [c_int32]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _LIB = lib
+    return lib
+
+
+def status_string(code: int) -> str:
+    return load().compresskv_status_string(int(code)).decode()
+
+
+def _check(code: int, what: str):
+    if code != CKV_OK:
+        raise CompressKVError(code, what)
+
+
+def _ptr(t) -> c_void_p:
+    if t is None:
+        return c_void_p(None)
+    return c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def _i32(arr) -> tuple:
+    a = np.ascontiguousarray(np.asarray(arr, dtype=np.int32))
+    return a, a.ctypes.data_as(POINTER(c_int32))
+
+
+class Problem:
+    """One layer's problem description (wraps ``ckv_problem``).
+
+    ``q_win`` is ``[B, H_q, W, d]`` and ``k`` is ``[T, H_kv, d]`` (any
+    strides with ``d`` contiguous); only shapes, strides and dtype are read.
+    """
+
+    def __init__(self, q_win: torch.Tensor, k: torch.Tensor, cu_seqlens, window: int,
+                 pool_width: int, scale: float = 0.0, trace: "Trace | None" = None):
+        if k.dtype not in (torch.float16, torch.bfloat16) or q_win.dtype != k.dtype:
+            raise CompressKVError(CKV_ERR_INVALID_ARG, "Q and K must share an f16/bf16 dtype")
+        self._cu, cu_ptr = _i32(cu_seqlens)
+        self.trace = trace
+        s = CkvProblem()
+        s.batch = len(self._cu) - 1
+        s.num_q_heads = q_win.shape[1]
+        s.num_kv_heads = k.shape[1]
+        s.head_dim = k.shape[2]
+        s.window = int(window)
+        s.pool_width = int(pool_width)
+        s.dtype = CKV_DTYPE_BF16 if k.dtype == torch.bfloat16 else CKV_DTYPE_F16
+        s.pool_kind = CKV_POOL_AVG
+        s.scale = float(scale)
+        s.reserved = 0
+        s.cu_seqlens = cu_ptr
+        s.kv_token_stride = k.stride(0)
+        s.kv_head_stride = k.stride(1)
+        s.q_batch_stride = q_win.stride(0)
+        s.q_head_stride = q_win.stride(1)
+        s.q_win_stride = q_win.stride(2)
+        s.trace = ctypes.pointer(trace.struct) if trace is not None else None
+        self.struct = s
+        self.batch = s.batch
+        self.num_kv_heads = s.num_kv_heads
+
+    @property
+    def ref(self):
+        return ctypes.byref(self.struct)
+
+
+class Trace:
+    """Launch trace: ``capacity`` launches bracketed by CUDA events."""
+
+    def __init__(self, capacity: int):
+        self.events = [torch.cuda.Event(enable_timing=True) for _ in range(2 * capacity)]
+        self._ev = (c_void_p * (2 * capacity))(*[e.cuda_event for e in self.events])
+        self._kinds = (c_int32 * capacity)()
+        self.struct = CkvTrace(ctypes.cast(self._ev, POINTER(c_void_p)),
+                               ctypes.cast(self._kinds, POINTER(c_int32)), capacity, 0, 0)
+
+    def reset(self):
+        self.struct.count = 0
+        self.struct.launches = 0
+
+    @property
+    def launches(self) -> int:
+        return int(self.struct.launches)
+
+    def records(self):
+        """[(kind name, elapsed ms)] for the recorded launches (call after a sync)."""
+        out = []
+        for i in range(self.struct.count):
+            out.append((KERNEL_KINDS.get(self._kinds[i], "?"),
+                        self.events[2 * i].elapsed_time(self.events[2 * i + 1])))
+        return out
+
+
+def workspace_size(problem: Problem) -> int:
+    n = load().compresskv_workspace_size(problem.ref)
+    if n == 0:
+        raise CompressKVError(CKV_ERR_INVALID_ARG, "compresskv_workspace_size")
+    return int(n)
+
+
+def workspace(problem: Problem, device=None, stream=None) -> torch.Tensor:
+    """A zero-status workspace tensor for ``problem`` (256-byte aligned)."""
+    n = workspace_size(problem)
+    ws = torch.empty(n, dtype=torch.uint8, device=device or "cuda")
+    assert ws.data_ptr() % 256 == 0
+    _check(load().compresskv_workspace_init(_ptr(ws), n, _stream(stream)), "workspace_init")
+    return ws
+
+
+def output_layout(problem: Problem, budgets):
+    b, bp = _i32(budgets)
+    cu_prefix = np.zeros(problem.batch + 1, np.int32)
+    cu_out = np.zeros(problem.batch + 1, np.int32)
+    _check(load().compresskv_output_layout(problem.ref, bp,
+                                           cu_prefix.ctypes.data_as(POINTER(c_int32)),
+                                           cu_out.ctypes.data_as(POINTER(c_int32))),
+           "output_layout")
+    return cu_prefix, cu_out
+
+
+def _mask(srh_mask):
+    m = np.ascontiguousarray(np.asarray(srh_mask).astype(np.uint8))
+    return m, c_void_p(m.ctypes.data)
+
+
+def score(problem: Problem, q_win, k, srh_mask, raw, ws, stream=None):
+    m, mp = _mask(srh_mask)
+    _check(load().compresskv_score(problem.ref, _ptr(q_win), _ptr(k), mp, _ptr(raw), _ptr(ws),
+                                   ws.numel(), _stream(stream)), "compresskv_score")
+
+
+def select(problem: Problem, raw, budgets, indices, ws, pooled=None, stream=None) -> np.ndarray:
+    b, bp = _i32(budgets)
+    cu_out = np.zeros(problem.batch + 1, np.int32)
+    _check(load().compresskv_select(problem.ref, _ptr(raw), bp, _ptr(indices),
+                                    cu_out.ctypes.data_as(POINTER(c_int32)), _ptr(pooled),
+                                    _ptr(ws), ws.numel(), _stream(stream)), "compresskv_select")
+    return cu_out
+
+
+def gather(problem: Problem, indices, cu_out, k, v, k_out, v_out, ws=None, stream=None):
+    c, cp = _i32(cu_out)
+    _check(load().compresskv_gather(problem.ref, _ptr(indices), cp, _ptr(k), _ptr(v),
+                                    _ptr(k_out), _ptr(v_out), _ptr(ws), _stream(stream)),
+           "compresskv_gather")
+
+
+def compress_layer(problem: Problem, q_win, k, v, srh_mask, budgets, indices, k_out, v_out, ws,
+                   raw=None, pooled=None, stream=None) -> np.ndarray:
+    m, mp = _mask(srh_mask)
+    b, bp = _i32(budgets)
+    cu_out = np.zeros(problem.batch + 1, np.int32)
+    _check(load().compresskv_compress_layer(
+        problem.ref, _ptr(q_win), _ptr(k), _ptr(v), mp, bp, _ptr(indices),
+        cu_out.ctypes.data_as(POINTER(c_int32)), _ptr(k_out), _ptr(v_out), _ptr(raw),
+        _ptr(pooled), _ptr(ws), ws.numel(), _stream(stream)), "compresskv_compress_layer")
+    return cu_out
+
+
+def read_device_status(ws, stream=None) -> int:
+    out = c_int32(0)
+    _check(load().compresskv_read_device_status(_ptr(ws), _stream(stream), ctypes.byref(out)),
+           "read_device_status")
+    return int(out.value)
+
+
+class LayerOutputs:
+    """Device buffers for one compressed layer, sized from the budgets."""
+
+    def __init__(self, problem: Problem, budgets, head_dim: int, dtype, device, scores=True):
+        cu_prefix, cu_out = output_layout(problem, budgets)
+        H = problem.num_kv_heads
+        self.cu_prefix, self.cu_out = cu_prefix, cu_out
+        self.indices = torch.empty((H, int(cu_out[-1])), dtype=torch.int32, device=device)
+        self.k_out = torch.empty((int(cu_out[-1]), H, head_dim), dtype=dtype, device=device)
+        self.v_out = torch.empty_like(self.k_out)
+        self.raw = torch.empty((H, int(cu_prefix[-1])), dtype=torch.float32, device=device) if scores else None
+        self.pooled = torch.empty_like(self.raw) if scores else None

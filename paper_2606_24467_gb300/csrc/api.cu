@@ -1,0 +1,528 @@
+// Host side of the C ABI declared in include/compresskv.h: argument
+// validation, SRH mask -> per-group head lists, unit-set and work-item
+// planning, K tensor map, workspace carving and kernel launches.
+// No device memory is allocated and no stream is synchronised here (except
+// in compresskv_read_device_status).
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "ckv_params.h"
+#include "compresskv.h"
+
+using namespace ckv;
+
+namespace {
+
+constexpr size_t kStatusBytes = 256;
+constexpr size_t kPartialBytes = static_cast<size_t>(kMaxItems) * kMaxQRows * sizeof(float2);
+
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+// ------------------------------------------------------------------ device facts
+struct DeviceFacts {
+  int sms = 0;
+  long long l2_bytes = 0;
+  bool smem_attr_set = false;
+};
+
+std::mutex g_mutex;
+DeviceFacts g_facts[64];
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+int device_facts(DeviceFacts** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return CKV_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_mutex);
+  DeviceFacts& f = g_facts[dev];
+  if (f.sms == 0) {
+    int sms = 0, l2 = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return CKV_ERR_CUDA;
+    if (cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev) != cudaSuccess) return CKV_ERR_CUDA;
+    f.sms = sms;
+    f.l2_bytes = l2;
+  }
+  if (!f.smem_attr_set) {
+    int optin = 0;
+    if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+      return CKV_ERR_CUDA;
+    if (score_set_smem_limit(static_cast<size_t>(optin)) != cudaSuccess) return CKV_ERR_CUDA;
+    if (select_set_smem_limit(static_cast<size_t>(optin) - 9 * 1024) != cudaSuccess)
+      return CKV_ERR_CUDA;
+    f.smem_attr_set = true;
+  }
+  if (!g_encode) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !fn)
+      return CKV_ERR_CUDA;
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }
+  *out = &f;
+  return CKV_OK;
+}
+
+// ------------------------------------------------------------------ validation
+struct Info {
+  int B = 0, Hq = 0, Hkv = 0, G = 0, W = 0, P = 0;
+  bool bf16 = false;
+  float scale = 0.f;
+  std::vector<int> cu, len, n, cu_prefix;
+  long long T = 0, p_total = 0;
+};
+
+bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
+
+int validate(const ckv_problem* p, Info& I) {
+  if (!p || !p->cu_seqlens) return CKV_ERR_INVALID_ARG;
+  if (p->batch < 1 || p->batch > kMaxBatch) return CKV_ERR_UNSUPPORTED;
+  if (p->num_kv_heads < 1 || p->num_q_heads < 1) return CKV_ERR_INVALID_ARG;
+  if (p->num_q_heads % p->num_kv_heads != 0) return CKV_ERR_INVALID_ARG;
+  if (p->num_kv_heads > kMaxKvHeads || p->num_q_heads > kMaxQHeads) return CKV_ERR_UNSUPPORTED;
+  if (p->head_dim != kHeadDim) return CKV_ERR_UNSUPPORTED;
+  if (p->window < 1) return CKV_ERR_INVALID_ARG;
+  if (p->pool_width < 1 || p->pool_width % 2 == 0 || p->pool_width > 63) return CKV_ERR_INVALID_ARG;
+  if (p->dtype != CKV_DTYPE_F16 && p->dtype != CKV_DTYPE_BF16) return CKV_ERR_INVALID_ARG;
+  if (p->pool_kind != CKV_POOL_AVG) return CKV_ERR_UNSUPPORTED;
+  if (p->reserved != 0) return CKV_ERR_INVALID_ARG;
+  if (!(p->scale >= 0.f) || std::isinf(p->scale)) return CKV_ERR_INVALID_ARG;
+  if (p->kv_token_stride <= 0 || p->kv_head_stride <= 0 || p->kv_token_stride % 8 ||
+      p->kv_head_stride % 8)
+    return CKV_ERR_INVALID_ARG;
+  if (p->q_batch_stride < 0 || p->q_head_stride < 0 || p->q_win_stride < 0 ||
+      p->q_batch_stride % 8 || p->q_head_stride % 8 || p->q_win_stride % 8)
+    return CKV_ERR_INVALID_ARG;
+  I.B = p->batch;
+  I.Hq = p->num_q_heads;
+  I.Hkv = p->num_kv_heads;
+  I.G = I.Hq / I.Hkv;
+  I.W = p->window;
+  I.P = p->pool_width;
+  I.bf16 = p->dtype == CKV_DTYPE_BF16;
+  I.scale = p->scale > 0.f ? p->scale : 1.0f / std::sqrt(static_cast<float>(kHeadDim));
+  I.cu.assign(p->cu_seqlens, p->cu_seqlens + I.B + 1);
+  if (I.cu[0] != 0) return CKV_ERR_INVALID_ARG;
+  I.len.resize(I.B);
+  I.n.resize(I.B);
+  I.cu_prefix.assign(I.B + 1, 0);
+  for (int s = 0; s < I.B; ++s) {
+    const long long L = static_cast<long long>(I.cu[s + 1]) - I.cu[s];
+    if (L < 0) return CKV_ERR_INVALID_ARG;
+    if (L > 65535LL * kTileTokens) return CKV_ERR_UNSUPPORTED;
+    I.len[s] = static_cast<int>(L);
+    I.n[s] = std::max(I.len[s] - I.W, 0);
+    I.cu_prefix[s + 1] = I.cu_prefix[s] + I.n[s];
+  }
+  I.T = I.cu[I.B];
+  I.p_total = I.cu_prefix[I.B];
+  if (static_cast<long long>(I.Hkv) * I.p_total > (1LL << 31) - 1) return CKV_ERR_UNSUPPORTED;
+  return CKV_OK;
+}
+
+int output_layout(const Info& I, const int32_t* budgets, std::vector<int>& cu_out) {
+  if (!budgets) return CKV_ERR_INVALID_ARG;
+  cu_out.assign(I.B + 1, 0);
+  for (int s = 0; s < I.B; ++s) {
+    if (budgets[s] < I.W) return CKV_ERR_BUDGET;
+    cu_out[s + 1] = cu_out[s] + std::min(budgets[s], I.len[s]);
+  }
+  if (static_cast<long long>(I.Hkv) * cu_out[I.B] > (1LL << 31) - 1) return CKV_ERR_UNSUPPORTED;
+  return CKV_OK;
+}
+
+struct Workspace {
+  int* status = nullptr;
+  float2* partials = nullptr;
+  float* raw = nullptr;
+  float* pooled = nullptr;
+};
+
+size_t workspace_bytes(const Info& I) {
+  const size_t scores = align256(static_cast<size_t>(I.Hkv) * I.p_total * sizeof(float));
+  return kStatusBytes + kPartialBytes + 2 * scores;
+}
+
+int carve(const Info& I, void* ws, size_t bytes, Workspace& out) {
+  if (!ws || bytes < workspace_bytes(I) || (reinterpret_cast<uintptr_t>(ws) & 255u))
+    return CKV_ERR_WORKSPACE;
+  char* b = static_cast<char*>(ws);
+  const size_t scores = align256(static_cast<size_t>(I.Hkv) * I.p_total * sizeof(float));
+  out.status = reinterpret_cast<int*>(b);
+  out.partials = reinterpret_cast<float2*>(b + kStatusBytes);
+  out.raw = reinterpret_cast<float*>(b + kStatusBytes + kPartialBytes);
+  out.pooled = reinterpret_cast<float*>(b + kStatusBytes + kPartialBytes + scores);
+  return CKV_OK;
+}
+
+// ------------------------------------------------------------------ tracing
+struct Tracer {
+  ckv_trace* t;
+  cudaStream_t s;
+  int slot = -1;
+  void begin(int kind) {
+    slot = -1;
+    if (!t) return;
+    if (t->count < t->capacity && t->events) {
+      slot = t->count++;
+      if (t->kinds) t->kinds[slot] = kind;
+      record(static_cast<cudaEvent_t>(t->events[2 * slot]));
+    }
+  }
+  void end() {
+    if (!t) return;
+    ++t->launches;
+    if (slot >= 0) record(static_cast<cudaEvent_t>(t->events[2 * slot + 1]));
+  }
+  void record(cudaEvent_t e) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    cudaStreamIsCapturing(s, &cs);
+    if (cs == cudaStreamCaptureStatusActive)
+      cudaEventRecordWithFlags(e, s, cudaEventRecordExternal);
+    else
+      cudaEventRecord(e, s);
+  }
+};
+
+// ------------------------------------------------------------------ scoring
+struct SrhLists {
+  std::vector<uint16_t> off;
+  std::vector<uint8_t> heads;
+  std::vector<int> rows;  // |S_g| * W per group
+};
+
+int srh_lists(const Info& I, const uint8_t* mask, SrhLists& S) {
+  if (!mask) return CKV_ERR_INVALID_ARG;
+  S.off.assign(I.Hkv + 1, 0);
+  S.heads.clear();
+  S.rows.assign(I.Hkv, 0);
+  bool any_scored = false;
+  for (int s = 0; s < I.B; ++s) any_scored |= I.n[s] > 0;
+  for (int g = 0; g < I.Hkv; ++g) {
+    for (int h = g * I.G; h < (g + 1) * I.G; ++h)
+      if (mask[h]) S.heads.push_back(static_cast<uint8_t>(h));
+    S.off[g + 1] = static_cast<uint16_t>(S.heads.size());
+    const int cnt = S.off[g + 1] - S.off[g];
+    if (cnt == 0 && any_scored) return CKV_ERR_EMPTY_SRH_GROUP;
+    S.rows[g] = cnt * I.W;
+    if (S.rows[g] > kMaxQRows) return CKV_ERR_UNSUPPORTED;
+  }
+  return CKV_OK;
+}
+
+int make_k_map(const Info& I, const ckv_problem* p, const void* k, CUtensorMap* map) {
+  if (I.T == 0) return CKV_OK;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(I.Hkv),
+                        static_cast<cuuint64_t>(I.T)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(p->kv_head_stride) * 2,
+                           static_cast<cuuint64_t>(p->kv_token_stride) * 2};
+  cuuint32_t box[3] = {64u, 1u, static_cast<cuuint32_t>(kTileTokens)};
+  cuuint32_t estr[3] = {1u, 1u, 1u};
+  CUresult r = g_encode(map, I.bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16,
+                        3, const_cast<void*>(k), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? CKV_OK : CKV_ERR_INVALID_ARG;
+}
+
+int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void* k,
+              const uint8_t* mask, float* raw, const Workspace& ws, cudaStream_t stream) {
+  if (!q_win || !k || !raw) return CKV_ERR_INVALID_ARG;
+  if (!aligned16(q_win) || !aligned16(k)) return CKV_ERR_INVALID_ARG;
+  SrhLists S;
+  int rc = srh_lists(I, mask, S);
+  if (rc != CKV_OK) return rc;
+  DeviceFacts* F = nullptr;
+  if ((rc = device_facts(&F)) != CKV_OK) return rc;
+  if (I.p_total == 0) return CKV_OK;
+
+  static thread_local ScoreParams P;  // large (about 17 KB): kept off the stack
+  std::memset(&P, 0, sizeof(P));
+  if ((rc = make_k_map(I, p, k, &P.tmap_k)) != CKV_OK) return rc;
+  P.q = static_cast<const uint16_t*>(q_win);
+  P.partials = ws.partials;
+  P.raw = raw;
+  P.status = ws.status;
+  P.q_bs = p->q_batch_stride;
+  P.q_hs = p->q_head_stride;
+  P.q_ws = p->q_win_stride;
+  P.c = static_cast<float>(static_cast<double>(I.scale) * 1.4426950408889634);
+  P.window = I.W;
+  P.num_kv_heads = I.Hkv;
+  P.p_total = static_cast<int>(I.p_total);
+  P.is_bf16 = I.bf16 ? 1 : 0;
+  P.use_evict_hint = 1;
+  for (int s = 0; s <= I.B; ++s) {
+    P.cu_seqlens[s] = I.cu[s];
+    P.cu_prefix[s] = I.cu_prefix[s];
+  }
+  for (int g = 0; g <= I.Hkv; ++g) P.srh_off[g] = S.off[g];
+  for (size_t h = 0; h < S.heads.size(); ++h) P.srh_heads[h] = S.heads[h];
+
+  // Units (s, g) with a prefix to score, grouped into sets whose K fits in
+  // about half of the L2, so that pass 2 re-reads K from L2.
+  struct Unit { int s, g, tiles; };
+  std::vector<Unit> units;
+  for (int s = 0; s < I.B; ++s)
+    if (I.n[s] > 0)
+      for (int g = 0; g < I.Hkv; ++g)
+        units.push_back({s, g, (I.len[s] + kTileTokens - 1) / kTileTokens});
+  const long long set_budget = std::max<long long>(F->l2_bytes / 2, 1LL << 20);
+  size_t u0 = 0;
+  Tracer tr{p->trace, stream};
+  while (u0 < units.size()) {
+    size_t u1 = u0;
+    long long bytes = 0;
+    long long tiles = 0;
+    while (u1 < units.size()) {
+      const long long ub = static_cast<long long>(units[u1].tiles) * kTileBytes;
+      if (u1 > u0 && (bytes + ub > set_budget || static_cast<long long>(u1 - u0) >= kMaxItems / 2))
+        break;
+      bytes += ub;
+      tiles += units[u1].tiles;
+      ++u1;
+    }
+    // Work items: about one per SM in total, balanced tile ranges per unit.
+    const long long target = std::max(1, F->sms);
+    const long long chunk = std::max<long long>(1, (tiles + target - 1) / target);
+    int n_items = 0;
+    int max_rows = 16;
+    for (size_t u = u0; u < u1; ++u) {
+      const Unit& U = units[u];
+      const int cnt = static_cast<int>((U.tiles + chunk - 1) / chunk);
+      if (n_items + cnt > kMaxItems) return CKV_ERR_UNSUPPORTED;
+      for (int c = 0; c < cnt; ++c) {
+        WorkItem& it = P.items[n_items + c];
+        it.seq = static_cast<uint16_t>(U.s);
+        it.group = static_cast<uint16_t>(U.g);
+        it.t0 = static_cast<uint16_t>(static_cast<long long>(U.tiles) * c / cnt);
+        it.t1 = static_cast<uint16_t>(static_cast<long long>(U.tiles) * (c + 1) / cnt);
+        it.first = static_cast<uint16_t>(n_items);
+        it.count = static_cast<uint16_t>(cnt);
+      }
+      n_items += cnt;
+      max_rows = std::max(max_rows, (S.rows[U.g] + 15) & ~15);
+    }
+    P.n_items = n_items;
+    P.q_half_bytes = ((max_rows * 128) + 1023) & ~1023;
+    const size_t smem = score_smem_bytes(P.q_half_bytes);
+    tr.begin(CKV_KERNEL_SCORE_STATS);
+    cudaError_t e = launch_score_stats(P, n_items, smem, stream);
+    tr.end();
+    if (e != cudaSuccess) return CKV_ERR_CUDA;
+    tr.begin(CKV_KERNEL_SCORE_ACCUM);
+    e = launch_score_accum(P, n_items, smem, stream);
+    tr.end();
+    if (e != cudaSuccess) return CKV_ERR_CUDA;
+    u0 = u1;
+  }
+  return CKV_OK;
+}
+
+// ------------------------------------------------------------------ select / gather
+int run_select(const ckv_problem* p, const Info& I, const float* raw, const std::vector<int>& cu_out,
+               int32_t* indices, float* pooled, const Workspace& ws, cudaStream_t stream) {
+  if (!raw && I.p_total > 0) return CKV_ERR_INVALID_ARG;
+  if (!indices && cu_out[I.B] > 0) return CKV_ERR_INVALID_ARG;
+  DeviceFacts* F = nullptr;
+  int rc = device_facts(&F);
+  if (rc != CKV_OK) return rc;
+  if (cu_out[I.B] == 0 && !pooled) return CKV_OK;
+  static thread_local SelectParams P;
+  std::memset(&P, 0, sizeof(P));
+  P.raw = raw;
+  P.pooled_out = pooled;
+  P.pooled_ws = ws.pooled;
+  P.indices = indices;
+  P.status = ws.status;
+  P.window = I.W;
+  P.pool_width = I.P;
+  P.num_kv_heads = I.Hkv;
+  P.p_total = static_cast<int>(I.p_total);
+  P.o_total = cu_out[I.B];
+  P.batch = I.B;
+  int max_n = 0;
+  for (int s = 0; s <= I.B; ++s) {
+    P.cu_seqlens[s] = I.cu[s];
+    P.cu_prefix[s] = I.cu_prefix[s];
+    P.cu_out[s] = cu_out[s];
+    if (s < I.B) max_n = std::max(max_n, I.n[s]);
+  }
+  P.smem_floats = std::min(max_n, select_max_smem_floats());
+  Tracer tr{p->trace, stream};
+  tr.begin(CKV_KERNEL_SELECT);
+  cudaError_t e = launch_select(P, I.B * I.Hkv, static_cast<size_t>(P.smem_floats) * 4, stream);
+  tr.end();
+  return e == cudaSuccess ? CKV_OK : CKV_ERR_CUDA;
+}
+
+int run_gather(const ckv_problem* p, const Info& I, const int32_t* indices,
+               const std::vector<int>& cu_out, const void* k, const void* v, void* k_out,
+               void* v_out, int* status, cudaStream_t stream) {
+  const long long rows = static_cast<long long>(cu_out[I.B]) * I.Hkv;
+  if (rows == 0) return CKV_OK;
+  if (!indices || !k || !v || !k_out || !v_out) return CKV_ERR_INVALID_ARG;
+  if (!aligned16(k) || !aligned16(v) || !aligned16(k_out) || !aligned16(v_out))
+    return CKV_ERR_INVALID_ARG;
+  static thread_local GatherParams P;
+  std::memset(&P, 0, sizeof(P));
+  P.k = static_cast<const uint4*>(k);
+  P.v = static_cast<const uint4*>(v);
+  P.k_out = static_cast<uint4*>(k_out);
+  P.v_out = static_cast<uint4*>(v_out);
+  P.indices = indices;
+  P.status = status;
+  P.tok_stride_v16 = p->kv_token_stride / 8;
+  P.head_stride_v16 = p->kv_head_stride / 8;
+  P.num_kv_heads = I.Hkv;
+  P.o_total = cu_out[I.B];
+  P.batch = I.B;
+  for (int s = 0; s <= I.B; ++s) {
+    P.cu_seqlens[s] = I.cu[s];
+    P.cu_out[s] = cu_out[s];
+  }
+  Tracer tr{p->trace, stream};
+  tr.begin(CKV_KERNEL_GATHER);
+  cudaError_t e = launch_gather(P, rows, stream);
+  tr.end();
+  return e == cudaSuccess ? CKV_OK : CKV_ERR_CUDA;
+}
+
+}  // namespace
+
+// ====================================================================== C ABI
+extern "C" {
+
+size_t compresskv_workspace_size(const ckv_problem* p) {
+  Info I;
+  if (validate(p, I) != CKV_OK) return 0;
+  return workspace_bytes(I);
+}
+
+int compresskv_workspace_init(void* workspace, size_t workspace_bytes, void* stream) {
+  if (!workspace || workspace_bytes < kStatusBytes) return CKV_ERR_WORKSPACE;
+  return cudaMemsetAsync(workspace, 0, kStatusBytes, static_cast<cudaStream_t>(stream)) ==
+                 cudaSuccess
+             ? CKV_OK
+             : CKV_ERR_CUDA;
+}
+
+int compresskv_output_layout(const ckv_problem* p, const int32_t* budgets, int32_t* cu_prefix,
+                             int32_t* cu_out) {
+  Info I;
+  int rc = validate(p, I);
+  if (rc != CKV_OK) return rc;
+  if (cu_prefix) std::copy(I.cu_prefix.begin(), I.cu_prefix.end(), cu_prefix);
+  if (cu_out) {
+    std::vector<int> co;
+    if ((rc = output_layout(I, budgets, co)) != CKV_OK) return rc;
+    std::copy(co.begin(), co.end(), cu_out);
+  }
+  return CKV_OK;
+}
+
+int compresskv_score(const ckv_problem* p, const void* q_win, const void* k,
+                     const uint8_t* srh_mask, float* raw_scores, void* workspace,
+                     size_t workspace_bytes, void* stream) {
+  Info I;
+  int rc = validate(p, I);
+  if (rc != CKV_OK) return rc;
+  Workspace ws;
+  if ((rc = carve(I, workspace, workspace_bytes, ws)) != CKV_OK) return rc;
+  return run_score(p, I, q_win, k, srh_mask, raw_scores, ws, static_cast<cudaStream_t>(stream));
+}
+
+int compresskv_select(const ckv_problem* p, const float* raw_scores, const int32_t* budgets,
+                      int32_t* indices, int32_t* cu_out, float* pooled_scores, void* workspace,
+                      size_t workspace_bytes, void* stream) {
+  Info I;
+  int rc = validate(p, I);
+  if (rc != CKV_OK) return rc;
+  std::vector<int> co;
+  if ((rc = output_layout(I, budgets, co)) != CKV_OK) return rc;
+  if (!cu_out) return CKV_ERR_INVALID_ARG;
+  Workspace ws;
+  if ((rc = carve(I, workspace, workspace_bytes, ws)) != CKV_OK) return rc;
+  std::copy(co.begin(), co.end(), cu_out);
+  return run_select(p, I, raw_scores, co, indices, pooled_scores, ws,
+                    static_cast<cudaStream_t>(stream));
+}
+
+int compresskv_gather(const ckv_problem* p, const int32_t* indices, const int32_t* cu_out,
+                      const void* k, const void* v, void* k_out, void* v_out, void* workspace,
+                      void* stream) {
+  Info I;
+  int rc = validate(p, I);
+  if (rc != CKV_OK) return rc;
+  if (!cu_out) return CKV_ERR_INVALID_ARG;
+  std::vector<int> co(cu_out, cu_out + I.B + 1);
+  if (co[0] != 0) return CKV_ERR_INVALID_ARG;
+  for (int s = 0; s < I.B; ++s)
+    if (co[s + 1] < co[s] || co[s + 1] - co[s] > I.len[s]) return CKV_ERR_INVALID_ARG;
+  if (static_cast<long long>(I.Hkv) * co[I.B] > (1LL << 31) - 1) return CKV_ERR_UNSUPPORTED;
+  int* status = nullptr;
+  if (workspace) {
+    if (reinterpret_cast<uintptr_t>(workspace) & 255u) return CKV_ERR_WORKSPACE;
+    status = static_cast<int*>(workspace);
+  }
+  return run_gather(p, I, indices, co, k, v, k_out, v_out, status,
+                    static_cast<cudaStream_t>(stream));
+}
+
+int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const void* k,
+                              const void* v, const uint8_t* srh_mask, const int32_t* budgets,
+                              int32_t* indices, int32_t* cu_out, void* k_out, void* v_out,
+                              float* raw_scores, float* pooled_scores, void* workspace,
+                              size_t workspace_bytes, void* stream) {
+  Info I;
+  int rc = validate(p, I);
+  if (rc != CKV_OK) return rc;
+  std::vector<int> co;
+  if ((rc = output_layout(I, budgets, co)) != CKV_OK) return rc;
+  if (!cu_out) return CKV_ERR_INVALID_ARG;
+  Workspace ws;
+  if ((rc = carve(I, workspace, workspace_bytes, ws)) != CKV_OK) return rc;
+  SrhLists S;
+  if ((rc = srh_lists(I, srh_mask, S)) != CKV_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  float* raw = raw_scores ? raw_scores : ws.raw;
+  std::copy(co.begin(), co.end(), cu_out);
+  if ((rc = run_score(p, I, q_win, k, srh_mask, raw, ws, st)) != CKV_OK) return rc;
+  if ((rc = run_select(p, I, raw, co, indices, pooled_scores, ws, st)) != CKV_OK) return rc;
+  return run_gather(p, I, indices, co, k, v, k_out, v_out, ws.status, st);
+}
+
+int compresskv_read_device_status(const void* workspace, void* stream, int32_t* status) {
+  if (!workspace || !status) return CKV_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int32_t v = 0;
+  if (cudaMemcpyAsync(&v, workspace, sizeof(v), cudaMemcpyDeviceToHost, st) != cudaSuccess)
+    return CKV_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return CKV_ERR_CUDA;
+  *status = v;
+  return CKV_OK;
+}
+
+const char* compresskv_status_string(int status) {
+  switch (status) {
+    case CKV_OK: return "ok";
+    case CKV_ERR_INVALID_ARG: return "invalid argument";
+    case CKV_ERR_UNSUPPORTED: return "unsupported problem shape";
+    case CKV_ERR_BUDGET: return "budget smaller than the observation window";
+    case CKV_ERR_EMPTY_SRH_GROUP: return "KV group without an SRH head";
+    case CKV_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    case CKV_ERR_CUDA: return "CUDA runtime error";
+    case CKV_ERR_DEVICE_TIMEOUT: return "device wait timed out";
+    case CKV_ERR_DEVICE_INDEX: return "gather index outside its sequence";
+    default: return "unknown status";
+  }
+}
+
+}  // extern "C"

@@ -1,0 +1,89 @@
+// Kernel parameter blocks shared by the host launcher and the kernels.
+// Parameters travel by value (__grid_constant__), so a launch needs no
+// device-side tables and can be captured into a CUDA graph as is.
+#pragma once
+
+#include <cstdint>
+#include <cuda.h>
+
+namespace ckv {
+
+constexpr int kHeadDim = 128;       // d: one 256-byte K row per token and group (16-bit types)
+constexpr int kTileTokens = 128;    // tokens per K tile = UMMA M = TMEM lanes
+constexpr int kStages = 4;          // K tiles in flight per CTA
+constexpr int kMaxQRows = 256;      // |S_g| * W rows per unit (UMMA N limit)
+constexpr int kMaxBatch = 512;
+constexpr int kMaxQHeads = 256;
+constexpr int kMaxKvHeads = 64;
+constexpr int kMaxItems = 1024;     // score work items per launch
+constexpr int kScoreThreads = 384;  // 12 warps: TMA, MMA, TMEM alloc, spare, 2 x 4 epilogue
+constexpr uint64_t kWaitTimeoutNs = 2000000000ull;  // 2 s: far above any legitimate wait
+
+// Device status codes (mirrors of the public CKV_ERR_* values).
+constexpr int CKV_DEV_ERR_TIMEOUT = -7;
+constexpr int CKV_DEV_ERR_INDEX = -8;
+
+constexpr int kTileBytes = kTileTokens * kHeadDim * 2;   // 32 KiB
+constexpr int kHalfTileBytes = kTileBytes / 2;           // 64 columns (128 B) of d
+constexpr int kQHalfBytes = kMaxQRows * 128;             // Q rows, one 64-column half
+
+// One score work item: a contiguous range of K tiles of one unit.  `first`
+// and `count` locate all items of the same unit in the item table (pass 2
+// merges their partial softmax statistics).
+struct WorkItem {
+  uint16_t seq, group, t0, t1, first, count;
+};
+
+struct ScoreParams {
+  CUtensorMap tmap_k;          // 3-D map over K: (d, kv head, token)
+  const uint16_t* q;           // window queries (f16/bf16 bits)
+  float2* partials;            // [n_items][kMaxQRows]: (max z*c, sum 2^(z*c - max))
+  float* raw;                  // score layout [num_kv_heads][p_total]
+  int* status;                 // device status word
+  long long q_bs, q_hs, q_ws;  // window-query strides, elements
+  float c;                     // scale * log2(e)
+  int window, num_kv_heads, p_total, n_items, is_bf16, use_evict_hint;
+  int q_half_bytes;            // bytes of one 64-column half of the Q rows in shared memory
+  int cu_seqlens[kMaxBatch + 1];
+  int cu_prefix[kMaxBatch + 1];
+  uint16_t srh_off[kMaxKvHeads + 1];   // SRH heads of group g: srh_heads[srh_off[g] .. srh_off[g+1])
+  uint8_t srh_heads[kMaxQHeads];
+  WorkItem items[kMaxItems];
+};
+
+struct SelectParams {
+  const float* raw;            // score layout
+  float* pooled_out;           // optional, score layout
+  float* pooled_ws;            // workspace copy of pooled scores, score layout
+  int32_t* indices;            // [num_kv_heads][o_total]
+  int* status;
+  int window, pool_width, num_kv_heads, p_total, o_total, batch, smem_floats;
+  int cu_seqlens[kMaxBatch + 1];
+  int cu_prefix[kMaxBatch + 1];
+  int cu_out[kMaxBatch + 1];
+};
+
+struct GatherParams {
+  const uint4* k;
+  const uint4* v;
+  uint4* k_out;
+  uint4* v_out;
+  const int32_t* indices;
+  int* status;                 // may be null
+  long long tok_stride_v16, head_stride_v16;  // K/V strides in 16-byte units
+  int num_kv_heads, o_total, batch;
+  int cu_seqlens[kMaxBatch + 1];
+  int cu_out[kMaxBatch + 1];
+};
+
+// Host-side launchers (defined next to each kernel).
+cudaError_t launch_score_stats(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s);
+cudaError_t launch_score_accum(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s);
+cudaError_t launch_select(const SelectParams& p, int n_units, size_t smem, cudaStream_t s);
+cudaError_t launch_gather(const GatherParams& p, long long rows, cudaStream_t s);
+size_t score_smem_bytes(int q_half_bytes);
+cudaError_t score_set_smem_limit(size_t bytes);
+cudaError_t select_set_smem_limit(size_t bytes);
+int select_max_smem_floats();
+
+}  // namespace ckv

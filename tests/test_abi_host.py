@@ -1,0 +1,111 @@
+"""The C ABI library without a GPU: it builds, loads, exports every function
+include/compresskv.h declares, and rejects bad arguments on the host before
+anything is enqueued (these calls make no CUDA call)."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2606_24467_gb300 as ckv
+from paper_2606_24467_gb300 import compresskv as B
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include",
+                      "compresskv.h")
+
+
+def _declared():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"\b(compresskv_\w+)\s*\(", text)))
+
+
+def test_header_and_binding_agree():
+    assert _declared() == sorted(B.EXPORTED)
+
+
+def test_library_loads_and_exports_every_symbol():
+    lib = ckv.load()
+    for name in _declared():
+        assert hasattr(lib, name), name
+    assert ckv.status_string(-3) == "budget smaller than the observation window"
+    assert ckv.status_string(0) == "ok"
+
+
+def _problem(L=(300, 40), Hq=8, Hkv=2, W=32, P=7, dtype=torch.bfloat16, **kw):
+    cu = np.concatenate([[0], np.cumsum(L)]).astype(np.int32)
+    q = torch.zeros((len(L), Hq, W, 128), dtype=dtype)
+    k = torch.zeros((int(cu[-1]), Hkv, 128), dtype=dtype)
+    return ckv.Problem(q, k, cu, W, P, **kw), q, k
+
+
+def test_workspace_size_and_layout():
+    prob, q, k = _problem()
+    n = ckv.workspace_size(prob)
+    assert n >= 2 * 2 * (268 + 8) * 4
+    cu_prefix, cu_out = ckv.output_layout(prob, [100, 100])
+    assert cu_prefix.tolist() == [0, 268, 276]
+    assert cu_out.tolist() == [0, 100, 140]
+
+
+def test_budget_below_window_is_rejected():
+    prob, q, k = _problem()
+    with pytest.raises(ckv.CompressKVError) as e:
+        ckv.output_layout(prob, [31, 100])
+    assert e.value.code == B.CKV_ERR_BUDGET
+
+
+def _fake_dev_ptr(n=1 << 20):
+    # An aligned address that is never dereferenced: every call below fails
+    # validation on the host first.
+    return 1 << 30
+
+
+def test_invalid_shapes_rejected():
+    lib = ckv.load()
+    prob, q, k = _problem()
+    s = prob.struct
+    for field, value, code in (("head_dim", 64, B.CKV_ERR_UNSUPPORTED),
+                               ("pool_width", 4, B.CKV_ERR_INVALID_ARG),
+                               ("window", 0, B.CKV_ERR_INVALID_ARG),
+                               ("num_q_heads", 7, B.CKV_ERR_INVALID_ARG),
+                               ("dtype", 5, B.CKV_ERR_INVALID_ARG),
+                               ("pool_kind", 1, B.CKV_ERR_UNSUPPORTED),
+                               ("kv_token_stride", 100, B.CKV_ERR_INVALID_ARG)):
+        old = getattr(s, field)
+        setattr(s, field, value)
+        assert lib.compresskv_workspace_size(prob.ref) == 0
+        rc = lib.compresskv_output_layout(prob.ref, None, None, None)
+        assert rc == code, (field, rc)
+        setattr(s, field, old)
+
+
+def test_compress_layer_host_errors():
+    lib = ckv.load()
+    prob, q, k = _problem()
+    vp = ctypes.c_void_p
+    ws = vp(_fake_dev_ptr())
+    n = ckv.workspace_size(prob)
+    mask_ok = np.zeros(8, np.uint8)
+    mask_ok[[1, 6]] = 1
+    mask_empty = np.zeros(8, np.uint8)
+    mask_empty[1] = 1  # group 1 (heads 4-7) has no SRH head
+    bud, bp = B._i32([64, 64])
+    cu_out = (ctypes.c_int32 * 3)()
+
+    def call(mask, budgets_ptr=bp, workspace=ws, wsn=n, qptr=vp(1 << 30)):
+        return lib.compresskv_compress_layer(
+            prob.ref, qptr, vp(1 << 30), vp(1 << 30), vp(mask.ctypes.data), budgets_ptr,
+            vp(1 << 30), cu_out, vp(1 << 30), vp(1 << 30), None, None, workspace, wsn, None)
+
+    assert call(mask_empty) == B.CKV_ERR_EMPTY_SRH_GROUP
+    assert call(mask_ok, workspace=vp(None)) == B.CKV_ERR_WORKSPACE
+    assert call(mask_ok, wsn=n - 1) == B.CKV_ERR_WORKSPACE
+    assert call(mask_ok, workspace=vp((1 << 30) + 16)) == B.CKV_ERR_WORKSPACE
+    b2, bp2 = B._i32([64, 10])
+    assert call(mask_ok, budgets_ptr=bp2) == B.CKV_ERR_BUDGET
+    big = np.ones(8, np.uint8)          # 4 heads x W=32 = 128 rows: fine
+    prob.struct.window = 80             # 4 x 80 = 320 rows > 256: unsupported
+    b3, bp3 = B._i32([100, 100])
+    assert call(big, budgets_ptr=bp3) == B.CKV_ERR_UNSUPPORTED

@@ -1,0 +1,201 @@
+"""CUDA path vs. the float64 oracle, through the C ABI (needs a GB300).
+
+Tolerances (spec acceptance, see oracle/compare.py): raw and pooled
+scores within 1e-3 relative + 1e-5 absolute; retained index sets identical
+except for near-ties within 1e-3 of the k-th pooled score; K/V rows
+bit-exact at the device's indices; device results deterministic.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2606_24467_gb300 as ckv
+import workloads as wl
+from oracle import compare
+
+pytestmark = pytest.mark.gpu
+
+
+def _bits(t):
+    return t.detach().cpu().contiguous().view(torch.int16).numpy()
+
+
+def run_gpu(d, window, pool_width, dev, mask=None, scale=0.0, budgets=None, k=None, v=None,
+            q=None):
+    q = d["q_win"].to(dev) if q is None else q
+    k = d["k"].to(dev) if k is None else k
+    v = d["v"].to(dev) if v is None else v
+    mask = d["srh_mask"] if mask is None else mask
+    budgets = d["budgets"] if budgets is None else budgets
+    prob = ckv.Problem(q, k, d["cu_seqlens"], window, pool_width, scale=scale)
+    out = ckv.LayerOutputs(prob, budgets, 128, k.dtype, dev)
+    ws = ckv.workspace(prob, dev)
+    cu_out = ckv.compress_layer(prob, q, k, v, mask, budgets, out.indices, out.k_out, out.v_out,
+                                ws, raw=out.raw, pooled=out.pooled)
+    torch.cuda.synchronize()
+    assert ckv.read_device_status(ws) == 0
+    return out, cu_out
+
+
+def run_oracle(d, window, pool_width, mask=None, scale=None, budgets=None):
+    mask = d["srh_mask"] if mask is None else mask
+    budgets = d["budgets"] if budgets is None else budgets
+    return oracle.compress_layer(d["q_win"].float().numpy(), d["k"].float().numpy(),
+                                 d["v"].float().numpy(), d["cu_seqlens"], mask, budgets,
+                                 window, pool_width, scale=scale)
+
+
+def check(d, window, pool_width, dev, mask=None, budgets=None, scale=None, **kw):
+    out, cu_out = run_gpu(d, window, pool_width, dev, mask=mask, budgets=budgets,
+                          scale=scale or 0.0, **kw)
+    res = run_oracle(d, window, pool_width, mask=mask, budgets=budgets, scale=scale)
+    assert np.array_equal(cu_out, res.cu_out)
+    idx = out.indices.cpu().numpy()
+    ties = compare.check_layer(res, out.raw.cpu().numpy(), out.pooled.cpu().numpy(), idx,
+                               d["cu_seqlens"], window)
+    compare.check_gather_bits(_bits(d["k"]), _bits(d["v"]), _bits(out.k_out), _bits(out.v_out),
+                              idx, d["cu_seqlens"], cu_out)
+    return out, res, ties
+
+
+# ---------------------------------------------------------------------------
+def test_llama8b_4k_single_layer(cuda_device):
+    """The 1-layer L=4096 fp16 workload, in full."""
+    cfg = wl.get("c1")
+    d = wl.make_layer(cfg, 0)
+    _, res, ties = check(d, cfg.window, cfg.pool_width, cuda_device)
+    assert ties <= 2
+
+
+@pytest.mark.parametrize("dtype", ["fp16", "bf16"])
+def test_ragged_batch_edge_lengths(cuda_device, dtype):
+    # lengths around the window and the 128-token tiles, plus an empty sequence
+    lens = [1000, 0, 5, 32, 33, 160, 161, 255, 256, 257, 128 + 32, 1, 700]
+    cfg = wl.get("c1").scaled(dtype=dtype, batch=len(lens), seq_len=0, srh_per_group=(1, 3))
+    bud = np.array([[64, 40, 40, 40, 33, 100, 161, 200, 32, 250, 64, 40, 5000]], np.int32)
+    d = wl.make_layer(cfg, 0, lengths=lens, budgets=bud)
+    check(d, cfg.window, cfg.pool_width, cuda_device)
+
+
+@pytest.mark.parametrize("W,P,heads", [(8, 5, 4), (16, 3, 3), (32, 1, 2), (64, 7, 3), (64, 9, 4),
+                                       (5, 7, 3), (7, 1, 1), (128, 7, 2)])
+def test_window_pool_and_srh_counts(cuda_device, W, P, heads):
+    """Query-row counts |S|*W from 7 to 256 (MMA N padding), pooling widths."""
+    cfg = wl.get("c1").scaled(seq_len=1500, window=W, pool_width=P, srh_per_group=(heads, heads),
+                              dtype="bf16")
+    bud = np.array([[W + 77]], np.int32)
+    d = wl.make_layer(cfg, 0, budgets=bud)
+    check(d, W, P, cuda_device)
+
+
+def test_all_heads_mask_is_snapkv_group_scoring(cuda_device):
+    cfg = wl.get("c1").scaled(seq_len=2500)
+    d = wl.make_layer(cfg, 0)
+    check(d, cfg.window, cfg.pool_width, cuda_device, mask=np.ones(32, bool))
+
+
+def test_budget_extremes(cuda_device):
+    lens = [900, 900, 900, 900, 900]
+    cfg = wl.get("c1").scaled(batch=5, seq_len=900, dtype="bf16")
+    bud = np.array([[32, 33, 899, 900, 4096]], np.int32)  # window only .. keep all
+    d = wl.make_layer(cfg, 0, lengths=lens, budgets=bud)
+    out, res, _ = check(d, cfg.window, cfg.pool_width, cuda_device)
+    assert res.cu_out.tolist() == [0, 32, 65, 964, 1864, 2764]
+
+
+def test_exact_ties_break_to_lower_position(cuda_device):
+    """All keys equal: every interior pooled score ties exactly, so the lowest
+    interior positions must be kept (closed form of the oracle pins)."""
+    cfg = wl.get("c1").scaled(seq_len=600, dtype="bf16")
+    d = wl.make_layer(cfg, 0, sinks=False, needle_gain=0.0)
+    d["k"][:] = d["k"][0:1]
+    out, res, ties = check(d, cfg.window, cfg.pool_width, cuda_device)
+    assert ties == 0
+    r = (cfg.pool_width - 1) // 2
+    k = 128 - cfg.window
+    idx = out.indices.cpu().numpy()
+    for g in range(8):
+        assert idx[g, :k].tolist() == list(range(r, r + k))
+
+
+def test_strided_inputs(cuda_device):
+    """K and V as views of one packed KV tensor; Q as a slice of a larger window."""
+    cfg = wl.get("c1").scaled(seq_len=777, dtype="bf16", srh_per_group=(2, 2))
+    d = wl.make_layer(cfg, 0)
+    T = d["k"].shape[0]
+    kv = torch.empty((T, 2, 8, 128), dtype=torch.bfloat16, device=cuda_device)
+    kv[:, 0] = d["k"].to(cuda_device)
+    kv[:, 1] = d["v"].to(cuda_device)
+    qbig = torch.zeros((1, 32, 48, 128), dtype=torch.bfloat16, device=cuda_device)
+    qbig[:, :, 16:] = d["q_win"].to(cuda_device)
+    check(d, cfg.window, cfg.pool_width, cuda_device, k=kv[:, 0], v=kv[:, 1],
+          q=qbig[:, :, 16:])
+
+
+def test_explicit_scale(cuda_device):
+    cfg = wl.get("c1").scaled(seq_len=1200, dtype="bf16")
+    d = wl.make_layer(cfg, 0)
+    check(d, cfg.window, cfg.pool_width, cuda_device, scale=0.5)
+
+
+def test_stage_entry_points_match_fused(cuda_device):
+    cfg = wl.get("c1").scaled(seq_len=3000, dtype="bf16", batch=2, srh_per_group=(1, 2))
+    d = wl.make_layer(cfg, 0, lengths=[3000, 1700],
+                      budgets=np.array([[300, 150]], np.int32))
+    dev = cuda_device
+    q, k, v = d["q_win"].to(dev), d["k"].to(dev), d["v"].to(dev)
+    fused, cu_fused = run_gpu(d, cfg.window, cfg.pool_width, dev)
+    prob = ckv.Problem(q, k, d["cu_seqlens"], cfg.window, cfg.pool_width)
+    out = ckv.LayerOutputs(prob, d["budgets"], 128, k.dtype, dev)
+    ws = ckv.workspace(prob, dev)
+    ckv.score(prob, q, k, d["srh_mask"], out.raw, ws)
+    cu_out = ckv.select(prob, out.raw, d["budgets"], out.indices, ws, pooled=out.pooled)
+    ckv.gather(prob, out.indices, cu_out, k, v, out.k_out, out.v_out, ws)
+    torch.cuda.synchronize()
+    assert np.array_equal(cu_out, cu_fused)
+    for a, b in ((out.raw, fused.raw), (out.pooled, fused.pooled), (out.indices, fused.indices)):
+        assert torch.equal(a, b)
+    assert torch.equal(out.k_out.view(torch.int16), fused.k_out.view(torch.int16))
+    assert torch.equal(out.v_out.view(torch.int16), fused.v_out.view(torch.int16))
+
+
+def test_deterministic(cuda_device):
+    cfg = wl.get("c1").scaled(seq_len=5000, dtype="bf16", srh_per_group=(1, 2))
+    d = wl.make_layer(cfg, 0)
+    a, _ = run_gpu(d, cfg.window, cfg.pool_width, cuda_device)
+    b, _ = run_gpu(d, cfg.window, cfg.pool_width, cuda_device)
+    assert torch.equal(a.raw.view(torch.int32), b.raw.view(torch.int32))
+    assert torch.equal(a.indices, b.indices)
+
+
+def test_gather_reports_bad_index(cuda_device):
+    cfg = wl.get("c1").scaled(seq_len=300, dtype="bf16")
+    d = wl.make_layer(cfg, 0)
+    dev = cuda_device
+    k, v = d["k"].to(dev), d["v"].to(dev)
+    prob = ckv.Problem(d["q_win"].to(dev), k, d["cu_seqlens"], cfg.window, cfg.pool_width)
+    ws = ckv.workspace(prob, dev)
+    cu_out = np.array([0, 10], np.int32)
+    idx = torch.arange(10, dtype=torch.int32, device=dev).repeat(8, 1).contiguous()
+    idx[3, 4] = 300  # one past the end of the sequence
+    k_out = torch.zeros((10, 8, 128), dtype=k.dtype, device=dev)
+    v_out = torch.zeros_like(k_out)
+    ckv.gather(prob, idx, cu_out, k, v, k_out, v_out, ws)
+    assert ckv.read_device_status(ws) == ckv.compresskv.CKV_ERR_DEVICE_INDEX
+    assert torch.equal(k_out[4, 3], torch.zeros_like(k_out[4, 3]))
+    assert torch.equal(k_out[5, 3], k[5, 3])
+
+
+# ---------------------------------------------------------------------------
+# full-size layers of the benchmark workloads (every unit of a sampled layer)
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("name,layer", [("c2", 5), ("c3", 17), ("c4", 3), ("c5", 40)])
+def test_full_size_layer(cuda_device, name, layer):
+    cfg = wl.get(name)
+    d = wl.make_layer(cfg, layer)
+    _, res, ties = check(d, cfg.window, cfg.pool_width, cuda_device)
+    n_units = len(res.units)
+    assert ties <= max(4, n_units)
