@@ -1,0 +1,507 @@
+#!/usr/bin/env python3
+"""Throughput of the CompressKV prefill-end compression path on GB300.
+
+One step = every layer of the workload compressed once (scoring with the SRH
+heads, pooling, budgeted top-k, K/V gather), inputs resident in HBM.  The
+default workload is 32 layers of a Llama-3.1-8B GQA shape at L = 32768
+(bf16, W = 32, P = 7, budgets with mean 256).  Prints one JSON line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...     # the float64 oracle on host cores
+
+Multi-GPU (torchrun, one process per GPU): every rank compresses its own
+replica of the workload (the path has no exchange step); value = tokens of
+all ranks / slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+import workloads as wl  # noqa: E402
+
+METRIC = ("prompt tokens compressed/sec per GB300 and achieved HBM GB/s vs peak at "
+          "L=32K–128K")
+UNIT = "tokens/s"
+PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "score_stats_llama8b_L32k.md")
+KERNEL_SOURCES = ["paper_2606_24467_gb300/csrc/score_kernel.cu",
+                  "paper_2606_24467_gb300/csrc/ckv_device.cuh",
+                  "paper_2606_24467_gb300/csrc/ckv_params.h",
+                  "paper_2606_24467_gb300/csrc/api.cu"]
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--workload", default="c2")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="compress only the first N layers (small profiling runs)")
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+# --------------------------------------------------------------------- distributed
+def dist_env():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)),
+            int(os.environ.get("LOCAL_RANK", 0)))
+
+
+def init_dist(world: int, backend: str):
+    if world <= 1:
+        return None
+    import torch.distributed as dist
+
+    os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+    dist.init_process_group(backend=backend)
+    return dist
+
+
+def reduce_max(dist, value: float, device) -> float:
+    """Max of a float over ranks (identity without a process group)."""
+    if dist is None:
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(dist):
+    if dist is not None:
+        dist.barrier()
+
+
+# --------------------------------------------------------------------- clocks
+_CLOCK_FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                 "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                 "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+_REASON_NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+
+class ClockSampler:
+    """nvidia-smi sampling (read-only) while the timed region runs."""
+
+    def __init__(self, device):
+        self.proc = None
+        self.lines = []
+        ident = []
+        try:
+            uuid = str(torch.cuda.get_device_properties(device).uuid)
+            ident = [f"--id=GPU-{uuid}" if not uuid.startswith("GPU-") else f"--id={uuid}"]
+        except Exception:
+            ident = []
+        self.cmd = ["nvidia-smi", *ident, f"--query-gpu={_CLOCK_FIELDS}",
+                    "--format=csv,noheader,nounits", "-lms", "100"]
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(self.cmd, stdout=subprocess.PIPE,
+                                         stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.25)
+
+    def stop(self) -> dict | None:
+        if self.proc is None:
+            return None
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        for line in out.strip().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for name, val in zip(_REASON_NAMES, parts[4:8]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------------- helpers
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for rel in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload: str):
+    """DRAM bytes per launch of the pass-1 scoring kernel from the committed
+    ncu summary, if it was taken on the current kernel sources."""
+    try:
+        text = open(PROFILE_TRAFFIC).read()
+    except OSError:
+        return None
+    m = re.search(r"traffic_bytes_per_launch:\s*(\d+)", text)
+    h = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", text)
+    w = re.search(r"workload:\s*(\S+)", text)
+    if not (m and h and w) or h.group(1) != kernel_source_hash() or w.group(1) != workload:
+        return None
+    return int(m.group(1))
+
+
+def cpu_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def build_layers(cfg, device):
+    lengths = wl.sequence_lengths(cfg)
+    masks = wl.srh_masks(cfg)
+    budgets = wl.layer_budgets(cfg, lengths)
+    layers = [wl.make_layer(cfg, l, device=device, lengths=lengths, masks=masks, budgets=budgets)
+              for l in range(cfg.n_layers)]
+    return lengths, masks, budgets, layers
+
+
+def algorithmic_bytes(cfg, layers, lengths):
+    """K read once for scoring + retained K and V read and written, per step,
+    plus the window-query rows of the SRH heads."""
+    d = cfg.head_dim
+    esz = 2
+    k_bytes = sum(lengths) * cfg.num_kv_heads * d * esz
+    total = 0
+    score_bytes = 0
+    for lay in layers:
+        kept = sum(min(int(b), L) for b, L in zip(lay["budgets"], lengths))
+        q_rows = int(lay["srh_mask"].sum()) * cfg.window * cfg.batch
+        score_bytes += k_bytes + q_rows * d * esz
+        total += k_bytes + q_rows * d * esz + 4 * kept * cfg.num_kv_heads * d * esz
+    return total, score_bytes
+
+
+# --------------------------------------------------------------------- our arm
+def run_ours(args):
+    import paper_2606_24467_gb300 as ckv
+
+    rank, world, local_rank = dist_env()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    dist = init_dist(world, "nccl")
+    cfg = wl.get(args.workload)
+    if args.layers:
+        cfg = cfg.scaled(n_layers=args.layers)
+    ckv.load(build_if_missing=(rank == 0 and world == 1))
+    lengths, masks, budgets, layers = build_layers(cfg, dev)
+    tokens = sum(lengths)
+
+    # library objects: one problem per layer, a shared workspace, per-layer outputs
+    trace = ckv.Trace(capacity=16 * cfg.n_layers)
+    probs = [ckv.Problem(lay["q_win"], lay["k"], lay["cu_seqlens"], cfg.window, cfg.pool_width,
+                         trace=trace) for lay in layers]
+    ws = ckv.workspace(probs[0], dev)
+    outs = [ckv.LayerOutputs(probs[l], budgets[l], cfg.head_dim, layers[l]["k"].dtype, dev,
+                             scores=False) for l in range(cfg.n_layers)]
+
+    def step():
+        for l, lay in enumerate(layers):
+            o = outs[l]
+            ckv.compress_layer(probs[l], lay["q_win"], lay["k"], lay["v"], lay["srh_mask"],
+                               lay["budgets"], o.indices, o.k_out, o.v_out, ws)
+
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        for _ in range(2):
+            step()
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    trace.reset()
+    with torch.cuda.graph(graph, capture_error_mode="thread_local"):
+        step()
+    launches_per_step = trace.launches
+    torch.cuda.synchronize()
+
+    for _ in range(max(args.warmup, 3)):
+        graph.replay()
+    torch.cuda.synchronize()
+    barrier(dist)
+    sampler = ClockSampler(dev)
+    sampler.start()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    barrier(dist)
+    t0.record()
+    for _ in range(args.steps):
+        graph.replay()
+    t1.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    barrier(dist)
+    elapsed_ms = reduce_max(dist, t0.elapsed_time(t1), dev)
+    ms_per_step = elapsed_ms / args.steps
+    value = world * tokens * args.steps / (elapsed_ms / 1e3)
+    assert ckv.read_device_status(ws) == 0, "device status set during the bench"
+
+    # per-kernel durations: the trace events of the last timed replay
+    per_kind: dict[str, list[float]] = {}
+    for kind, ms in trace.records():
+        per_kind.setdefault(kind, []).append(ms)
+    step_bytes, score_bytes = algorithmic_bytes(cfg, layers, lengths)
+    peak, peak_src = measured_peaks()
+    stats_ms = per_kind.get("score_stats", [float("nan")])
+    n_stats = len(stats_ms)
+    avg_stats_ms = sum(stats_ms) / max(n_stats, 1)
+    bytes_per_launch = score_bytes / max(n_stats, 1)
+    achieved = bytes_per_launch / (avg_stats_ms / 1e3) / 1e9
+    roofline = {"bound": "hbm", "kernel": "score_stats (pass 1)", "achieved": round(achieved, 1),
+                "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4),
+                "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
+                else "fallback 6.8 TB/s",
+                "bytes_per_launch": int(bytes_per_launch), "launches_per_step": n_stats,
+                "avg_launch_us": round(avg_stats_ms * 1e3, 2),
+                "traffic": profiled_traffic(cfg.name)}
+    path_gbs = step_bytes / (ms_per_step / 1e3) / 1e9
+    kernels = {k: {"launches_per_step": len(v), "avg_us": round(1e3 * sum(v) / len(v), 2),
+                   "total_us_per_step": round(1e3 * sum(v), 1)} for k, v in per_kind.items()}
+
+    result = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": round(ms_per_step, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded generator: Gaussian Q/K/V, sinks, planted needles)",
+        "config": {"workload": cfg.name, "layers": cfg.n_layers, "batch": cfg.batch,
+                   "seq_len": cfg.seq_len if cfg.length_range is None else "ragged",
+                   "q_heads": cfg.num_q_heads, "kv_heads": cfg.num_kv_heads,
+                   "head_dim": cfg.head_dim, "window": cfg.window, "pool_width": cfg.pool_width,
+                   "mean_budget": float(np.mean(budgets)),
+                   "l2": f"inputs larger than L2: {sum(l['k'].numel() * 2 * 2 for l in layers) / 1e9:.2f} GB "
+                         "of K/V per step, each layer's K read cold; no flush",
+                   "cuda_graph": True, "parallelism": f"replicas x{world}",
+                   "l2_bytes": torch.cuda.get_device_properties(dev).L2_cache_size,
+                   "sms": torch.cuda.get_device_properties(dev).multi_processor_count},
+        "roofline": roofline,
+        "path": {"algorithmic_bytes_per_step": step_bytes, "achieved_gbs": round(path_gbs, 1),
+                 "frac_of_peak": round(path_gbs / peak, 4),
+                 "frac_of_8tbs_nominal": round(path_gbs / 8000.0, 4),
+                 "layer_tokens_per_s": round(value * cfg.n_layers, 1)},
+        "kernels": kernels,
+        "gpu_launches": int(launches_per_step * args.steps),
+        "clocks": clocks,
+    }
+
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"], result["parity_layer0"] = cpu_baseline(cfg, layers[0], outs[0])
+    if not args.no_e2e:
+        result["e2e"] = run_e2e(args, cfg, layers, probs, ws, dev, dist, world)
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+def cpu_baseline(cfg, layer, out):
+    """The float64 oracle, as it stands, on one layer (every unit) of the same
+    workload; extrapolated to all layers.  Also checks that layer's device
+    result against the oracle."""
+    import oracle
+    from oracle import compare
+
+    q = layer["q_win"].float().cpu().numpy()
+    k = layer["k"].float().cpu().numpy()
+    v = layer["v"].float().cpu().numpy()
+    t = time.perf_counter()
+    res = oracle.compress_layer(q, k, v, layer["cu_seqlens"], layer["srh_mask"],
+                                layer["budgets"], cfg.window, cfg.pool_width)
+    dt = time.perf_counter() - t
+    tokens = int(layer["cu_seqlens"][-1])
+    value = tokens / (dt * cfg.n_layers)
+    parity = "ok"
+    try:
+        idx = out.indices.cpu().numpy()
+        ties = 0
+        for (s, g), unit in res.units.items():
+            L = int(layer["cu_seqlens"][s + 1] - layer["cu_seqlens"][s])
+            o0, o1 = int(res.cu_out[s]), int(res.cu_out[s + 1])
+            ties += compare.check_unit_indices(idx[g, o0:o1], unit, L, cfg.window)
+        parity = f"ok ({ties} near-tie differences)"
+    except AssertionError as e:
+        parity = f"FAILED: {e}"
+    base = {"value": round(value, 2), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+            "sample": f"layer 0 of {cfg.n_layers} ({len(res.units)} units, {tokens} tokens) in "
+                      f"{dt:.2f} s, extrapolated x{cfg.n_layers} layers; numpy float64 "
+                      "(BLAS threads for q.k^T, one core for the rest)"}
+    return base, parity
+
+
+def run_e2e(args, cfg, layers, probs, ws, dev, dist, world):
+    """The same metric through the public API with host buffers: every step
+    copies each layer's Q window, K and V from pinned host memory, compresses
+    it and reads the compressed cache and indices back.  Copies of layer l+1
+    overlap the compression of layer l (two device slots, copy stream)."""
+    import paper_2606_24467_gb300 as ckv
+
+    host = []
+    for lay in layers:
+        host.append({k: lay[k].cpu().pin_memory() for k in ("q_win", "k", "v")})
+    slots = [{k: torch.empty_like(layers[0][k]) for k in ("q_win", "k", "v")} for _ in range(2)]
+    outs_h, outs_d = [], []
+    for l, lay in enumerate(layers):
+        o = ckv.LayerOutputs(probs[l], lay["budgets"], cfg.head_dim, lay["k"].dtype, dev,
+                             scores=False)
+        outs_d.append(o)
+        outs_h.append({"indices": torch.empty(o.indices.shape, dtype=o.indices.dtype, pin_memory=True),
+                       "k_out": torch.empty(o.k_out.shape, dtype=o.k_out.dtype, pin_memory=True),
+                       "v_out": torch.empty(o.v_out.shape, dtype=o.v_out.dtype, pin_memory=True)})
+    h2d = sum(t.numel() * t.element_size() for h in host for t in h.values())
+    d2h = sum(t.numel() * t.element_size() for h in outs_h for t in h.values())
+    comp = torch.cuda.current_stream()
+    copy = torch.cuda.Stream()
+    # Problems built on the slot tensors (same shapes/strides as the resident ones)
+    sprobs = [[ckv.Problem(slots[i]["q_win"], slots[i]["k"], lay["cu_seqlens"], cfg.window,
+                           cfg.pool_width) for i in range(2)] for lay in layers]
+
+    def step():
+        done = [torch.cuda.Event() for _ in range(2)]
+        ready = [torch.cuda.Event() for _ in range(len(layers))]
+        for l in range(len(layers) + 1):
+            if l < len(layers):
+                i = l % 2
+                with torch.cuda.stream(copy):
+                    if l >= 2:
+                        copy.wait_event(done[i])
+                    for key in ("q_win", "k", "v"):
+                        slots[i][key].copy_(host[l][key], non_blocking=True)
+                    ready[l].record(copy)
+            if l >= 1:
+                j = l - 1
+                i = j % 2
+                comp.wait_event(ready[j])
+                o = outs_d[j]
+                ckv.compress_layer(sprobs[j][i], slots[i]["q_win"], slots[i]["k"], slots[i]["v"],
+                                   layers[j]["srh_mask"], layers[j]["budgets"], o.indices,
+                                   o.k_out, o.v_out, ws, stream=comp)
+                done[i].record(comp)
+                for key in ("indices", "k_out", "v_out"):
+                    outs_h[j][key].copy_(getattr(o, key), non_blocking=True)
+        comp.synchronize()
+
+    step()
+    torch.cuda.synchronize()
+    barrier(dist)
+    t = time.perf_counter()
+    for _ in range(args.e2e_steps):
+        step()
+    torch.cuda.synchronize()
+    el = reduce_max(dist, time.perf_counter() - t, dev)
+    tokens = sum(int(lay["cu_seqlens"][-1]) for lay in layers[:1])
+    return {"value": round(world * tokens * args.e2e_steps / el, 1), "unit": UNIT,
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "steps": args.e2e_steps, "ms_per_step": round(1e3 * el / args.e2e_steps, 3),
+            "note": "pinned host buffers, copies overlapped with compression on a second stream"}
+
+
+# --------------------------------------------------------------------- reference arm
+def run_reference(args):
+    """The float64 oracle on the host cores, as it stands: each step is one
+    unit (sequence x KV group) of layer 0 of the workload, extrapolated to the
+    whole workload (all units of all layers)."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    import oracle
+
+    cfg = wl.get(args.workload)
+    lengths = wl.sequence_lengths(cfg)
+    masks = wl.srh_masks(cfg)
+    budgets = wl.layer_budgets(cfg, lengths)
+    lay = wl.make_layer(cfg, 0, lengths=lengths, masks=masks, budgets=budgets)
+    q = lay["q_win"].float().numpy()
+    k = lay["k"].float().numpy()
+    G = cfg.group_size
+    cu = lay["cu_seqlens"]
+    units = [(s, g) for s in range(cfg.batch) for g in range(cfg.num_kv_heads)]
+
+    def one(i):
+        s, g = units[i % len(units)]
+        heads = oracle.srh_heads(lay["srh_mask"], g, G)
+        return oracle.compress_unit(q[s, heads], k[cu[s]:cu[s + 1], g], cfg.window,
+                                    cfg.pool_width, int(lay["budgets"][s]),
+                                    oracle.default_scale(cfg.head_dim))
+
+    for i in range(max(args.warmup, 1)):
+        one(i)
+    times = []
+    for i in range(args.steps):
+        t = time.perf_counter()
+        one(i)
+        times.append(time.perf_counter() - t)
+    per_unit = statistics.mean(times)
+    tokens = sum(lengths)
+    n_units_total = len(units) * cfg.n_layers
+    value = tokens / (per_unit * n_units_total)
+    step_ms = per_unit * n_units_total * 1e3
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": UNIT,
+        "n_gpus": world, "steps": args.steps, "warmup": max(args.warmup, 1),
+        "ms_per_step": round(step_ms, 1), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic (same seeded generator)",
+        "config": {"workload": cfg.name, "layers": cfg.n_layers, "batch": cfg.batch,
+                   "window": cfg.window, "pool_width": cfg.pool_width},
+        "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": cpu_cores(),
+                         "kind": "oracle",
+                         "sample": f"each step = 1 unit (1 sequence x 1 KV group, L={lengths[0]}) "
+                                   f"of layer 0, mean {per_unit:.3f} s, extrapolated to "
+                                   f"{n_units_total} units"},
+        "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

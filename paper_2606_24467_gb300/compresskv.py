@@ -175,6 +175,9 @@ class Trace:
 
     def __init__(self, capacity: int):
         self.events = [torch.cuda.Event(enable_timing=True) for _ in range(2 * capacity)]
+        for e in self.events:  # torch creates the CUDA event on its first record
+            e.record()
+        torch.cuda.synchronize()
         self._ev = (c_void_p * (2 * capacity))(*[e.cuda_event for e in self.events])
         self._kinds = (c_int32 * capacity)()
         self.struct = CkvTrace(ctypes.cast(self._ev, POINTER(c_void_p)),

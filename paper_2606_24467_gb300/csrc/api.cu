@@ -20,6 +20,12 @@ using namespace ckv;
 namespace {
 
 constexpr size_t kStatusBytes = 256;
+// Share of the L2 that the K of the units scored together may occupy, so
+// that pass 2 finds K in L2.
+#ifndef CKV_L2_SET_FRACTION
+#define CKV_L2_SET_FRACTION 0.6
+#endif
+constexpr double kL2SetFraction = CKV_L2_SET_FRACTION;
 constexpr size_t kPartialBytes = static_cast<size_t>(kMaxItems) * kMaxQRows * sizeof(float2);
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
@@ -163,33 +169,56 @@ int carve(const Info& I, void* ws, size_t bytes, Workspace& out) {
 }
 
 // ------------------------------------------------------------------ tracing
+// Records the caller's trace events around each launch.  A failed record
+// (for example a null event handle) is reported as CKV_ERR_INVALID_ARG and
+// the runtime's last-error state is cleared.
 struct Tracer {
   ckv_trace* t;
   cudaStream_t s;
   int slot = -1;
-  void begin(int kind) {
+  int begin(int kind) {
     slot = -1;
-    if (!t) return;
+    if (!t) return CKV_OK;
     if (t->count < t->capacity && t->events) {
       slot = t->count++;
       if (t->kinds) t->kinds[slot] = kind;
-      record(static_cast<cudaEvent_t>(t->events[2 * slot]));
+      return record(static_cast<cudaEvent_t>(t->events[2 * slot]));
     }
+    return CKV_OK;
   }
-  void end() {
-    if (!t) return;
+  int end() {
+    if (!t) return CKV_OK;
     ++t->launches;
-    if (slot >= 0) record(static_cast<cudaEvent_t>(t->events[2 * slot + 1]));
+    if (slot >= 0) return record(static_cast<cudaEvent_t>(t->events[2 * slot + 1]));
+    return CKV_OK;
   }
-  void record(cudaEvent_t e) {
+  int record(cudaEvent_t e) {
+    if (!e) return CKV_ERR_INVALID_ARG;
     cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
-    cudaStreamIsCapturing(s, &cs);
-    if (cs == cudaStreamCaptureStatusActive)
-      cudaEventRecordWithFlags(e, s, cudaEventRecordExternal);
-    else
-      cudaEventRecord(e, s);
+    cudaError_t err = cudaStreamIsCapturing(s, &cs);
+    if (err == cudaSuccess) {
+      err = cs == cudaStreamCaptureStatusActive
+                ? cudaEventRecordWithFlags(e, s, cudaEventRecordExternal)
+                : cudaEventRecord(e, s);
+    }
+    if (err != cudaSuccess) {
+      cudaGetLastError();
+      return CKV_ERR_INVALID_ARG;
+    }
+    return CKV_OK;
   }
 };
+
+// Launch `fn` bracketed by the trace: trace errors win over a clean launch.
+template <class F>
+int traced(Tracer& tr, int kind, F&& fn) {
+  int rc = tr.begin(kind);
+  if (rc != CKV_OK) return rc;
+  const cudaError_t e = fn();
+  const int rc2 = tr.end();
+  if (e != cudaSuccess) return CKV_ERR_CUDA;
+  return rc2;
+}
 
 // ------------------------------------------------------------------ scoring
 struct SrhLists {
@@ -274,7 +303,8 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
     if (I.n[s] > 0)
       for (int g = 0; g < I.Hkv; ++g)
         units.push_back({s, g, (I.len[s] + kTileTokens - 1) / kTileTokens});
-  const long long set_budget = std::max<long long>(F->l2_bytes / 2, 1LL << 20);
+  const long long set_budget =
+      std::max<long long>(static_cast<long long>(F->l2_bytes * kL2SetFraction), 1LL << 20);
   size_t u0 = 0;
   Tracer tr{p->trace, stream};
   while (u0 < units.size()) {
@@ -313,14 +343,12 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
     P.n_items = n_items;
     P.q_half_bytes = ((max_rows * 128) + 1023) & ~1023;
     const size_t smem = score_smem_bytes(P.q_half_bytes);
-    tr.begin(CKV_KERNEL_SCORE_STATS);
-    cudaError_t e = launch_score_stats(P, n_items, smem, stream);
-    tr.end();
-    if (e != cudaSuccess) return CKV_ERR_CUDA;
-    tr.begin(CKV_KERNEL_SCORE_ACCUM);
-    e = launch_score_accum(P, n_items, smem, stream);
-    tr.end();
-    if (e != cudaSuccess) return CKV_ERR_CUDA;
+    rc = traced(tr, CKV_KERNEL_SCORE_STATS,
+                [&] { return launch_score_stats(P, n_items, smem, stream); });
+    if (rc != CKV_OK) return rc;
+    rc = traced(tr, CKV_KERNEL_SCORE_ACCUM,
+                [&] { return launch_score_accum(P, n_items, smem, stream); });
+    if (rc != CKV_OK) return rc;
     u0 = u1;
   }
   return CKV_OK;
@@ -357,10 +385,9 @@ int run_select(const ckv_problem* p, const Info& I, const float* raw, const std:
   }
   P.smem_floats = std::min(max_n, select_max_smem_floats());
   Tracer tr{p->trace, stream};
-  tr.begin(CKV_KERNEL_SELECT);
-  cudaError_t e = launch_select(P, I.B * I.Hkv, static_cast<size_t>(P.smem_floats) * 4, stream);
-  tr.end();
-  return e == cudaSuccess ? CKV_OK : CKV_ERR_CUDA;
+  return traced(tr, CKV_KERNEL_SELECT, [&] {
+    return launch_select(P, I.B * I.Hkv, static_cast<size_t>(P.smem_floats) * 4, stream);
+  });
 }
 
 int run_gather(const ckv_problem* p, const Info& I, const int32_t* indices,
@@ -389,10 +416,7 @@ int run_gather(const ckv_problem* p, const Info& I, const int32_t* indices,
     P.cu_out[s] = cu_out[s];
   }
   Tracer tr{p->trace, stream};
-  tr.begin(CKV_KERNEL_GATHER);
-  cudaError_t e = launch_gather(P, rows, stream);
-  tr.end();
-  return e == cudaSuccess ? CKV_OK : CKV_ERR_CUDA;
+  return traced(tr, CKV_KERNEL_GATHER, [&] { return launch_gather(P, rows, stream); });
 }
 
 }  // namespace
