@@ -75,8 +75,14 @@ enum {
   CKV_ERR_WORKSPACE = -5,       /* workspace null or smaller than compresskv_workspace_size */
   CKV_ERR_CUDA = -6,            /* a CUDA runtime call or kernel launch failed */
   CKV_ERR_DEVICE_TIMEOUT = -7,  /* a kernel's bounded wait ran out (device status only) */
-  CKV_ERR_DEVICE_INDEX = -8     /* compresskv_gather got an index outside its sequence */
+  CKV_ERR_DEVICE_INDEX = -8,    /* compresskv_gather got an index outside its sequence */
+  CKV_ERR_STATIC_SCRATCH = -9   /* problem needs more than CKV_STATIC_SCRATCH_BYTES of scratch */
 };
+
+/* Size of the scratch built into the library for
+ * compresskv_compress_layer_noalloc (every GPU that loads the library holds
+ * it until the process exits). */
+#define CKV_STATIC_SCRATCH_BYTES (16u * 1024u * 1024u)
 
 enum { CKV_DTYPE_F16 = 0, CKV_DTYPE_BF16 = 1 };
 enum { CKV_POOL_AVG = 0 };
@@ -176,6 +182,30 @@ int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const voi
                               int32_t* indices, int32_t* cu_out, void* k_out, void* v_out,
                               float* raw_scores, float* pooled_scores,
                               void* workspace, size_t workspace_bytes, void* stream);
+
+/* compresskv_compress_layer for callers that cannot allocate device memory
+ * (the paper has no counterpart; this is a deployment convenience).  Some
+ * hosts own every byte of device memory and give a plugin no allocator (an
+ * inference engine that pre-reserves HBM for its KV cache), and some callers
+ * run where cudaMalloc is not allowed or would stall the device.  They pass
+ * inputs and outputs exactly as for compresskv_compress_layer, but no
+ * workspace: the scratch is a static device array of CKV_STATIC_SCRATCH_BYTES
+ * inside the library, and this call allocates nothing.
+ * - A problem whose compresskv_workspace_size exceeds CKV_STATIC_SCRATCH_BYTES
+ *   is rejected with CKV_ERR_STATIC_SCRATCH before anything is enqueued.
+ * - The first call on a device looks up the array's device address (with that
+ *   device current); make that first call before any stream capture.
+ * - Every call on a device shares the one array, which keeps the last call's
+ *   contents: calls whose work may overlap on the GPU (different streams,
+ *   different host threads) race and must be serialised by the caller.
+ * - device_status: optional device int32; receives this call's device status
+ *   word (0, or a CKV_ERR_DEVICE_* code) in stream order.  NULL skips it. */
+int compresskv_compress_layer_noalloc(const ckv_problem* p, const void* q_win, const void* k,
+                                      const void* v, const uint8_t* srh_mask,
+                                      const int32_t* budgets, int32_t* indices, int32_t* cu_out,
+                                      void* k_out, void* v_out, float* raw_scores,
+                                      float* pooled_scores, int32_t* device_status,
+                                      void* stream);
 
 /* Synchronise `stream`, copy the workspace status word to *status and return
  * CKV_OK (or CKV_ERR_CUDA if the copy fails). */

@@ -12,6 +12,7 @@ from .compresskv import (  # noqa: F401
     Problem,
     Trace,
     compress_layer,
+    compress_layer_noalloc,
     gather,
     load,
     output_layout,

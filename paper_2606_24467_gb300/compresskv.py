@@ -25,6 +25,8 @@ CKV_ERR_WORKSPACE = -5
 CKV_ERR_CUDA = -6
 CKV_ERR_DEVICE_TIMEOUT = -7
 CKV_ERR_DEVICE_INDEX = -8
+CKV_ERR_STATIC_SCRATCH = -9
+STATIC_SCRATCH_BYTES = 16 * 1024 * 1024
 CKV_DTYPE_F16 = 0
 CKV_DTYPE_BF16 = 1
 CKV_POOL_AVG = 0
@@ -38,6 +40,7 @@ EXPORTED = (
     "compresskv_select",
     "compresskv_gather",
     "compresskv_compress_layer",
+    "compresskv_compress_layer_noalloc",
     "compresskv_read_device_status",
     "compresskv_status_string",
 )
@@ -93,6 +96,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         "compresskv_gather": (c_int32, [pp, vp, i32p, vp, vp, vp, vp, vp, vp]),
         "compresskv_compress_layer": (c_int32, [pp, vp, vp, vp, vp, i32p, vp, i32p, vp, vp,
                                                  vp, vp, vp, c_size_t, vp]),
+        "compresskv_compress_layer_noalloc": (c_int32, [pp, vp, vp, vp, vp, i32p, vp, i32p, vp,
+                                                         vp, vp, vp, vp, vp]),
         "compresskv_read_device_status": (c_int32, [vp, vp, i32p]),
         "compresskv_status_string": (ctypes.c_char_p, [c_int32]),
     }
@@ -263,6 +268,21 @@ def compress_layer(problem: Problem, q_win, k, v, srh_mask, budgets, indices, k_
         problem.ref, _ptr(q_win), _ptr(k), _ptr(v), mp, bp, _ptr(indices),
         cu_out.ctypes.data_as(POINTER(c_int32)), _ptr(k_out), _ptr(v_out), _ptr(raw),
         _ptr(pooled), _ptr(ws), ws.numel(), _stream(stream)), "compresskv_compress_layer")
+    return cu_out
+
+
+def compress_layer_noalloc(problem: Problem, q_win, k, v, srh_mask, budgets, indices, k_out,
+                           v_out, raw=None, pooled=None, device_status=None,
+                           stream=None) -> np.ndarray:
+    """compress_layer without a workspace: the library's static scratch is
+    used (for callers that cannot allocate device memory)."""
+    m, mp = _mask(srh_mask)
+    b, bp = _i32(budgets)
+    cu_out = np.zeros(problem.batch + 1, np.int32)
+    _check(load().compresskv_compress_layer_noalloc(
+        problem.ref, _ptr(q_win), _ptr(k), _ptr(v), mp, bp, _ptr(indices),
+        cu_out.ctypes.data_as(POINTER(c_int32)), _ptr(k_out), _ptr(v_out), _ptr(raw),
+        _ptr(pooled), _ptr(device_status), _stream(stream)), "compresskv_compress_layer_noalloc")
     return cu_out
 
 

@@ -545,8 +545,65 @@ const char* compresskv_status_string(int status) {
     case CKV_ERR_CUDA: return "CUDA runtime error";
     case CKV_ERR_DEVICE_TIMEOUT: return "device wait timed out";
     case CKV_ERR_DEVICE_INDEX: return "gather index outside its sequence";
+    case CKV_ERR_STATIC_SCRATCH:
+      return "problem needs more scratch than the library's static scratch holds";
     default: return "unknown status";
   }
 }
 
 }  // extern "C"
+
+// ====================================================================== no-alloc variant
+// Scratch for compresskv_compress_layer_noalloc, for callers that cannot
+// allocate device memory.  In host code `g_static_scratch` only names a
+// host-side stand-in, so its device address is looked up once per device.
+static __device__ __align__(256) unsigned char g_static_scratch[CKV_STATIC_SCRATCH_BYTES];
+
+namespace {
+
+std::mutex g_scratch_mutex;
+void* g_scratch_addr[64] = {};
+
+int static_scratch_address(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return CKV_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_scratch_mutex);
+  if (!g_scratch_addr[dev]) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_static_scratch) != cudaSuccess || !ptr) {
+      cudaGetLastError();
+      return CKV_ERR_CUDA;
+    }
+    g_scratch_addr[dev] = ptr;
+  }
+  *out = g_scratch_addr[dev];
+  return CKV_OK;
+}
+
+}  // namespace
+
+extern "C" int compresskv_compress_layer_noalloc(
+    const ckv_problem* p, const void* q_win, const void* k, const void* v,
+    const uint8_t* srh_mask, const int32_t* budgets, int32_t* indices, int32_t* cu_out,
+    void* k_out, void* v_out, float* raw_scores, float* pooled_scores, int32_t* device_status,
+    void* stream) {
+  Info I;
+  int rc = validate(p, I);
+  if (rc != CKV_OK) return rc;
+  if (workspace_bytes(I) > static_cast<size_t>(CKV_STATIC_SCRATCH_BYTES))
+    return CKV_ERR_STATIC_SCRATCH;
+  void* scratch = nullptr;
+  if ((rc = static_scratch_address(&scratch)) != CKV_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // The array keeps the previous call's contents; the status word must start at zero.
+  if (cudaMemsetAsync(scratch, 0, kStatusBytes, st) != cudaSuccess) return CKV_ERR_CUDA;
+  rc = compresskv_compress_layer(p, q_win, k, v, srh_mask, budgets, indices, cu_out, k_out, v_out,
+                                 raw_scores, pooled_scores, scratch,
+                                 static_cast<size_t>(CKV_STATIC_SCRATCH_BYTES), stream);
+  if (rc != CKV_OK) return rc;
+  if (device_status &&
+      cudaMemcpyAsync(device_status, scratch, sizeof(int32_t), cudaMemcpyDeviceToDevice, st) !=
+          cudaSuccess)
+    return CKV_ERR_CUDA;
+  return CKV_OK;
+}
