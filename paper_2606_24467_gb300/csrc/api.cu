@@ -33,6 +33,7 @@ size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 // ------------------------------------------------------------------ device facts
 struct DeviceFacts {
   int sms = 0;
+  int smem_optin = 0;
   long long l2_bytes = 0;
   bool smem_attr_set = false;
 };
@@ -58,8 +59,9 @@ int device_facts(DeviceFacts** out) {
     int optin = 0;
     if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
       return CKV_ERR_CUDA;
+    f.smem_optin = optin;
     if (score_set_smem_limit(static_cast<size_t>(optin)) != cudaSuccess) return CKV_ERR_CUDA;
-    if (select_set_smem_limit(static_cast<size_t>(optin) - 9 * 1024) != cudaSuccess)
+    if (select_set_smem_limit(static_cast<size_t>(select_max_smem_floats()) * 4) != cudaSuccess)
       return CKV_ERR_CUDA;
     f.smem_attr_set = true;
   }
@@ -310,39 +312,60 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
   while (u0 < units.size()) {
     size_t u1 = u0;
     long long bytes = 0;
-    long long tiles = 0;
     while (u1 < units.size()) {
       const long long ub = static_cast<long long>(units[u1].tiles) * kTileBytes;
       if (u1 > u0 && (bytes + ub > set_budget || static_cast<long long>(u1 - u0) >= kMaxItems / 2))
         break;
       bytes += ub;
-      tiles += units[u1].tiles;
       ++u1;
     }
-    // Work items: about one per SM in total, balanced tile ranges per unit.
-    const long long target = std::max(1, F->sms);
-    const long long chunk = std::max<long long>(1, (tiles + target - 1) / target);
+    // Work items: one wave of exactly max(#units, #SMs) CTAs.  A tile of a
+    // unit costs about (64 + query rows) (the epilogue scales with the rows);
+    // every unit gets one item, the remaining items go one at a time to the
+    // unit with the largest work per item, then each unit's tiles are split
+    // into balanced ranges.
+    auto cost = [&](const Unit& U) { return 64LL + ((S.rows[U.g] + 15) & ~15); };
+    const int nu = static_cast<int>(u1 - u0);
+    std::vector<int> cnt(nu, 1);
+    std::vector<long long> uw(nu);
+    for (int u = 0; u < nu; ++u)
+      uw[u] = static_cast<long long>(units[u0 + u].tiles) * cost(units[u0 + u]);
+    const int target = std::min(kMaxItems, std::max(nu, F->sms));
+    for (int extra = target - nu; extra > 0; --extra) {
+      int best = -1;
+      for (int u = 0; u < nu; ++u) {
+        if (cnt[u] >= units[u0 + u].tiles) continue;
+        if (best < 0 || uw[u] * cnt[best] > uw[best] * cnt[u]) best = u;
+      }
+      if (best < 0) break;
+      ++cnt[best];
+    }
     int n_items = 0;
     int max_rows = 16;
-    for (size_t u = u0; u < u1; ++u) {
-      const Unit& U = units[u];
-      const int cnt = static_cast<int>((U.tiles + chunk - 1) / chunk);
-      if (n_items + cnt > kMaxItems) return CKV_ERR_UNSUPPORTED;
-      for (int c = 0; c < cnt; ++c) {
+    for (int u = 0; u < nu; ++u) {
+      const Unit& U = units[u0 + u];
+      const int c_u = cnt[u];
+      if (n_items + c_u > kMaxItems) return CKV_ERR_UNSUPPORTED;
+      for (int c = 0; c < c_u; ++c) {
         WorkItem& it = P.items[n_items + c];
         it.seq = static_cast<uint16_t>(U.s);
         it.group = static_cast<uint16_t>(U.g);
-        it.t0 = static_cast<uint16_t>(static_cast<long long>(U.tiles) * c / cnt);
-        it.t1 = static_cast<uint16_t>(static_cast<long long>(U.tiles) * (c + 1) / cnt);
+        it.t0 = static_cast<uint16_t>(static_cast<long long>(U.tiles) * c / c_u);
+        it.t1 = static_cast<uint16_t>(static_cast<long long>(U.tiles) * (c + 1) / c_u);
         it.first = static_cast<uint16_t>(n_items);
-        it.count = static_cast<uint16_t>(cnt);
+        it.count = static_cast<uint16_t>(c_u);
       }
-      n_items += cnt;
+      n_items += c_u;
       max_rows = std::max(max_rows, (S.rows[U.g] + 15) & ~15);
     }
     P.n_items = n_items;
     P.q_half_bytes = ((max_rows * 128) + 1023) & ~1023;
-    const size_t smem = score_smem_bytes(P.q_half_bytes);
+    P.small_n = max_rows <= 64 ? 1 : 0;
+    P.stages = kStages;
+    while (P.stages > 2 &&
+           score_smem_bytes(P.q_half_bytes, P.stages) > static_cast<size_t>(F->smem_optin))
+      --P.stages;
+    const size_t smem = score_smem_bytes(P.q_half_bytes, P.stages);
     rc = traced(tr, CKV_KERNEL_SCORE_STATS,
                 [&] { return launch_score_stats(P, n_items, smem, stream); });
     if (rc != CKV_OK) return rc;
@@ -356,9 +379,17 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
 
 // ------------------------------------------------------------------ select / gather
 int run_select(const ckv_problem* p, const Info& I, const float* raw, const std::vector<int>& cu_out,
-               int32_t* indices, float* pooled, const Workspace& ws, cudaStream_t stream) {
+               int32_t* indices, float* pooled, const Workspace& ws, cudaStream_t stream,
+               const void* k = nullptr, const void* v = nullptr, void* k_out = nullptr,
+               void* v_out = nullptr) {
   if (!raw && I.p_total > 0) return CKV_ERR_INVALID_ARG;
   if (!indices && cu_out[I.B] > 0) return CKV_ERR_INVALID_ARG;
+  const bool gather = k != nullptr;
+  if (gather && cu_out[I.B] > 0) {
+    if (!v || !k_out || !v_out) return CKV_ERR_INVALID_ARG;
+    if (!aligned16(k) || !aligned16(v) || !aligned16(k_out) || !aligned16(v_out))
+      return CKV_ERR_INVALID_ARG;
+  }
   DeviceFacts* F = nullptr;
   int rc = device_facts(&F);
   if (rc != CKV_OK) return rc;
@@ -370,6 +401,13 @@ int run_select(const ckv_problem* p, const Info& I, const float* raw, const std:
   P.pooled_ws = ws.pooled;
   P.indices = indices;
   P.status = ws.status;
+  P.k = static_cast<const uint4*>(k);
+  P.v = static_cast<const uint4*>(v);
+  P.k_out = static_cast<uint4*>(k_out);
+  P.v_out = static_cast<uint4*>(v_out);
+  P.tok_stride_v16 = p->kv_token_stride / 8;
+  P.head_stride_v16 = p->kv_head_stride / 8;
+  P.gather = gather ? 1 : 0;
   P.window = I.W;
   P.pool_width = I.P;
   P.num_kv_heads = I.Hkv;
@@ -383,11 +421,17 @@ int run_select(const ckv_problem* p, const Info& I, const float* raw, const std:
     P.cu_out[s] = cu_out[s];
     if (s < I.B) max_n = std::max(max_n, I.n[s]);
   }
-  P.smem_floats = std::min(max_n, select_max_smem_floats());
+  // A cluster of up to 8 CTAs per unit, about 4096 prefix tokens per CTA.
+  const int C = std::min(8, std::max(1, (max_n + 4095) / 4096));
+  const int S = std::max(32, ((max_n + C - 1) / C + 31) / 32 * 32);
+  const int r = (I.P - 1) / 2;
+  const bool fits = 2 * S + 2 * r <= select_max_smem_floats();
+  P.cluster = C;
+  P.slice = S;
+  P.smem_slice = fits ? 1 : 0;
+  const size_t smem = fits ? static_cast<size_t>(2 * S + 2 * r) * 4 : 0;
   Tracer tr{p->trace, stream};
-  return traced(tr, CKV_KERNEL_SELECT, [&] {
-    return launch_select(P, I.B * I.Hkv, static_cast<size_t>(P.smem_floats) * 4, stream);
-  });
+  return traced(tr, CKV_KERNEL_SELECT, [&] { return launch_select(P, I.B * I.Hkv, smem, stream); });
 }
 
 int run_gather(const ckv_problem* p, const Info& I, const int32_t* indices,
@@ -519,8 +563,7 @@ int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const voi
   float* raw = raw_scores ? raw_scores : ws.raw;
   std::copy(co.begin(), co.end(), cu_out);
   if ((rc = run_score(p, I, q_win, k, srh_mask, raw, ws, st)) != CKV_OK) return rc;
-  if ((rc = run_select(p, I, raw, co, indices, pooled_scores, ws, st)) != CKV_OK) return rc;
-  return run_gather(p, I, indices, co, k, v, k_out, v_out, ws.status, st);
+  return run_select(p, I, raw, co, indices, pooled_scores, ws, st, k, v, k_out, v_out);
 }
 
 int compresskv_read_device_status(const void* workspace, void* stream, int32_t* status) {

@@ -10,13 +10,12 @@ namespace ckv {
 
 constexpr int kHeadDim = 128;       // d: one 256-byte K row per token and group (16-bit types)
 constexpr int kTileTokens = 128;    // tokens per K tile = UMMA M = TMEM lanes
-constexpr int kStages = 4;          // K tiles in flight per CTA
+constexpr int kStages = 4;          // most K tiles in flight per CTA (fewer when Q rows are large)
 constexpr int kMaxQRows = 256;      // |S_g| * W rows per unit (UMMA N limit)
 constexpr int kMaxBatch = 512;
 constexpr int kMaxQHeads = 256;
 constexpr int kMaxKvHeads = 64;
 constexpr int kMaxItems = 1024;     // score work items per launch
-constexpr int kScoreThreads = 384;  // 12 warps: TMA, MMA, TMEM alloc, spare, 2 x 4 epilogue
 constexpr uint64_t kWaitTimeoutNs = 2000000000ull;  // 2 s: far above any legitimate wait
 
 // Device status codes (mirrors of the public CKV_ERR_* values).
@@ -44,6 +43,8 @@ struct ScoreParams {
   float c;                     // scale * log2(e)
   int window, num_kv_heads, p_total, n_items, is_bf16, use_evict_hint;
   int q_half_bytes;            // bytes of one 64-column half of the Q rows in shared memory
+  int small_n;                 // 1: every unit of the launch has at most 64 query rows
+  int stages;                  // K tiles in the shared-memory ring (2..kStages)
   int cu_seqlens[kMaxBatch + 1];
   int cu_prefix[kMaxBatch + 1];
   uint16_t srh_off[kMaxKvHeads + 1];   // SRH heads of group g: srh_heads[srh_off[g] .. srh_off[g+1])
@@ -57,7 +58,16 @@ struct SelectParams {
   float* pooled_ws;            // workspace copy of pooled scores, score layout
   int32_t* indices;            // [num_kv_heads][o_total]
   int* status;
-  int window, pool_width, num_kv_heads, p_total, o_total, batch, smem_floats;
+  const uint4* k;              // gather sources / destinations (when gather != 0)
+  const uint4* v;
+  uint4* k_out;
+  uint4* v_out;
+  long long tok_stride_v16, head_stride_v16;  // K/V strides in 16-byte units
+  int window, pool_width, num_kv_heads, p_total, o_total, batch;
+  int cluster;                 // CTAs per unit (thread-block cluster size, 1..8)
+  int slice;                   // prefix tokens per CTA (multiple of 32)
+  int smem_slice;              // 1: raw and pooled slices live in shared memory
+  int gather;                  // 1: also copy the retained K/V rows
   int cu_seqlens[kMaxBatch + 1];
   int cu_prefix[kMaxBatch + 1];
   int cu_out[kMaxBatch + 1];
@@ -81,7 +91,7 @@ cudaError_t launch_score_stats(const ScoreParams& p, int n_items, size_t smem, c
 cudaError_t launch_score_accum(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, int n_units, size_t smem, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, long long rows, cudaStream_t s);
-size_t score_smem_bytes(int q_half_bytes);
+size_t score_smem_bytes(int q_half_bytes, int stages);
 cudaError_t score_set_smem_limit(size_t bytes);
 cudaError_t select_set_smem_limit(size_t bytes);
 int select_max_smem_floats();

@@ -15,19 +15,23 @@
 // Each CTA owns one work item: a contiguous range of 128-token K tiles of one
 // unit.  Warp roles:
 //   warp 0     TMA producer: K tiles (two 64-column halves, 128-byte swizzle)
-//              into a kStages-deep shared-memory ring;
-//   warp 1     UMMA issuer: D[128 tokens x N] = K_tile . Q_S^T  (tcgen05.mma
-//              kind::f16, M=128, N = |S_g|*W rounded to 16, K = d = 128),
-//              fp32 accumulators in TMEM, 2 or 4 buffers;
-//   warp 2     TMEM allocation;
-//   warps 4-11 two epilogue warpgroups (alternate tiles); thread = token
-//              (TMEM lane), it reads its row of N logits with tcgen05.ld.
+//              into a kStages-deep shared-memory ring; it starts streaming
+//              while the other warps stage the query rows;
+//   warp 1     TMEM allocation, then UMMA issue: D[128 tokens x N] =
+//              K_tile . Q_S^T  (tcgen05.mma kind::f16, M=128, N = |S_g|*W
+//              rounded to 16, K = d = 128), fp32 accumulators in TMEM, 2 or 4
+//              buffers;
+//   warps 2-9  two epilogue warpgroups (alternate tiles); thread = token
+//              (TMEM lane), it loads its row of N logits from TMEM, hands the
+//              buffer back to the MMA warp at once and works from registers.
 // Tokens sit on the MMA's M side so every epilogue lane holds real work for
-// any N; in pass 2 the per-token sum over queries stays inside a thread.  In
-// pass 1 the per-query sums over tokens are formed with a 32x32 transpose-
-// reduction across the warp (31 shuffles per 1024 values) against a per-warp,
-// per-query reference that is only raised when a logit exceeds it by more
-// than 2^kTau, so the common path costs one exp per logit.
+// any N; in pass 2 the per-token sum over queries stays inside a thread.
+// Pass 1 keeps, per warp and query, a running reference (raised only when a
+// logit exceeds it by more than 2^kTau) and sums 2^(z*c - ref):
+//   * up to 64 query rows (kSmallN): every lane accumulates its own tokens
+//     in registers; the lanes are combined once per CTA by a 32x32
+//     transpose-reduction (31 shuffles per 32 queries);
+//   * more rows: the transpose-reduction runs per tile.
 #include <cuda_runtime.h>
 
 #include <cfloat>
@@ -39,31 +43,58 @@ namespace ckv {
 namespace {
 
 constexpr float kTau = 8.0f;  // log2 headroom before a running reference is raised
-constexpr int kNumEpiWarps = 8;
+constexpr int kNumEpiWarps = 8;  // pass-1 epilogue warps (2 warpgroups)
 constexpr int kEpiThreads = kNumEpiWarps * 32;
-constexpr int kMiscBytes = 256 + 2 * kNumEpiWarps * kMaxQRows * 4;
+// Epilogue warpgroups per pass: pass 1 keeps per-lane sums in registers and
+// runs 2; pass 2 needs few registers and runs 4 to hide TMEM-load latency.
+template <bool kAccum>
+struct Roles {
+  static constexpr int kWG = kAccum ? 4 : 2;
+  static constexpr int kThreads = 64 + 128 * kWG;
+  static constexpr int kStaged = kThreads - 32;  // warps 1.. stage the Q rows
+};
+// misc region: barriers (256 B) | refs/bias [8][256] f32 | sums [8][256] f32 |
+// rescale factors [8][256] f32 | window position of each query row [256] i32 |
+// per-warp logit scratch [8][32 lanes][33] f32 (pass 1, rare path)
+constexpr int kZScratchFloats = 32 * 33;
+constexpr int kMiscBytes =
+    256 + 3 * kNumEpiWarps * kMaxQRows * 4 + kMaxQRows * 4 + kNumEpiWarps * kZScratchFloats * 4;
 constexpr float kNegInf = -INFINITY;
+constexpr int kBarEpi = 1;       // named barrier: the 8 epilogue warps
+constexpr int kBarStaged = 2;    // named barrier: warps 1..9 after staging Q
+constexpr int kFirstEpiWarp = 2;
 
 __device__ __forceinline__ void wait_plain(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
   volatile int never = 0;
   mbar_wait_bounded(bar, parity, &never, nullptr, timeout_ns);
 }
 
-template <bool kAccum>
-__global__ void __launch_bounds__(kScoreThreads, 1)
+// Logit validity on tiles that reach the window or the end of the sequence:
+// key `tok` is visible to query row q (window position w = q mod W) iff
+// tok < L and tok <= n + w.
+__device__ __forceinline__ bool causal_ok(int tok, int L, int n, int q, int W) {
+  return tok < L && tok <= n + (q % W);
+}
+
+template <bool kAccum, bool kSmallN>
+__global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
     score_kernel(const __grid_constant__ ScoreParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sK = base;
-  uint8_t* sQ = base + kStages * kTileBytes;
+  const int nst = p.stages;  // K stages in the ring (2..kStages)
+  uint8_t* sQ = base + nst * kTileBytes;
   const int qh = p.q_half_bytes;
   uint8_t* sMisc = sQ + 2 * qh;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sMisc);  // full[S] empty[S] tfull[4] tempty[4]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sMisc);  // full[4] empty[4] tfull[4] tempty[4]
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(sMisc + 192);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(sMisc + 196);
   float* sRef = reinterpret_cast<float*>(sMisc + 256);   // [8][kMaxQRows] refs / pass-2 bias
-  float* sAcc = sRef + kNumEpiWarps * kMaxQRows;         // [8][kMaxQRows]
+  float* sAcc = sRef + kNumEpiWarps * kMaxQRows;         // [8][kMaxQRows] sums
+  float* sFac = sAcc + kNumEpiWarps * kMaxQRows;         // [8][kMaxQRows] rescale factors
+  int* sWpos = reinterpret_cast<int*>(sFac + kNumEpiWarps * kMaxQRows);  // [kMaxQRows]
+  float* sZ = reinterpret_cast<float*>(sWpos + kMaxQRows);               // [8][32][33]
 
   const uint32_t full0 = smem_u32(bars);
   const uint32_t empty0 = full0 + 8 * kStages;
@@ -94,7 +125,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
 
   // ------------------------------------------------------------ set-up
   if (threadIdx.x == 0) {
-    for (int i = 0; i < kStages; ++i) {
+    for (int i = 0; i < nst; ++i) {
       mbar_init(full0 + 8 * i, 1);
       mbar_init(empty0 + 8 * i, 1);
     }
@@ -106,59 +137,24 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) tma_prefetch_map(&p.tmap_k);
-  if (warp == 2) {
+  if (warp == 1) {
     tmem_alloc(smem_u32(tmem_holder), tcols);
     tmem_relinquish();
-  }
-  // Window-query rows of the SRH heads -> shared memory in the UMMA K-major
-  // 128-byte-swizzle layout (row r, 16-byte chunk ch of each 64-column half
-  // lands at chunk ch ^ (r & 7)); rows N..Npad-1 are zero.
-  for (int idx = threadIdx.x; idx < Npad * 16; idx += blockDim.x) {
-    const int r = idx >> 4;
-    const int ch = idx & 15;
-    uint4 val = make_uint4(0u, 0u, 0u, 0u);
-    if (r < N) {
-      const int head = p.srh_heads[h0 + r / W];
-      const int w = r - (r / W) * W;
-      const uint16_t* src = p.q + static_cast<long long>(s) * p.q_bs +
-                            static_cast<long long>(head) * p.q_hs +
-                            static_cast<long long>(w) * p.q_ws + ch * 8;
-      val = *reinterpret_cast<const uint4*>(src);
-    }
-    const int half = ch >> 3;
-    const int c8 = ch & 7;
-    *reinterpret_cast<uint4*>(sQ + half * qh + r * 128 + ((c8 ^ (r & 7)) << 4)) = val;
-  }
-  fence_proxy_async_smem();
-  if (kAccum) {
-    // Merge the unit's pass-1 partials (fixed order => deterministic) into
-    // the per-query bias m_q + log2 Z_q.
-    for (int q = threadIdx.x; q < N; q += blockDim.x) {
-      float m = kNegInf;
-      for (int i = 0; i < it.count; ++i)
-        m = fmaxf(m, p.partials[static_cast<long long>(it.first + i) * kMaxQRows + q].x);
-      float z = 0.f;
-      for (int i = 0; i < it.count; ++i) {
-        const float2 pr = p.partials[static_cast<long long>(it.first + i) * kMaxQRows + q];
-        if (pr.x != kNegInf) z += pr.y * ex2_approx(pr.x - m);
-      }
-      sRef[q] = m + log2f(z);
-    }
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tbase = *tmem_holder;
 
-  // ------------------------------------------------------------ roles
   if (warp == 0) {
+    // ---------------------------------------------------------- TMA producer
     if (lane == 0) {
       const uint64_t pol =
           (kAccum || !p.use_evict_hint) ? l2_policy_evict_first() : l2_policy_evict_last();
       int issued = 0;
       for (int i = 0; i < ntiles; ++i) {
-        const int st = i % kStages;
-        const uint32_t ph = static_cast<uint32_t>(i / kStages) & 1u;
+        const int st = i % nst;
+        const uint32_t ph = static_cast<uint32_t>(i / nst) & 1u;
         if (!mbar_wait_bounded(empty0 + 8 * st, ph ^ 1u, abort_flag, p.status)) break;
         mbar_arrive_expect_tx(full0 + 8 * st, kTileBytes);
         const int row = seq0 + (t0 + i) * kTileTokens;
@@ -169,150 +165,309 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
       }
       if (*abort_flag) {
         // let the copies already issued land before the CTA can exit
-        for (int i = max(0, issued - kStages); i < issued; ++i)
-          wait_plain(full0 + 8 * (i % kStages), static_cast<uint32_t>(i / kStages) & 1u,
-                     100000000ull);
+        for (int i = max(0, issued - nst); i < issued; ++i)
+          wait_plain(full0 + 8 * (i % nst), static_cast<uint32_t>(i / nst) & 1u, 100000000ull);
       }
     }
-  } else if (warp == 1) {
-    if (lane == 0) {
-      const uint32_t idesc = umma_idesc_f16(kTileTokens, Npad, p.is_bf16 != 0);
-      const uint32_t sq = smem_u32(sQ);
-      const uint32_t sk = smem_u32(sK);
-      int issued = 0;
-      for (int i = 0; i < ntiles; ++i) {
-        const int st = i % kStages;
-        const uint32_t ph = static_cast<uint32_t>(i / kStages) & 1u;
+    __syncwarp();  // reconverge before the CTA-wide (aligned) barrier below
+  } else {
+    // ---------------------------------------------------------- staging
+    // Window-query rows of the SRH heads -> shared memory in the UMMA K-major
+    // 128-byte-swizzle layout (row r, 16-byte chunk ch of each 64-column half
+    // lands at chunk ch ^ (r & 7)); rows N..Npad-1 are zero.
+    const int st_tid = threadIdx.x - 32;
+    constexpr int kStagedThreads = Roles<kAccum>::kStaged;
+    for (int idx = st_tid; idx < Npad * 16; idx += kStagedThreads) {
+      const int r = idx >> 4;
+      const int ch = idx & 15;
+      uint4 val = make_uint4(0u, 0u, 0u, 0u);
+      if (r < N) {
+        const int head = p.srh_heads[h0 + r / W];
+        const int w = r - (r / W) * W;
+        const uint16_t* src = p.q + static_cast<long long>(s) * p.q_bs +
+                              static_cast<long long>(head) * p.q_hs +
+                              static_cast<long long>(w) * p.q_ws + ch * 8;
+        val = *reinterpret_cast<const uint4*>(src);
+      }
+      const int half = ch >> 3;
+      const int c8 = ch & 7;
+      *reinterpret_cast<uint4*>(sQ + half * qh + r * 128 + ((c8 ^ (r & 7)) << 4)) = val;
+    }
+    fence_proxy_async_smem();
+    for (int q = st_tid; q < kMaxQRows; q += kStagedThreads) sWpos[q] = q < N ? q % W : 0;
+    if (kAccum) {
+      // Merge the unit's pass-1 partials (fixed order => deterministic) into
+      // the per-query bias m_q + log2 Z_q.
+      for (int q = st_tid; q < N; q += kStagedThreads) {
+        float m = kNegInf;
+        for (int i = 0; i < it.count; ++i)
+          m = fmaxf(m, p.partials[static_cast<long long>(it.first + i) * kMaxQRows + q].x);
+        float z = 0.f;
+        for (int i = 0; i < it.count; ++i) {
+          const float2 pr = p.partials[static_cast<long long>(it.first + i) * kMaxQRows + q];
+          if (pr.x != kNegInf) z += pr.y * ex2_approx(pr.x - m);
+        }
+        sRef[q] = m + log2f(z);
+      }
+    } else {
+      const int ew = warp - kFirstEpiWarp;
+      if (ew >= 0) {
+        for (int q = lane; q < kMaxQRows; q += 32) {
+          // padded rows (q >= N) never see a masked value, so they start at 0
+          sRef[ew * kMaxQRows + q] = q < N ? kNegInf : 0.f;
+          sAcc[ew * kMaxQRows + q] = 0.f;
+        }
+      }
+    }
+    named_bar_sync(kBarStaged, kStagedThreads);
+
+    if (warp == 1) {
+      // -------------------------------------------------------- UMMA issuer
+      if (lane == 0) {
+        const uint32_t idesc = umma_idesc_f16(kTileTokens, Npad, p.is_bf16 != 0);
+        // descriptor start addresses advance in 16-byte units (no carry out of
+        // the 14-bit field: shared memory is below 256 KB)
+        const uint64_t dq0 = smem_desc_sw128(smem_u32(sQ));
+        const uint64_t dk0 = smem_desc_sw128(smem_u32(sK));
+        int issued = 0;
+        for (int i = 0; i < ntiles; ++i) {
+          const int st = i % nst;
+          const uint32_t ph = static_cast<uint32_t>(i / nst) & 1u;
+          const int b = i % nbuf;
+          const uint32_t use = static_cast<uint32_t>(i / nbuf) & 1u;
+          if (!mbar_wait_bounded(tempty0 + 8 * b, use ^ 1u, abort_flag, p.status)) break;
+          tc_fence_after();
+          if (!mbar_wait_bounded(full0 + 8 * st, ph, abort_flag, p.status)) break;
+          tc_fence_after();
+          const uint32_t d = tbase + static_cast<uint32_t>(b * tstride);
+#pragma unroll
+          for (int kk = 0; kk < kHeadDim / 16; ++kk) {
+            const uint32_t koff = st * kTileBytes + (kk >> 2) * kHalfTileBytes + (kk & 3) * 32;
+            const uint32_t qoff = (kk >> 2) * qh + (kk & 3) * 32;
+            umma_f16(d, dk0 + (koff >> 4), dq0 + (qoff >> 4), idesc, kk > 0 ? 1u : 0u);
+          }
+          umma_commit(empty0 + 8 * st);
+          umma_commit(tfull0 + 8 * b);
+          ++issued;
+        }
+        if (*abort_flag && issued > 0) {
+          // the last commit covers every MMA issued: wait for it before TMEM is freed
+          const int i = issued - 1;
+          wait_plain(tfull0 + 8 * (i % nbuf), static_cast<uint32_t>(i / nbuf) & 1u,
+                     100000000ull);
+        }
+      }
+      __syncwarp();  // reconverge before the CTA-wide (aligned) barrier below
+    } else {
+      // -------------------------------------------------------- epilogue
+      const int ew = warp - kFirstEpiWarp;  // 0..7
+      constexpr int kWG = Roles<kAccum>::kWG;
+      const int wg = ew >> 2;   // epilogue warpgroup: tiles i with i % kWG == wg
+      const int qd = warp & 3;  // TMEM lane quarter this warp may access
+      const float c = p.c;
+      float* ref = sRef + ew * kMaxQRows;
+      float* acc_s = sAcc + ew * kMaxQRows;
+      float acc[kSmallN ? 64 : 1];  // pass 1, kSmallN: this lane's sums per query
+#pragma unroll
+      for (int j = 0; j < (kSmallN ? 64 : 1); ++j) acc[j] = 0.f;
+      const int nhalf = (N + 31) >> 5;  // 32-column groups per tile
+      float* zs = sZ + ew * kZScratchFloats;
+      float* fac = sFac + ew * kMaxQRows;
+
+      // Every TMEM buffer must belong to one warpgroup: an mbarrier parity
+      // wait cannot tell phase k from phase k+2, so warpgroups sharing a
+      // buffer could read it early.  With fewer buffers than warpgroups the
+      // extra warpgroups stay idle.
+      const int nwg = kWG < nbuf ? kWG : nbuf;
+      for (int i = wg; wg < nwg && i < ntiles; i += nwg) {
         const int b = i % nbuf;
         const uint32_t use = static_cast<uint32_t>(i / nbuf) & 1u;
-        if (!mbar_wait_bounded(tempty0 + 8 * b, use ^ 1u, abort_flag, p.status)) break;
+        const bool got = mbar_wait_bounded(tfull0 + 8 * b, use, abort_flag, p.status);
+        if (!__all_sync(0xffffffffu, got)) break;  // warp-uniform exit on abort
         tc_fence_after();
-        if (!mbar_wait_bounded(full0 + 8 * st, ph, abort_flag, p.status)) break;
-        tc_fence_after();
-        const uint32_t d = tbase + static_cast<uint32_t>(b * tstride);
-#pragma unroll
-        for (int kk = 0; kk < kHeadDim / 16; ++kk) {
-          const uint32_t koff = (kk >> 2) * kHalfTileBytes + (kk & 3) * 32;
-          const uint32_t qoff = (kk >> 2) * qh + (kk & 3) * 32;
-          umma_f16(d, smem_desc_sw128(sk + st * kTileBytes + koff), smem_desc_sw128(sq + qoff),
-                   idesc, kk > 0 ? 1u : 0u);
-        }
-        umma_commit(empty0 + 8 * st);
-        umma_commit(tfull0 + 8 * b);
-        ++issued;
-      }
-      if (*abort_flag && issued > 0) {
-        // the last commit covers every MMA issued: wait for it before TMEM is freed
-        const int i = issued - 1;
-        wait_plain(tfull0 + 8 * (i % nbuf), static_cast<uint32_t>(i / nbuf) & 1u, 100000000ull);
-      }
-    }
-  } else if (warp >= 4) {
-    const int ew = warp - 4;  // 0..7
-    const int wg = ew >> 2;   // epilogue warpgroup: tiles i with i % 2 == wg
-    const int qd = warp & 3;  // TMEM lane quarter this warp may access
-    const int nch = (N + 31) >> 5;
-    const float c = p.c;
-    float* ref = sRef + ew * kMaxQRows;
-    float* acc = sAcc + ew * kMaxQRows;
-    if (!kAccum) {
-      for (int q = lane; q < kMaxQRows; q += 32) {
-        ref[q] = kNegInf;
-        acc[q] = 0.f;
-      }
-      __syncwarp();
-    }
-    for (int i = wg; i < ntiles; i += 2) {
-      const int b = i % nbuf;
-      const uint32_t use = static_cast<uint32_t>(i / nbuf) & 1u;
-      const bool got = mbar_wait_bounded(tfull0 + 8 * b, use, abort_flag, p.status);
-      if (!__all_sync(0xffffffffu, got)) break;  // warp-uniform exit on abort
-      tc_fence_after();
-      const int tok = (t0 + i) * kTileTokens + qd * 32 + lane;  // position in the sequence
-      const uint32_t taddr =
-          tbase + (static_cast<uint32_t>(qd * 32) << 16) + static_cast<uint32_t>(b * tstride);
-      if (kAccum) {
-        float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-        for (int ch = 0; ch < nch; ++ch) {
-          float z[32];
-          tmem_load32(taddr + ch * 32, z);
-          const float* bias = sRef + ch * 32;
-          const int lim = N - ch * 32;
-#pragma unroll
-          for (int j = 0; j < 32; j += 4) {
-            const float4 bq = *reinterpret_cast<const float4*>(bias + j);
-            if (j + 0 < lim) s0 += ex2_approx(fmaf(z[j + 0], c, -bq.x));
-            if (j + 1 < lim) s1 += ex2_approx(fmaf(z[j + 1], c, -bq.y));
-            if (j + 2 < lim) s2 += ex2_approx(fmaf(z[j + 2], c, -bq.z));
-            if (j + 3 < lim) s3 += ex2_approx(fmaf(z[j + 3], c, -bq.w));
-          }
-        }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(tempty0 + 8 * b);
-        if (tok < n) {
-          p.raw[static_cast<long long>(g) * p.p_total + p.cu_prefix[s] + tok] =
-              (s0 + s1) + (s2 + s3);
-        }
-      } else {
-        // tiles reaching the window (causal mask) or past the sequence end
+        const int tok = (t0 + i) * kTileTokens + qd * 32 + lane;  // position in the sequence
+        const uint32_t taddr =
+            tbase + (static_cast<uint32_t>(qd * 32) << 16) + static_cast<uint32_t>(b * tstride);
+        // tiles that reach the window (causal mask) or pass the sequence end
         const bool edge = (t0 + i + 1) * kTileTokens > n;
-        for (int ch = 0; ch < nch; ++ch) {
-          float z[32];
-          tmem_load32(taddr + ch * 32, z);
-          const float* rf = ref + ch * 32;
-          float t[32];
-          float tmax = kNegInf;
+        const int vis = n - tok;  // query row q sees this key iff tok < L and wpos(q) >= -vis
+        float s_tok = 0.f;        // pass 2: this token's score
+
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const int q = ch * 32 + j;
-            bool valid = q < N;
-            if (edge) valid = valid && tok < L && tok <= n + (q % W);
-            z[j] = valid ? z[j] * c : kNegInf;
-            t[j] = valid ? z[j] - rf[j] : kNegInf;
-            tmax = fmaxf(tmax, t[j]);
-          }
-          if (__any_sync(0xffffffffu, tmax > kTau)) {
-            // raise the references of this chunk's queries to their column max
-            float zz[32];
-#pragma unroll
-            for (int j = 0; j < 32; ++j) zz[j] = z[j];
-            const float cmax = warp_transpose_max32(zz, lane);
-            const int q = ch * 32 + lane;
-            const float old = ref[q];
-            const float nw = fmaxf(old, cmax);
-            if (nw != old) {
-              acc[q] *= (old == kNegInf) ? 0.f : ex2_approx(old - nw);
-              ref[q] = nw;
+        for (int hh = 0; hh < (kSmallN ? 2 : 1); ++hh) {
+          for (int hr = 0; hr < (kSmallN ? 1 : nhalf); ++hr) {
+            const int h = kSmallN ? hh : hr;
+            if (kSmallN && h >= nhalf) break;  // uniform: N <= 32
+            const int c0 = 32 * h;
+            uint32_t r[32];
+            tmem_load32_async(taddr + c0, r);
+            tmem_wait_ld(r);
+            if (kAccum && h == nhalf - 1) {
+              // every column of this tile is in registers: hand the buffer back
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(tempty0 + 8 * b);
             }
-            __syncwarp();
+            const int lim = min(32, N - c0);  // valid columns in this group
+            const bool masked = edge || lim < 32;
+            float z[32];  // raw logits (scaled by c inside the FFMA below)
 #pragma unroll
-            for (int j = 0; j < 32; ++j) t[j] = (z[j] == kNegInf) ? kNegInf : z[j] - rf[j];
+            for (int j = 0; j < 32; ++j) z[j] = __uint_as_float(r[j]);
+            if (masked) {
+#pragma unroll
+              for (int j = 0; j < 32; j += 4) {
+                const int4 wq = *reinterpret_cast<const int4*>(sWpos + c0 + j);
+                const int wv[4] = {wq.x, wq.y, wq.z, wq.w};
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                  const bool ok = (j + u) < lim && (!edge || (tok < L && wv[u] >= -vis));
+                  z[j + u] = ok ? z[j + u] : kNegInf;
+                }
+              }
+            }
+
+            if constexpr (kAccum) {
+              // ---------------------------------------------- pass 2
+              const float* bias = sRef + c0;
+              float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll
+              for (int j = 0; j < 32; j += 4) {
+                const float4 bq = *reinterpret_cast<const float4*>(bias + j);
+                a0 += ex2_approx(fmaf(z[j + 0], c, -bq.x));
+                a1 += ex2_approx(fmaf(z[j + 1], c, -bq.y));
+                a2 += ex2_approx(fmaf(z[j + 2], c, -bq.z));
+                a3 += ex2_approx(fmaf(z[j + 3], c, -bq.w));
+              }
+              s_tok += (a0 + a1) + (a2 + a3);
+            } else {
+              // ---------------------------------------------- pass 1
+              float* rf = ref + c0;
+              // t = z*c - ref, computed once; -inf where masked
+              float t[32];
+              float tmax = kNegInf;
+              if (masked) {
+#pragma unroll
+                for (int j = 0; j < 32; j += 4) {
+                  const float4 rq = *reinterpret_cast<const float4*>(rf + j);
+                  const float rv[4] = {rq.x, rq.y, rq.z, rq.w};
+#pragma unroll
+                  for (int u = 0; u < 4; ++u) {
+                    t[j + u] = z[j + u] == kNegInf ? kNegInf : fmaf(z[j + u], c, -rv[u]);
+                    tmax = fmaxf(tmax, t[j + u]);
+                  }
+                }
+              } else {
+#pragma unroll
+                for (int j = 0; j < 32; j += 4) {
+                  const float4 rq = *reinterpret_cast<const float4*>(rf + j);
+                  t[j + 0] = fmaf(z[j + 0], c, -rq.x);
+                  t[j + 1] = fmaf(z[j + 1], c, -rq.y);
+                  t[j + 2] = fmaf(z[j + 2], c, -rq.z);
+                  t[j + 3] = fmaf(z[j + 3], c, -rq.w);
+                  tmax = fmaxf(fmaxf(tmax, fmaxf(t[j], t[j + 1])), fmaxf(t[j + 2], t[j + 3]));
+                }
+              }
+              if (__any_sync(0xffffffffu, tmax > kTau)) {
+                // Rare: raise each query's reference to its column max over
+                // the warp and rescale the sums kept so far by 2^(old - new).
+                // The scaled logits go through shared memory so this path
+                // stays small.
+                {
+                  // re-read this group's logits (the buffer is still held)
+                  uint32_t r2[32];
+                  tmem_load32_async(taddr + c0, r2);
+                  tmem_wait_ld(r2);
+#pragma unroll
+                  for (int j = 0; j < 32; ++j)
+                    zs[lane * 33 + j] = t[j] == kNegInf ? kNegInf : __uint_as_float(r2[j]) * c;
+                }
+                __syncwarp();
+                float m = kNegInf;
+                for (int rr = 0; rr < 32; ++rr) m = fmaxf(m, zs[rr * 33 + lane]);
+                const float old = rf[lane];
+                const float nw = fmaxf(old, m);
+                const float f =
+                    (nw == old) ? 1.f : ((old == kNegInf) ? 0.f : ex2_approx(old - nw));
+                rf[lane] = nw;
+                if constexpr (kSmallN) {
+                  fac[c0 + lane] = f;
+                } else {
+                  acc_s[c0 + lane] *= f;
+                }
+                __syncwarp();
+#pragma unroll
+                for (int j = 0; j < 32; j += 4) {
+                  const float4 rq = *reinterpret_cast<const float4*>(rf + j);
+                  const float rv[4] = {rq.x, rq.y, rq.z, rq.w};
+#pragma unroll
+                  for (int u = 0; u < 4; ++u) {
+                    const float zc = zs[lane * 33 + j + u];
+                    t[j + u] = zc == kNegInf ? kNegInf : zc - rv[u];
+                  }
+                }
+                if constexpr (kSmallN) {
+#pragma unroll
+                  for (int j = 0; j < 32; j += 4) {
+                    const float4 fq = *reinterpret_cast<const float4*>(fac + c0 + j);
+                    acc[32 * hh + j + 0] *= fq.x;
+                    acc[32 * hh + j + 1] *= fq.y;
+                    acc[32 * hh + j + 2] *= fq.z;
+                    acc[32 * hh + j + 3] *= fq.w;
+                  }
+                }
+              }
+              if constexpr (kSmallN) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) acc[32 * hh + j] += ex2_approx(t[j]);
+              } else {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) t[j] = ex2_approx(t[j]);
+                const float colsum = warp_transpose_sum32(t, lane);
+                acc_s[c0 + lane] += colsum;
+              }
+              __syncwarp();
+            }
           }
+        }
+        if (!kAccum) {
+          // pass 1 keeps the buffer until the tile is done (the rare path re-reads it)
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(tempty0 + 8 * b);
+        }
+        if (kAccum && tok < n) {
+          p.raw[static_cast<long long>(g) * p.p_total + p.cu_prefix[s] + tok] = s_tok;
+        }
+      }
+
+      if (!kAccum) {
+        if constexpr (kSmallN) {
+          // one cross-lane reduction of the per-lane sums per CTA
 #pragma unroll
-          for (int j = 0; j < 32; ++j) t[j] = ex2_approx(t[j]);
-          const float colsum = warp_transpose_sum32(t, lane);
-          acc[ch * 32 + lane] += colsum;
+          for (int h = 0; h < 2; ++h) {
+            if (h * 32 < N) {
+              float v[32];
+#pragma unroll
+              for (int j = 0; j < 32; ++j) v[j] = acc[32 * h + j];
+              const float colsum = warp_transpose_sum32(v, lane);
+              acc_s[32 * h + lane] = colsum;
+            }
+          }
           __syncwarp();
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(tempty0 + 8 * b);
-      }
-    }
-    if (!kAccum) {
-      // combine the 8 epilogue warps' (reference, sum) pairs per query
-      named_bar_sync(1, kEpiThreads);
-      const int te = threadIdx.x - 4 * 32;
-      if (te < N && !*abort_flag) {
-        float m = kNegInf;
-        for (int w = 0; w < kNumEpiWarps; ++w) m = fmaxf(m, sRef[w * kMaxQRows + te]);
-        float z = 0.f;
-        for (int w = 0; w < kNumEpiWarps; ++w) {
-          const float r = sRef[w * kMaxQRows + te];
-          if (r != kNegInf) z += sAcc[w * kMaxQRows + te] * ex2_approx(r - m);
+        // combine the 8 epilogue warps' (reference, sum) pairs per query
+        named_bar_sync(kBarEpi, kEpiThreads);
+        const int te = static_cast<int>(threadIdx.x) - kFirstEpiWarp * 32;
+        if (te < N && !*abort_flag) {
+          float m = kNegInf;
+          for (int w = 0; w < kNumEpiWarps; ++w) m = fmaxf(m, sRef[w * kMaxQRows + te]);
+          float z = 0.f;
+          for (int w = 0; w < kNumEpiWarps; ++w) {
+            const float r = sRef[w * kMaxQRows + te];
+            if (r != kNegInf) z += sAcc[w * kMaxQRows + te] * ex2_approx(r - m);
+          }
+          p.partials[static_cast<long long>(blockIdx.x) * kMaxQRows + te] = make_float2(m, z);
         }
-        p.partials[static_cast<long long>(blockIdx.x) * kMaxQRows + te] = make_float2(m, z);
       }
     }
   }
@@ -320,43 +475,52 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
   // ------------------------------------------------------------ teardown
   tc_fence_before();
   __syncthreads();
-  if (warp == 2) {
+  if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tbase, tcols);
   }
 }
 
-template <bool kAccum>
+template <bool kAccum, bool kSmallN>
 cudaError_t launch(const ScoreParams& p, int n_items, size_t smem, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(n_items));
-  cfg.blockDim = dim3(kScoreThreads);
+  cfg.blockDim = dim3(Roles<kAccum>::kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  return cudaLaunchKernelEx(&cfg, score_kernel<kAccum>, p);
+  return cudaLaunchKernelEx(&cfg, score_kernel<kAccum, kSmallN>, p);
 }
 
 }  // namespace
 
-size_t score_smem_bytes(int q_half_bytes) {
-  return 1024 + static_cast<size_t>(kStages) * kTileBytes + 2 * static_cast<size_t>(q_half_bytes) +
+size_t score_smem_bytes(int q_half_bytes, int stages) {
+  return 1024 + static_cast<size_t>(stages) * kTileBytes + 2 * static_cast<size_t>(q_half_bytes) +
          kMiscBytes;
 }
 
 cudaError_t score_set_smem_limit(size_t bytes) {
-  cudaError_t e = cudaFuncSetAttribute(score_kernel<false>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(bytes));
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(score_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(bytes));
+  const int b = static_cast<int>(bytes);
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(score_kernel<false, false>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, b)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(score_kernel<true, false>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, b)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(score_kernel<false, true>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, b)) != cudaSuccess)
+    return e;
+  return cudaFuncSetAttribute(score_kernel<true, true>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize, b);
 }
 
 cudaError_t launch_score_stats(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s) {
-  return launch<false>(p, n_items, smem, s);
+  return p.small_n ? launch<false, true>(p, n_items, smem, s)
+                   : launch<false, false>(p, n_items, smem, s);
 }
 cudaError_t launch_score_accum(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s) {
-  return launch<true>(p, n_items, smem, s);
+  return p.small_n ? launch<true, true>(p, n_items, smem, s)
+                   : launch<true, false>(p, n_items, smem, s);
 }
 
 }  // namespace ckv

@@ -1,32 +1,41 @@
 // Pooling + budgeted top-k + window append (CompressKV Sec. 3.3: pooled
 // window scores, the top-N prefix tokens are retained; Sec. 4: pooling kernel
-// over the token dimension, the last W tokens are always kept).
+// over the token dimension, the last W tokens are always kept), optionally
+// fused with the K/V gather of the retained rows (Sec. 3.3 eviction).
 //
-// One CTA of 1024 threads per unit (sequence, KV group):
-//   1. pooled_j = (sum_{t=-r..r} raw_{j+t}) / P over the prefix, zero outside
-//      [0, n) (fixed summation order, so results are deterministic); the
-//      pooled vector lives in shared memory when it fits, otherwise in the
-//      workspace (it is re-read from L2);
-//   2. the k-th largest pooled value is found exactly by a 3-pass radix select
-//      on the fp32 bit patterns (pooled >= 0, so bit order == value order),
-//      11/11/10 bits, shared-memory histograms with warp-aggregated atomics;
+// One thread-block cluster of C CTAs (C <= 8) per unit (sequence, KV group).
+// CTA r of the cluster owns the contiguous prefix slice [r*S, (r+1)*S):
+//   1. it stages raw[slice - halo] in shared memory (all loads in flight) and
+//      computes pooled_j = (sum_{t=-h..h} raw_{j+t}) / P, zero outside [0, n),
+//      in a fixed summation order (deterministic);
+//   2. the k-th largest pooled value is found exactly by a 4-pass radix
+//      select on the fp32 bit patterns (pooled >= 0, so bit order == value
+//      order), 8 bits per pass: each CTA builds a shared-memory histogram of
+//      its slice, one cluster barrier, then every CTA sums the C histograms
+//      over distributed shared memory and picks the same bin (a unit with a
+//      single CTA is launched without a cluster and uses __syncthreads);
 //   3. ordered compaction: every token above the k-th value plus the
-//      lowest-position tokens equal to it, written in ascending position;
-//      each warp owns a contiguous segment, segments are placed by one
-//      block-wide scan;
-//   4. the W window positions n..L-1 follow.
+//      lowest-position tokens equal to it; slices are placed by an exclusive
+//      scan of the per-CTA counts read over distributed shared memory;
+//   4. the last CTA appends the W window positions;
+//   5. (gather) each warp copies the K and V rows of the tokens it selected.
+// Slices larger than the shared-memory budget keep the pooled scores in the
+// workspace instead (re-read from L2).
+#include <cooperative_groups.h>
 #include <cuda_runtime.h>
 
 #include "ckv_device.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace ckv {
 
 namespace {
 
-constexpr int kSelThreads = 1024;
+constexpr int kSelThreads = 512;
 constexpr int kSelWarps = kSelThreads / 32;
-constexpr int kBins = 2048;
-constexpr int kSelStaticSmem = kBins * 4 + 4 * kSelWarps * 4 + 64;
+constexpr int kBins = 256;
+constexpr int kSelStaticSmem = 2 * kBins * 4 + kBins * 4 + 8 * kSelWarps * 4 + 256;
 
 __device__ __forceinline__ uint32_t lanemask_lt(int lane) { return (1u << lane) - 1u; }
 
@@ -40,19 +49,65 @@ __device__ __forceinline__ int warp_exclusive_scan(int v, int lane) {
   return x - v;
 }
 
-__global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_constant__ SelectParams p) {
-  extern __shared__ float s_pooled[];
-  __shared__ uint32_t hist[kBins];
-  __shared__ int s_gt[kSelWarps], s_eq[kSelWarps], s_eqbase[kSelWarps], s_selbase[kSelWarps];
-  __shared__ int s_bin, s_above;
+// Cluster-wide barrier.  The .aligned forms require every thread of a warp
+// to execute them together, so the warp is reconverged first.
+__device__ __forceinline__ void cluster_barrier() {
+  __syncwarp();
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
 
+// Barrier over the CTAs that share a unit: the whole cluster, or just this
+// CTA when a unit has one CTA (launched without a cluster).
+template <bool kCluster>
+__device__ __forceinline__ void unit_barrier() {
+  if (kCluster) {
+    cluster_barrier();
+  } else {
+    __syncthreads();
+  }
+}
+
+// Shared-memory word `ptr` of CTA `rank` of this unit's cluster.
+template <bool kCluster, class T>
+__device__ __forceinline__ T* unit_rank_ptr(T* ptr, int rank) {
+  if (kCluster) return cg::this_cluster().map_shared_rank(ptr, rank);
+  return ptr;
+}
+
+// One warp copies the K and V rows of token `tok` (position in its sequence)
+// to output row `orow`: lanes 0-15 move K, lanes 16-31 move V.
+__device__ __forceinline__ void copy_kv_row(const SelectParams& p, int seq0, int g, int tok,
+                                            long long orow, int lane) {
+  const long long src = static_cast<long long>(seq0 + tok) * p.tok_stride_v16 +
+                        static_cast<long long>(g) * p.head_stride_v16;
+  const long long dst = (orow * p.num_kv_heads + g) * (kHeadDim * 2 / 16);
+  const int part = lane & 15;
+  if (lane < 16) {
+    p.k_out[dst + part] = __ldg(p.k + src + part);
+  } else {
+    p.v_out[dst + part] = __ldg(p.v + src + part);
+  }
+}
+
+template <bool kCluster>
+__global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_constant__ SelectParams p) {
+  extern __shared__ float s_dyn[];
+  __shared__ uint32_t hist[2][kBins];
+  __shared__ uint32_t ghist[kBins];
+  __shared__ int s_gt[kSelWarps], s_eq[kSelWarps], s_eqbase[kSelWarps], s_selbase[kSelWarps];
+  __shared__ int s_bin, s_above, s_cta_gt, s_cta_eq;
+
+  const int C = kCluster ? static_cast<int>(cg::this_cluster().num_blocks()) : 1;
+  const int crank = kCluster ? static_cast<int>(cg::this_cluster().block_rank()) : 0;
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
   const int lane = tid & 31;
-  const int u = blockIdx.x;
+  const int u = blockIdx.x / C;
   const int s = u / p.num_kv_heads;
   const int g = u - s * p.num_kv_heads;
-  const int L = p.cu_seqlens[s + 1] - p.cu_seqlens[s];
+  const int seq0 = p.cu_seqlens[s];
+  const int L = p.cu_seqlens[s + 1] - seq0;
   const int W = p.window;
   const int n = max(L - W, 0);
   const int out0 = p.cu_out[s];
@@ -60,56 +115,111 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   int32_t* out = p.indices + static_cast<long long>(g) * p.o_total + out0;
   const long long soff = static_cast<long long>(g) * p.p_total + p.cu_prefix[s];
   const float* raw = p.raw + soff;
-  float* buf = (n <= p.smem_floats) ? s_pooled : p.pooled_ws + soff;
   float* pout = p.pooled_out ? p.pooled_out + soff : nullptr;
-
-  // 1. average pooling
   const int r = (p.pool_width - 1) >> 1;
+  const int S = p.slice;  // prefix tokens per CTA (multiple of 32)
+  const int lo = min(n, crank * S);
+  const int hi = min(n, lo + S);
+  const int len = hi - lo;
+  const bool in_smem = p.smem_slice;
+  float* raw_s = s_dyn;                                  // [S + 2r] when in_smem
+  float* pooled = in_smem ? s_dyn + S + 2 * r : p.pooled_ws + soff + lo;  // [len]
+
+  // 1. pooling ---------------------------------------------------------------
   const float fP = static_cast<float>(p.pool_width);
-  for (int j = tid; j < n; j += kSelThreads) {
-    float a = 0.f;
-    for (int t = -r; t <= r; ++t) {
-      const int jj = j + t;
-      if (jj >= 0 && jj < n) a += raw[jj];
+  if (len > 0) {
+    if (in_smem) {
+      const int span = len + 2 * r;
+      for (int base = 0; base < span; base += 8 * kSelThreads) {
+        float v[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int li = base + i * kSelThreads + tid;
+          const int j = lo - r + li;
+          v[i] = (li < span && j >= 0 && j < n) ? raw[j] : 0.f;
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int li = base + i * kSelThreads + tid;
+          if (li < span) raw_s[li] = v[i];
+        }
+      }
+      __syncthreads();
+      for (int i = tid; i < len; i += kSelThreads) {
+        float a = 0.f;
+        for (int t = 0; t <= 2 * r; ++t) a += raw_s[i + t];
+        const float pv = a / fP;
+        pooled[i] = pv;
+        if (pout) pout[lo + i] = pv;
+      }
+    } else {
+      for (int i = tid; i < len; i += kSelThreads) {
+        const int j = lo + i;
+        float a = 0.f;
+        for (int t = -r; t <= r; ++t) {
+          const int jj = j + t;
+          a += (jj >= 0 && jj < n) ? raw[jj] : 0.f;
+        }
+        const float pv = a / fP;
+        pooled[i] = pv;
+        if (pout) pout[j] = pv;
+      }
     }
-    const float v = a / fP;
-    buf[j] = v;
-    if (pout) pout[j] = v;
   }
-  if (kept >= L) {  // budget covers the sequence (or L <= W): everything kept
-    for (int i = tid; i < L; i += kSelThreads) out[i] = i;
-    return;
+
+  // keep-everything units (budget >= L, or L <= W): indices 0..L-1
+  if (kept >= L) {
+    const int per = (L + C - 1) / C;
+    const int a0 = min(L, crank * per);
+    const int a1 = min(L, a0 + per);
+    for (int i = a0 + tid; i < a1; i += kSelThreads) out[i] = i;
+    if (p.gather) {
+      for (int i = a0 + warp; i < a1; i += kSelWarps) copy_kv_row(p, seq0, g, i, out0 + i, lane);
+    }
+    return;  // uniform over the cluster: no cluster barrier is pending
   }
   const int k = kept - W;  // 0 <= k < n
-  for (int w = tid; w < W; w += kSelThreads) out[k + w] = n + w;
-  if (k == 0) return;
+  if (crank == C - 1) {
+    for (int w = tid; w < W; w += kSelThreads) out[k + w] = n + w;
+    if (p.gather) {
+      for (int w = warp; w < W; w += kSelWarps) copy_kv_row(p, seq0, g, n + w, out0 + k + w, lane);
+    }
+  }
+  if (k == 0) return;  // window only (uniform over the cluster)
   __syncthreads();
-  const uint32_t* keys = reinterpret_cast<const uint32_t*>(buf);
+  const uint32_t* keys = reinterpret_cast<const uint32_t*>(pooled);
 
-  // 2. radix select of the k-th largest key
+  // 2. radix select of the k-th largest key --------------------------------
   uint32_t prefix = 0u, pmask = 0u;
   int rem = k;
 #pragma unroll 1
-  for (int pass = 0; pass < 3; ++pass) {
-    const int sh = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
-    const uint32_t nb = pass == 2 ? 1024u : 2048u;
-    for (int b = tid; b < kBins; b += kSelThreads) hist[b] = 0u;
+  for (int pass = 0; pass < 4; ++pass) {
+    const int sh = 24 - 8 * pass;
+    uint32_t* h = hist[pass & 1];
+    for (int b = tid; b < kBins; b += kSelThreads) h[b] = 0u;
     __syncthreads();
-    for (int base = 0; base < n; base += kSelThreads) {
-      const int j = base + tid;
-      const uint32_t key = j < n ? keys[j] : 0u;
-      const bool match = j < n && (key & pmask) == prefix;
-      const uint32_t bin = (key >> sh) & (nb - 1u);
+    for (int base = 0; base < len; base += kSelThreads) {
+      const int i = base + tid;
+      const uint32_t key = i < len ? keys[i] : 0u;
+      const bool match = i < len && (key & pmask) == prefix;
+      const uint32_t bin = (key >> sh) & 255u;
       const uint32_t active = __ballot_sync(0xffffffffu, match);
       if (match) {
         const uint32_t peers = __match_any_sync(active, bin);
-        if (lane == __ffs(peers) - 1) atomicAdd(&hist[bin], static_cast<uint32_t>(__popc(peers)));
+        if (lane == __ffs(peers) - 1) atomicAdd(&h[bin], static_cast<uint32_t>(__popc(peers)));
       }
+    }
+    unit_barrier<kCluster>();
+    for (int b = tid; b < kBins; b += kSelThreads) {
+      uint32_t tot = 0u;
+      for (int q = 0; q < C; ++q) tot += unit_rank_ptr<kCluster>(h, q)[b];
+      ghist[b] = tot;
     }
     __syncthreads();
     if (warp == 0) {
       uint32_t cnt = 0u;
-      for (int b = 0; b < kBins / 32; ++b) cnt += hist[lane * (kBins / 32) + b];
+#pragma unroll
+      for (int b = 0; b < kBins / 32; ++b) cnt += ghist[lane * (kBins / 32) + b];
       uint32_t suf = cnt;  // inclusive suffix sum over lanes
 #pragma unroll
       for (int off = 1; off < 32; off <<= 1) {
@@ -117,18 +227,17 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
         if (lane + off < 32) suf += y;
       }
       const uint32_t ok = __ballot_sync(0xffffffffu, suf >= static_cast<uint32_t>(rem));
-      const int top = 31 - __clz(ok);  // highest lane whose suffix still holds rem keys
+      const int top = ok ? 31 - __clz(ok) : 0;
       const uint32_t nxt = __shfl_sync(0xffffffffu, suf, top < 31 ? top + 1 : 31);
-      const uint32_t above0 = top < 31 ? nxt : 0u;
       if (lane == top) {
-        uint32_t above = above0;
+        uint32_t above = top < 31 ? nxt : 0u;
         int bsel = lane * (kBins / 32);
         for (int b = lane * (kBins / 32) + kBins / 32 - 1; b >= lane * (kBins / 32); --b) {
-          if (above + hist[b] >= static_cast<uint32_t>(rem)) {
+          if (above + ghist[b] >= static_cast<uint32_t>(rem)) {
             bsel = b;
             break;
           }
-          above += hist[b];
+          above += ghist[b];
         }
         s_bin = bsel;
         s_above = static_cast<int>(above);
@@ -137,21 +246,20 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
     __syncthreads();
     rem -= s_above;
     prefix |= static_cast<uint32_t>(s_bin) << sh;
-    pmask |= (nb - 1u) << sh;
-    __syncthreads();
+    pmask |= 255u << sh;
   }
   const uint32_t tau = prefix;  // bit pattern of the k-th largest pooled value
   const int need_eq = rem;      // how many of the values equal to tau are kept
 
-  // 3. ordered compaction
-  const int seg = ((n + kSelWarps * 32 - 1) / (kSelWarps * 32)) * 32;
-  const int lo = min(n, warp * seg);
-  const int hi = min(n, lo + seg);
+  // 3. ordered compaction ----------------------------------------------------
+  const int seg = ((len + kSelWarps * 32 - 1) / (kSelWarps * 32)) * 32;
+  const int wlo = min(len, warp * seg);
+  const int whi = min(len, wlo + seg);
   int cgt = 0, ceq = 0;
-  for (int b0 = lo; b0 < hi; b0 += 32) {
-    const int j = b0 + lane;
-    const bool in = j < hi;
-    const uint32_t key = in ? keys[j] : 0u;
+  for (int b0 = wlo; b0 < whi; b0 += 32) {
+    const int i = b0 + lane;
+    const bool in = i < whi;
+    const uint32_t key = in ? keys[i] : 0u;
     cgt += __popc(__ballot_sync(0xffffffffu, in && key > tau));
     ceq += __popc(__ballot_sync(0xffffffffu, in && key == tau));
   }
@@ -161,27 +269,58 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   }
   __syncthreads();
   if (warp == 0) {
-    const int e = s_eq[lane];
-    const int eq_before = warp_exclusive_scan(e, lane);
-    const int take = min(max(need_eq - eq_before, 0), e);
-    const int sel = s_gt[lane] + take;
-    s_eqbase[lane] = eq_before;
-    s_selbase[lane] = warp_exclusive_scan(sel, lane);
+    const int e = lane < kSelWarps ? s_eq[lane] : 0;
+    const int gt = lane < kSelWarps ? s_gt[lane] : 0;
+    const int eq_incl = warp_exclusive_scan(e, lane) + e;
+    const int gt_incl = warp_exclusive_scan(gt, lane) + gt;
+    if (lane == 31) {
+      s_cta_gt = gt_incl;
+      s_cta_eq = eq_incl;
+    }
   }
-  __syncthreads();
+  unit_barrier<kCluster>();  // every CTA's totals are visible
+  if (warp == 0) {
+    // totals of the lower-ranked CTAs of the cluster
+    int gt_before = 0, eq_before = 0;
+    for (int q = 0; q < crank; ++q) {
+      gt_before += *unit_rank_ptr<kCluster>(&s_cta_gt, q);
+      eq_before += *unit_rank_ptr<kCluster>(&s_cta_eq, q);
+    }
+    const int take_before = min(need_eq, eq_before);  // ties are taken in position order
+    const int e = lane < kSelWarps ? s_eq[lane] : 0;
+    const int w_eq_before = eq_before + warp_exclusive_scan(e, lane);
+    const int take = min(max(need_eq - w_eq_before, 0), e);
+    const int sel = (lane < kSelWarps ? s_gt[lane] : 0) + take;
+    const int sel_before = warp_exclusive_scan(sel, lane);  // every lane takes part
+    if (lane < kSelWarps) {
+      s_eqbase[lane] = w_eq_before;
+      s_selbase[lane] = gt_before + take_before + sel_before;
+    }
+  }
+  unit_barrier<kCluster>();  // no CTA leaves while others may still read its shared memory
   int eq_seen = s_eqbase[warp];
   int pos = s_selbase[warp];
-  for (int b0 = lo; b0 < hi; b0 += 32) {
-    const int j = b0 + lane;
-    const bool in = j < hi;
-    const uint32_t key = in ? keys[j] : 0u;
+  for (int b0 = wlo; b0 < whi; b0 += 32) {
+    const int i = b0 + lane;
+    const bool in = i < whi;
+    const uint32_t key = in ? keys[i] : 0u;
     const uint32_t mgt = __ballot_sync(0xffffffffu, in && key > tau);
     const uint32_t meq = __ballot_sync(0xffffffffu, in && key == tau);
     const bool take_eq =
         in && key == tau && (eq_seen + __popc(meq & lanemask_lt(lane))) < need_eq;
     const uint32_t msel = mgt | __ballot_sync(0xffffffffu, take_eq);
     const int o = pos + __popc(msel & lanemask_lt(lane));
-    if ((msel & (1u << lane)) && o < k) out[o] = j;
+    if ((msel & (1u << lane)) && o < k) out[o] = lo + i;
+    if (p.gather) {
+      uint32_t m = msel;
+      int oo = pos;
+      while (m) {
+        const int bit = __ffs(m) - 1;
+        m &= m - 1;
+        if (oo < k) copy_kv_row(p, seq0, g, lo + b0 + bit, out0 + oo, lane);
+        ++oo;
+      }
+    }
     pos += __popc(msel);
     eq_seen += __popc(meq);
   }
@@ -192,17 +331,29 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
 int select_max_smem_floats() { return (227 * 1024 - kSelStaticSmem - 1024) / 4; }
 
 cudaError_t select_set_smem_limit(size_t bytes) {
-  return cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(select_kernel<false>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(bytes));
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(select_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               static_cast<int>(bytes));
 }
 
 cudaError_t launch_select(const SelectParams& p, int n_units, size_t smem, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(n_units));
+  cfg.gridDim = dim3(static_cast<unsigned>(n_units * p.cluster));
   cfg.blockDim = dim3(kSelThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  return cudaLaunchKernelEx(&cfg, select_kernel, p);
+  if (p.cluster <= 1) return cudaLaunchKernelEx(&cfg, select_kernel<false>, p);
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(p.cluster);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, select_kernel<true>, p);
 }
 
 }  // namespace ckv
