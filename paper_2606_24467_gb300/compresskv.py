@@ -179,12 +179,14 @@ class Trace:
     """Launch trace: ``capacity`` launches bracketed by CUDA events."""
 
     def __init__(self, capacity: int):
+        """``capacity`` = 0 only counts launches (no events are recorded)."""
         self.events = [torch.cuda.Event(enable_timing=True) for _ in range(2 * capacity)]
         for e in self.events:  # torch creates the CUDA event on its first record
             e.record()
-        torch.cuda.synchronize()
-        self._ev = (c_void_p * (2 * capacity))(*[e.cuda_event for e in self.events])
-        self._kinds = (c_int32 * capacity)()
+        if capacity:
+            torch.cuda.synchronize()
+        self._ev = (c_void_p * max(1, 2 * capacity))(*[e.cuda_event for e in self.events])
+        self._kinds = (c_int32 * max(1, capacity))()
         self.struct = CkvTrace(ctypes.cast(self._ev, POINTER(c_void_p)),
                                ctypes.cast(self._kinds, POINTER(c_int32)), capacity, 0, 0)
 

@@ -219,6 +219,17 @@ __device__ __forceinline__ void tmem_order_after_wait(uint32_t (&r)[32]) {
                : "memory");
 }
 
+// ---------------------------------------------------------------- PDL
+// Programmatic dependent launch: let the next kernel of the stream start its
+// prologue now, and wait for the previous kernel's results before reading or
+// overwriting anything it may touch.  Without the launch attribute both are
+// no-ops.  Every kernel executes pdl_wait() before it exits, so completion of
+// a kernel implies completion of all kernels before it.
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ---------------------------------------------------------------- math
 // Hardware base-2 exponential (MUFU); ex2(-inf) = +0.
 __device__ __forceinline__ float ex2_approx(float x) {

@@ -14,6 +14,8 @@ constexpr int kGatherThreads = 256;
 constexpr int kRowsPerBlock = kGatherThreads / 32;
 
 __global__ void __launch_bounds__(kGatherThreads) gather_kernel(const __grid_constant__ GatherParams p) {
+  pdl_launch_dependents();
+  pdl_wait();  // the indices come from the select kernel
   const long long row = static_cast<long long>(blockIdx.x) * kRowsPerBlock + (threadIdx.x >> 5);
   const long long rows = static_cast<long long>(p.o_total) * p.num_kv_heads;
   if (row >= rows) return;
@@ -52,6 +54,11 @@ cudaError_t launch_gather(const GatherParams& p, long long rows, cudaStream_t st
   cfg.blockDim = dim3(kGatherThreads);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, gather_kernel, p);
 }
 

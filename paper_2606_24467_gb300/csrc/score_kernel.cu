@@ -69,13 +69,6 @@ __device__ __forceinline__ void wait_plain(uint32_t bar, uint32_t parity, uint64
   mbar_wait_bounded(bar, parity, &never, nullptr, timeout_ns);
 }
 
-// Logit validity on tiles that reach the window or the end of the sequence:
-// key `tok` is visible to query row q (window position w = q mod W) iff
-// tok < L and tok <= n + w.
-__device__ __forceinline__ bool causal_ok(int tok, int L, int n, int q, int W) {
-  return tok < L && tok <= n + (q % W);
-}
-
 template <bool kAccum, bool kSmallN>
 __global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
     score_kernel(const __grid_constant__ ScoreParams p) {
@@ -121,7 +114,11 @@ __global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
   if (kAccum) t1 = min(t1, (n + kTileTokens - 1) / kTileTokens);
   const int ntiles = max(t1 - t0, 0);
 
-  if (ntiles == 0) return;  // uniform over the CTA: nothing allocated yet
+  pdl_launch_dependents();
+  if (ntiles == 0) {  // uniform over the CTA: nothing allocated yet
+    pdl_wait();
+    return;
+  }
 
   // ------------------------------------------------------------ set-up
   if (threadIdx.x == 0) {
@@ -196,6 +193,7 @@ __global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
     fence_proxy_async_smem();
     for (int q = st_tid; q < kMaxQRows; q += kStagedThreads) sWpos[q] = q < N ? q % W : 0;
     if (kAccum) {
+      pdl_wait();  // the partials come from the pass-1 kernel
       // Merge the unit's pass-1 partials (fixed order => deterministic) into
       // the per-query bias m_q + log2 Z_q.
       for (int q = st_tid; q < N; q += kStagedThreads) {
@@ -457,6 +455,8 @@ __global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
         }
         // combine the 8 epilogue warps' (reference, sum) pairs per query
         named_bar_sync(kBarEpi, kEpiThreads);
+        // the previous kernels of the stream may still read the partials
+        pdl_wait();
         const int te = static_cast<int>(threadIdx.x) - kFirstEpiWarp * 32;
         if (te < N && !*abort_flag) {
           float m = kNegInf;
@@ -473,6 +473,7 @@ __global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
   }
 
   // ------------------------------------------------------------ teardown
+  pdl_wait();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
@@ -488,6 +489,11 @@ cudaError_t launch(const ScoreParams& p, int n_items, size_t smem, cudaStream_t 
   cfg.blockDim = dim3(Roles<kAccum>::kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, score_kernel<kAccum, kSmallN>, p);
 }
 

@@ -75,18 +75,40 @@ __device__ __forceinline__ T* unit_rank_ptr(T* ptr, int rank) {
   return ptr;
 }
 
-// One warp copies the K and V rows of token `tok` (position in its sequence)
-// to output row `orow`: lanes 0-15 move K, lanes 16-31 move V.
-__device__ __forceinline__ void copy_kv_row(const SelectParams& p, int seq0, int g, int tok,
-                                            long long orow, int lane) {
-  const long long src = static_cast<long long>(seq0 + tok) * p.tok_stride_v16 +
-                        static_cast<long long>(g) * p.head_stride_v16;
-  const long long dst = (orow * p.num_kv_heads + g) * (kHeadDim * 2 / 16);
-  const int part = lane & 15;
-  if (lane < 16) {
-    p.k_out[dst + part] = __ldg(p.k + src + part);
-  } else {
-    p.v_out[dst + part] = __ldg(p.v + src + part);
+// The whole CTA copies the K and V rows of `count` tokens to consecutive
+// output rows: token i is out[first + i] (a position in the sequence) and goes
+// to output row out0 + first + i.  Each thread moves 16-byte chunks, issuing
+// a batch of loads before the matching stores.
+__device__ __forceinline__ void copy_kv_rows(const SelectParams& p, int seq0, int g,
+                                             const int32_t* out, int out0, int first, int count) {
+  constexpr int kChunks = 2 * kHeadDim * 2 / 16;  // 16 K + 16 V chunks per token
+  constexpr int kBatch = 4;
+  const int total = count * kChunks;
+  for (int base = 0; base < total; base += kBatch * kSelThreads) {
+    uint4 v[kBatch];
+    long long dst[kBatch];
+    bool is_v[kBatch];
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      const int e = base + u * kSelThreads + static_cast<int>(threadIdx.x);
+      dst[u] = -1;
+      if (e < total) {
+        const int i = e / kChunks;
+        const int ch = e - i * kChunks;
+        const int tok = out[first + i];
+        is_v[u] = ch >= kChunks / 2;
+        const int part = ch & (kChunks / 2 - 1);
+        const long long src = static_cast<long long>(seq0 + tok) * p.tok_stride_v16 +
+                              static_cast<long long>(g) * p.head_stride_v16 + part;
+        v[u] = __ldg((is_v[u] ? p.v : p.k) + src);
+        dst[u] = (static_cast<long long>(out0 + first + i) * p.num_kv_heads + g) *
+                     (kHeadDim * 2 / 16) + part;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      if (dst[u] >= 0) (is_v[u] ? p.v_out : p.k_out)[dst[u]] = v[u];
+    }
   }
 }
 
@@ -96,7 +118,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   __shared__ uint32_t hist[2][kBins];
   __shared__ uint32_t ghist[kBins];
   __shared__ int s_gt[kSelWarps], s_eq[kSelWarps], s_eqbase[kSelWarps], s_selbase[kSelWarps];
-  __shared__ int s_bin, s_above, s_cta_gt, s_cta_eq;
+  __shared__ int s_bin, s_above, s_cta_gt, s_cta_eq, s_cta_first, s_cta_count;
 
   const int C = kCluster ? static_cast<int>(cg::this_cluster().num_blocks()) : 1;
   const int crank = kCluster ? static_cast<int>(cg::this_cluster().block_rank()) : 0;
@@ -124,6 +146,9 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   const bool in_smem = p.smem_slice;
   float* raw_s = s_dyn;                                  // [S + 2r] when in_smem
   float* pooled = in_smem ? s_dyn + S + 2 * r : p.pooled_ws + soff + lo;  // [len]
+
+  pdl_launch_dependents();
+  pdl_wait();  // raw scores come from the scoring kernel
 
   // 1. pooling ---------------------------------------------------------------
   const float fP = static_cast<float>(p.pool_width);
@@ -173,19 +198,23 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
     const int a0 = min(L, crank * per);
     const int a1 = min(L, a0 + per);
     for (int i = a0 + tid; i < a1; i += kSelThreads) out[i] = i;
-    if (p.gather) {
-      for (int i = a0 + warp; i < a1; i += kSelWarps) copy_kv_row(p, seq0, g, i, out0 + i, lane);
+    if (p.gather && a1 > a0) {
+      __syncthreads();  // the indices written above are read back by the copy
+      copy_kv_rows(p, seq0, g, out, out0, a0, a1 - a0);
     }
     return;  // uniform over the cluster: no cluster barrier is pending
   }
   const int k = kept - W;  // 0 <= k < n
   if (crank == C - 1) {
     for (int w = tid; w < W; w += kSelThreads) out[k + w] = n + w;
-    if (p.gather) {
-      for (int w = warp; w < W; w += kSelWarps) copy_kv_row(p, seq0, g, n + w, out0 + k + w, lane);
-    }
   }
-  if (k == 0) return;  // window only (uniform over the cluster)
+  if (k == 0) {  // window only (uniform over the cluster)
+    if (p.gather && crank == C - 1) {
+      __syncthreads();
+      copy_kv_rows(p, seq0, g, out, out0, k, W);
+    }
+    return;
+  }
   __syncthreads();
   const uint32_t* keys = reinterpret_cast<const uint32_t*>(pooled);
 
@@ -211,8 +240,12 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
     }
     unit_barrier<kCluster>();
     for (int b = tid; b < kBins; b += kSelThreads) {
+      uint32_t part[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) part[q] = q < C ? unit_rank_ptr<kCluster>(h, q)[b] : 0u;
       uint32_t tot = 0u;
-      for (int q = 0; q < C; ++q) tot += unit_rank_ptr<kCluster>(h, q)[b];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) tot += part[q];
       ghist[b] = tot;
     }
     __syncthreads();
@@ -292,9 +325,14 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
     const int take = min(max(need_eq - w_eq_before, 0), e);
     const int sel = (lane < kSelWarps ? s_gt[lane] : 0) + take;
     const int sel_before = warp_exclusive_scan(sel, lane);  // every lane takes part
+    const int sel_total = __shfl_sync(0xffffffffu, sel_before + sel, 31);
     if (lane < kSelWarps) {
       s_eqbase[lane] = w_eq_before;
       s_selbase[lane] = gt_before + take_before + sel_before;
+    }
+    if (lane == 0) {
+      s_cta_first = gt_before + take_before;  // this CTA's first output slot
+      s_cta_count = sel_total;                // and how many it fills
     }
   }
   unit_barrier<kCluster>();  // no CTA leaves while others may still read its shared memory
@@ -311,18 +349,16 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
     const uint32_t msel = mgt | __ballot_sync(0xffffffffu, take_eq);
     const int o = pos + __popc(msel & lanemask_lt(lane));
     if ((msel & (1u << lane)) && o < k) out[o] = lo + i;
-    if (p.gather) {
-      uint32_t m = msel;
-      int oo = pos;
-      while (m) {
-        const int bit = __ffs(m) - 1;
-        m &= m - 1;
-        if (oo < k) copy_kv_row(p, seq0, g, lo + b0 + bit, out0 + oo, lane);
-        ++oo;
-      }
-    }
     pos += __popc(msel);
     eq_seen += __popc(meq);
+  }
+  if (p.gather) {
+    // 5. copy this CTA's retained rows (and the window, last CTA)
+    __syncthreads();  // the indices written above are read back by the copy
+    const int cta_first = s_cta_first;
+    const int cta_count = min(k - cta_first, s_cta_count);
+    if (cta_count > 0) copy_kv_rows(p, seq0, g, out, out0, cta_first, cta_count);
+    if (crank == C - 1) copy_kv_rows(p, seq0, g, out, out0, k, W);
   }
 }
 
@@ -345,14 +381,17 @@ cudaError_t launch_select(const SelectParams& p, int n_units, size_t smem, cudaS
   cfg.blockDim = dim3(kSelThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  if (p.cluster <= 1) return cudaLaunchKernelEx(&cfg, select_kernel<false>, p);
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = static_cast<unsigned>(p.cluster);
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  if (p.cluster <= 1) return cudaLaunchKernelEx(&cfg, select_kernel<false>, p);
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = static_cast<unsigned>(p.cluster);
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, select_kernel<true>, p);
 }
 

@@ -199,3 +199,56 @@ def test_full_size_layer(cuda_device, name, layer):
     _, res, ties = check(d, cfg.window, cfg.pool_width, cuda_device)
     n_units = len(res.units)
     assert ties <= max(4, n_units)
+
+
+def test_graph_captured_multilayer_step_matches(cuda_device):
+    """Several layers back to back in one CUDA graph: consecutive kernels
+    overlap (programmatic dependent launch) and share one workspace; every
+    layer must still equal its own eager result and the oracle."""
+    dev = cuda_device
+    cfg = wl.get("c2").scaled(seq_len=6000, n_layers=4)
+    lengths = wl.sequence_lengths(cfg)
+    masks = wl.srh_masks(cfg)
+    budgets = wl.layer_budgets(cfg, lengths)
+    layers = [wl.make_layer(cfg, l, lengths=lengths, masks=masks, budgets=budgets)
+              for l in range(cfg.n_layers)]
+    dl = [{k: lay[k].to(dev) for k in ("q_win", "k", "v")} for lay in layers]
+    probs = [ckv.Problem(d["q_win"], d["k"], lay["cu_seqlens"], cfg.window, cfg.pool_width)
+             for d, lay in zip(dl, layers)]
+    ws = ckv.workspace(probs[0], dev)
+    outs = [ckv.LayerOutputs(probs[l], budgets[l], 128, torch.bfloat16, dev)
+            for l in range(cfg.n_layers)]
+
+    def step():
+        for l, (d, lay) in enumerate(zip(dl, layers)):
+            o = outs[l]
+            ckv.compress_layer(probs[l], d["q_win"], d["k"], d["v"], lay["srh_mask"],
+                               lay["budgets"], o.indices, o.k_out, o.v_out, ws, raw=o.raw,
+                               pooled=o.pooled)
+
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        step()
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    eager = [(o.raw.clone(), o.indices.clone(), o.k_out.clone()) for o in outs]
+    for o in outs:
+        o.raw.zero_()
+        o.indices.zero_()
+        o.k_out.zero_()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, capture_error_mode="thread_local"):
+        step()
+    for _ in range(3):
+        graph.replay()
+    torch.cuda.synchronize()
+    assert ckv.read_device_status(ws) == 0
+    for l, o in enumerate(outs):
+        raw_e, idx_e, k_e = eager[l]
+        assert torch.equal(o.raw, raw_e), l
+        assert torch.equal(o.indices, idx_e), l
+        assert torch.equal(o.k_out.view(torch.int16), k_e.view(torch.int16)), l
+        res = run_oracle(layers[l], cfg.window, cfg.pool_width)
+        compare.check_layer(res, o.raw.cpu().numpy(), o.pooled.cpu().numpy(),
+                            o.indices.cpu().numpy(), layers[l]["cu_seqlens"], cfg.window)
