@@ -37,7 +37,7 @@ import workloads as wl  # noqa: E402
 METRIC = ("prompt tokens compressed/sec per GB300 and achieved HBM GB/s vs peak at "
           "L=32K–128K")
 UNIT = "tokens/s"
-PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "score_stats_llama8b_L32k.md")
+PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "score_llama8b_L32k.md")
 KERNEL_SOURCES = ["paper_2606_24467_gb300/csrc/score_kernel.cu",
                   "paper_2606_24467_gb300/csrc/ckv_device.cuh",
                   "paper_2606_24467_gb300/csrc/ckv_params.h",
@@ -168,7 +168,7 @@ def kernel_source_hash() -> str:
 
 
 def profiled_traffic(workload: str):
-    """DRAM bytes per launch of the pass-1 scoring kernel from the committed
+    """DRAM bytes per launch of the scoring kernel from the committed
     ncu summary, if it was taken on the current kernel sources."""
     try:
         text = open(PROFILE_TRAFFIC).read()
@@ -309,12 +309,12 @@ def run_ours(args):
         per_kind.setdefault(kind, []).append(ms)
     step_bytes, score_bytes = algorithmic_bytes(cfg, layers, lengths)
     peak, peak_src = measured_peaks()
-    stats_ms = per_kind.get("score_stats", [float("nan")])
+    stats_ms = per_kind.get("score", [float("nan")])
     n_stats = len(stats_ms)
     avg_stats_ms = sum(stats_ms) / max(n_stats, 1)
     bytes_per_launch = score_bytes / max(n_stats, 1)
     achieved = bytes_per_launch / (avg_stats_ms / 1e3) / 1e9
-    roofline = {"bound": "hbm", "kernel": "score_stats (pass 1)", "achieved": round(achieved, 1),
+    roofline = {"bound": "hbm", "kernel": "score (one pass over K)", "achieved": round(achieved, 1),
                 "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4),
                 "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
                 else "fallback 6.8 TB/s",

@@ -89,8 +89,8 @@ enum { CKV_POOL_AVG = 0 };
 
 /* Kernel kinds reported through ckv_trace. */
 enum {
-  CKV_KERNEL_SCORE_STATS = 1,   /* scoring pass 1: per-query softmax max / normaliser */
-  CKV_KERNEL_SCORE_ACCUM = 2,   /* scoring pass 2: normalised attention summed per token */
+  CKV_KERNEL_SCORE = 1,         /* window logits over K: softmax statistics + exponent table */
+  CKV_KERNEL_COMBINE = 2,       /* normalised scores summed over queries, then pooled */
   CKV_KERNEL_SELECT = 3,        /* pooling + top-k + window append */
   CKV_KERNEL_GATHER = 4         /* retained K/V rows -> compressed cache */
 };
@@ -149,6 +149,8 @@ int compresskv_output_layout(const ckv_problem* p, const int32_t* budgets,
 /* Step 1 (Sec. 3.3): raw prefix scores.
  * srh_mask: host uint8 [num_q_heads], non-zero = SRH head of this layer.
  * raw_scores: device float, score layout, written for every prefix token.
+ * The per-query attention weights pass through an fp16 table scaled so
+ * that each weight keeps a relative error below 2^-11 (plus the fp32 sums).
  * Per unit, |S_g| * W must not exceed 256 query rows (CKV_ERR_UNSUPPORTED). */
 int compresskv_score(const ckv_problem* p, const void* q_win, const void* k,
                      const uint8_t* srh_mask, float* raw_scores,
@@ -175,8 +177,9 @@ int compresskv_gather(const ckv_problem* p, const int32_t* indices, const int32_
                       void* workspace, void* stream);
 
 /* Steps 1-4 fused for one layer: score, select, gather.
- * raw_scores / pooled_scores are optional outputs (NULL: kept in the
- * workspace).  cu_out: host int32 [batch+1], written. */
+ * raw_scores / pooled_scores are optional outputs in score layout (NULL: raw
+ * scores are not materialised, pooled scores stay in the workspace).
+ * cu_out: host int32 [batch+1], written. */
 int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const void* k,
                               const void* v, const uint8_t* srh_mask, const int32_t* budgets,
                               int32_t* indices, int32_t* cu_out, void* k_out, void* v_out,

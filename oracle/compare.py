@@ -25,9 +25,10 @@ def check_scores(name, gpu, ref, rtol=RTOL, atol=ATOL):
     ref = np.asarray(ref, np.float64)
     assert gpu.shape == ref.shape, f"{name}: shape {gpu.shape} vs {ref.shape}"
     err = np.abs(gpu - ref)
-    bad = err > rtol * np.abs(ref) + atol
+    bad = ~(err <= rtol * np.abs(ref) + atol)  # NaN or inf anywhere fails
     if bad.any():
-        i = np.unravel_index(np.argmax(err - rtol * np.abs(ref)), err.shape)
+        i = np.unravel_index(np.argmax(np.where(bad, np.nan_to_num(err, nan=np.inf), -np.inf)),
+                             err.shape)
         raise AssertionError(f"{name}: {int(bad.sum())} of {bad.size} outside tolerance; "
                              f"worst at {i}: gpu={gpu[i]!r} oracle={ref[i]!r}")
 

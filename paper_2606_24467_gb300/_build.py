@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB_PATH = os.path.join(OUT_DIR, "libcompresskv.so")
-SOURCES = ["api.cu", "score_kernel.cu", "select_kernel.cu", "gather_kernel.cu"]
+SOURCES = ["api.cu", "score_kernel.cu", "combine_kernel.cu", "select_kernel.cu", "gather_kernel.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

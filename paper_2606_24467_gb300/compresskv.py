@@ -30,7 +30,7 @@ STATIC_SCRATCH_BYTES = 16 * 1024 * 1024
 CKV_DTYPE_F16 = 0
 CKV_DTYPE_BF16 = 1
 CKV_POOL_AVG = 0
-KERNEL_KINDS = {1: "score_stats", 2: "score_accum", 3: "select", 4: "gather"}
+KERNEL_KINDS = {1: "score", 2: "combine", 3: "select", 4: "gather"}
 
 EXPORTED = (
     "compresskv_workspace_size",

@@ -20,12 +20,14 @@ using namespace ckv;
 namespace {
 
 constexpr size_t kStatusBytes = 256;
-// Share of the L2 that the K of the units scored together may occupy, so
-// that pass 2 finds K in L2.
-#ifndef CKV_L2_SET_FRACTION
-#define CKV_L2_SET_FRACTION 0.6
+// Units are scored in sets whose exponent tables (bounded with every head of
+// a group counted as SRH) take at most this many bytes; one set's table is
+// written by the scoring kernel and read back by the combine kernel, ideally
+// while still in L2.
+#ifndef CKV_EXPO_SET_BYTES
+#define CKV_EXPO_SET_BYTES (64ll << 20)
 #endif
-constexpr double kL2SetFraction = CKV_L2_SET_FRACTION;
+constexpr long long kExpoSetBytes = CKV_EXPO_SET_BYTES;
 constexpr size_t kPartialBytes = static_cast<size_t>(kMaxItems) * kMaxQRows * sizeof(float2);
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
@@ -35,6 +37,7 @@ struct DeviceFacts {
   int sms = 0;
   int smem_optin = 0;
   long long l2_bytes = 0;
+  size_t combine_smem_max = 0;  // dynamic shared memory the combine kernel may use
   bool smem_attr_set = false;
 };
 
@@ -61,6 +64,8 @@ int device_facts(DeviceFacts** out) {
       return CKV_ERR_CUDA;
     f.smem_optin = optin;
     if (score_set_smem_limit(static_cast<size_t>(optin)) != cudaSuccess) return CKV_ERR_CUDA;
+    if (combine_set_smem_limit(static_cast<size_t>(optin), &f.combine_smem_max) != cudaSuccess)
+      return CKV_ERR_CUDA;
     if (select_set_smem_limit(static_cast<size_t>(select_max_smem_floats()) * 4) != cudaSuccess)
       return CKV_ERR_CUDA;
     f.smem_attr_set = true;
@@ -146,27 +151,79 @@ int output_layout(const Info& I, const int32_t* budgets, std::vector<int>& cu_ou
   return CKV_OK;
 }
 
+// Units (s, g) with a prefix to score, in (s, g) order, cut into sets.  The
+// cut uses the largest exponent row any SRH mask can give (all G heads of a
+// group), so the workspace size depends on the problem alone.
+struct UnitSet {
+  int u0, u1;             // units [u0, u1) of the unit list
+  long long expo_elems;   // fp16 elements of the set's exponent table (bound)
+  long long ref_floats;   // floats of its reference table (bound)
+};
+
+int expo_row_bound(const Info& I) { return expo_stride(std::min(I.G * I.W, kMaxQRows)); }
+
+void plan_sets(const Info& I, std::vector<UnitSet>& sets) {
+  sets.clear();
+  const long long nr = expo_row_bound(I);
+  int u = 0, u0 = 0;
+  long long e = 0, r = 0;
+  for (int s = 0; s < I.B; ++s) {
+    if (I.n[s] <= 0) continue;
+    const long long ue = static_cast<long long>(I.n[s]) * nr;
+    const long long ur =
+        static_cast<long long>((I.len[s] + kTileTokens - 1) / kTileTokens) * kQuarters * nr;
+    for (int g = 0; g < I.Hkv; ++g, ++u) {
+      if (u > u0 && (2 * (e + ue) > kExpoSetBytes || u - u0 >= kMaxItems / 2)) {
+        sets.push_back({u0, u, e, r});
+        u0 = u;
+        e = r = 0;
+      }
+      e += ue;
+      r += ur;
+    }
+  }
+  if (u > u0) sets.push_back({u0, u, e, r});
+}
+
 struct Workspace {
   int* status = nullptr;
   float2* partials = nullptr;
-  float* raw = nullptr;
-  float* pooled = nullptr;
+  float* pooled = nullptr;   // score layout
+  uint16_t* expo = nullptr;  // one set's exponent table
+  float* refs = nullptr;     // one set's reference table
 };
 
-size_t workspace_bytes(const Info& I) {
-  const size_t scores = align256(static_cast<size_t>(I.Hkv) * I.p_total * sizeof(float));
-  return kStatusBytes + kPartialBytes + 2 * scores;
+struct WorkspaceLayout {
+  size_t pooled, expo, refs, total;
+};
+
+WorkspaceLayout workspace_layout(const Info& I) {
+  std::vector<UnitSet> sets;
+  plan_sets(I, sets);
+  long long e = 0, r = 0;
+  for (const UnitSet& S : sets) {
+    e = std::max(e, S.expo_elems);
+    r = std::max(r, S.ref_floats);
+  }
+  WorkspaceLayout W;
+  W.pooled = kStatusBytes + kPartialBytes;
+  W.expo = W.pooled + align256(static_cast<size_t>(I.Hkv) * I.p_total * sizeof(float));
+  W.refs = W.expo + align256(static_cast<size_t>(e) * sizeof(uint16_t));
+  W.total = W.refs + align256(static_cast<size_t>(r) * sizeof(float));
+  return W;
 }
 
+size_t workspace_bytes(const Info& I) { return workspace_layout(I).total; }
+
 int carve(const Info& I, void* ws, size_t bytes, Workspace& out) {
-  if (!ws || bytes < workspace_bytes(I) || (reinterpret_cast<uintptr_t>(ws) & 255u))
-    return CKV_ERR_WORKSPACE;
+  const WorkspaceLayout W = workspace_layout(I);
+  if (!ws || bytes < W.total || (reinterpret_cast<uintptr_t>(ws) & 255u)) return CKV_ERR_WORKSPACE;
   char* b = static_cast<char*>(ws);
-  const size_t scores = align256(static_cast<size_t>(I.Hkv) * I.p_total * sizeof(float));
   out.status = reinterpret_cast<int*>(b);
   out.partials = reinterpret_cast<float2*>(b + kStatusBytes);
-  out.raw = reinterpret_cast<float*>(b + kStatusBytes + kPartialBytes);
-  out.pooled = reinterpret_cast<float*>(b + kStatusBytes + kPartialBytes + scores);
+  out.pooled = reinterpret_cast<float*>(b + W.pooled);
+  out.expo = reinterpret_cast<uint16_t*>(b + W.expo);
+  out.refs = reinterpret_cast<float*>(b + W.refs);
   return CKV_OK;
 }
 
@@ -263,9 +320,13 @@ int make_k_map(const Info& I, const ckv_problem* p, const void* k, CUtensorMap* 
   return r == CUDA_SUCCESS ? CKV_OK : CKV_ERR_INVALID_ARG;
 }
 
+// Scores every unit: per set, the scoring kernel (one pass over K) and the
+// combine kernel, which leaves pooled scores (and raw scores when `raw` is
+// given) in score layout.
 int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void* k,
-              const uint8_t* mask, float* raw, const Workspace& ws, cudaStream_t stream) {
-  if (!q_win || !k || !raw) return CKV_ERR_INVALID_ARG;
+              const uint8_t* mask, float* raw, float* pooled, const Workspace& ws,
+              cudaStream_t stream) {
+  if (!q_win || !k || !pooled) return CKV_ERR_INVALID_ARG;
   if (!aligned16(q_win) || !aligned16(k)) return CKV_ERR_INVALID_ARG;
   SrhLists S;
   int rc = srh_lists(I, mask, S);
@@ -274,12 +335,15 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
   if ((rc = device_facts(&F)) != CKV_OK) return rc;
   if (I.p_total == 0) return CKV_OK;
 
-  static thread_local ScoreParams P;  // large (about 17 KB): kept off the stack
+  static thread_local ScoreParams P;    // large (about 17 KB): kept off the stack
+  static thread_local CombineParams C;  // likewise
   std::memset(&P, 0, sizeof(P));
+  std::memset(&C, 0, sizeof(C));
   if ((rc = make_k_map(I, p, k, &P.tmap_k)) != CKV_OK) return rc;
   P.q = static_cast<const uint16_t*>(q_win);
   P.partials = ws.partials;
-  P.raw = raw;
+  P.expo = ws.expo;
+  P.refs = ws.refs;
   P.status = ws.status;
   P.q_bs = p->q_batch_stride;
   P.q_hs = p->q_head_stride;
@@ -287,45 +351,43 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
   P.c = static_cast<float>(static_cast<double>(I.scale) * 1.4426950408889634);
   P.window = I.W;
   P.num_kv_heads = I.Hkv;
-  P.p_total = static_cast<int>(I.p_total);
   P.is_bf16 = I.bf16 ? 1 : 0;
   P.use_evict_hint = 1;
+  C.partials = ws.partials;
+  C.expo = ws.expo;
+  C.refs = ws.refs;
+  C.raw_out = raw;
+  C.pooled = pooled;
+  C.window = I.W;
+  C.pool_width = I.P;
+  C.num_kv_heads = I.Hkv;
+  C.p_total = static_cast<int>(I.p_total);
   for (int s = 0; s <= I.B; ++s) {
     P.cu_seqlens[s] = I.cu[s];
-    P.cu_prefix[s] = I.cu_prefix[s];
+    C.cu_seqlens[s] = I.cu[s];
+    C.cu_prefix[s] = I.cu_prefix[s];
   }
-  for (int g = 0; g <= I.Hkv; ++g) P.srh_off[g] = S.off[g];
+  for (int g = 0; g <= I.Hkv; ++g) P.srh_off[g] = C.srh_off[g] = S.off[g];
   for (size_t h = 0; h < S.heads.size(); ++h) P.srh_heads[h] = S.heads[h];
 
-  // Units (s, g) with a prefix to score, grouped into sets whose K fits in
-  // about half of the L2, so that pass 2 re-reads K from L2.
-  struct Unit { int s, g, tiles; };
+  struct Unit { int s, g, tiles, quarters; };
   std::vector<Unit> units;
   for (int s = 0; s < I.B; ++s)
     if (I.n[s] > 0)
       for (int g = 0; g < I.Hkv; ++g)
-        units.push_back({s, g, (I.len[s] + kTileTokens - 1) / kTileTokens});
-  const long long set_budget =
-      std::max<long long>(static_cast<long long>(F->l2_bytes * kL2SetFraction), 1LL << 20);
-  size_t u0 = 0;
+        units.push_back({s, g, (I.len[s] + kTileTokens - 1) / kTileTokens, (I.n[s] + 31) / 32});
+  std::vector<UnitSet> sets;
+  plan_sets(I, sets);
   Tracer tr{p->trace, stream};
-  while (u0 < units.size()) {
-    size_t u1 = u0;
-    long long bytes = 0;
-    while (u1 < units.size()) {
-      const long long ub = static_cast<long long>(units[u1].tiles) * kTileBytes;
-      if (u1 > u0 && (bytes + ub > set_budget || static_cast<long long>(u1 - u0) >= kMaxItems / 2))
-        break;
-      bytes += ub;
-      ++u1;
-    }
-    // Work items: one wave of exactly max(#units, #SMs) CTAs.  A tile of a
-    // unit costs about (64 + query rows) (the epilogue scales with the rows);
-    // every unit gets one item, the remaining items go one at a time to the
-    // unit with the largest work per item, then each unit's tiles are split
-    // into balanced ranges.
+  for (const UnitSet& set : sets) {
+    const int u0 = set.u0;
+    const int nu = set.u1 - set.u0;
+    // Score work items: one wave of exactly max(#units, #SMs) CTAs.  A tile
+    // of a unit costs about (64 + query rows) (the epilogue scales with the
+    // rows); every unit gets one item, the remaining items go one at a time
+    // to the unit with the largest work per item, then each unit's tiles are
+    // split into balanced ranges.
     auto cost = [&](const Unit& U) { return 64LL + ((S.rows[U.g] + 15) & ~15); };
-    const int nu = static_cast<int>(u1 - u0);
     std::vector<int> cnt(nu, 1);
     std::vector<long long> uw(nu);
     for (int u = 0; u < nu; ++u)
@@ -340,11 +402,21 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
       if (best < 0) break;
       ++cnt[best];
     }
-    int n_items = 0;
+    // Combine items: chunks of 32-token quarters, about four CTAs per SM.
+    long long quarters = 0;
+    for (int u = 0; u < nu; ++u) quarters += units[u0 + u].quarters;
+    const long long ctarget = std::max(1, std::min(kMaxItems - nu, 4 * F->sms));
+    const int chunk_q = static_cast<int>(std::max(8LL, (quarters + ctarget - 1) / ctarget));
+    const size_t csmem = combine_smem_bytes(chunk_q * 32, I.P);
+    if (csmem > F->combine_smem_max) return CKV_ERR_UNSUPPORTED;
+
+    int n_items = 0, n_comb = 0;
     int max_rows = 16;
+    uint32_t eoff = 0, roff = 0;
     for (int u = 0; u < nu; ++u) {
       const Unit& U = units[u0 + u];
       const int c_u = cnt[u];
+      const int nr = expo_stride(S.rows[U.g]);
       if (n_items + c_u > kMaxItems) return CKV_ERR_UNSUPPORTED;
       for (int c = 0; c < c_u; ++c) {
         WorkItem& it = P.items[n_items + c];
@@ -354,11 +426,23 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
         it.t1 = static_cast<uint16_t>(static_cast<long long>(U.tiles) * (c + 1) / c_u);
         it.first = static_cast<uint16_t>(n_items);
         it.count = static_cast<uint16_t>(c_u);
+        it.eoff = eoff;
+        it.roff = roff;
+      }
+      for (int q0 = 0; q0 < U.quarters; q0 += chunk_q) {
+        if (n_comb >= kMaxItems) return CKV_ERR_UNSUPPORTED;
+        WorkItem& it = C.items[n_comb++];
+        it = P.items[n_items];
+        it.t0 = static_cast<uint16_t>(q0);
+        it.t1 = static_cast<uint16_t>(std::min(U.quarters, q0 + chunk_q));
       }
       n_items += c_u;
+      eoff += static_cast<uint32_t>(I.n[U.s]) * static_cast<uint32_t>(nr);
+      roff += static_cast<uint32_t>(U.tiles * kQuarters * nr);
       max_rows = std::max(max_rows, (S.rows[U.g] + 15) & ~15);
     }
     P.n_items = n_items;
+    C.n_items = n_comb;
     P.q_half_bytes = ((max_rows * 128) + 1023) & ~1023;
     P.small_n = max_rows <= 64 ? 1 : 0;
     P.stages = kStages;
@@ -366,23 +450,23 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
            score_smem_bytes(P.q_half_bytes, P.stages) > static_cast<size_t>(F->smem_optin))
       --P.stages;
     const size_t smem = score_smem_bytes(P.q_half_bytes, P.stages);
-    rc = traced(tr, CKV_KERNEL_SCORE_STATS,
-                [&] { return launch_score_stats(P, n_items, smem, stream); });
+    rc = traced(tr, CKV_KERNEL_SCORE, [&] { return launch_score(P, n_items, smem, stream); });
     if (rc != CKV_OK) return rc;
-    rc = traced(tr, CKV_KERNEL_SCORE_ACCUM,
-                [&] { return launch_score_accum(P, n_items, smem, stream); });
+    rc = traced(tr, CKV_KERNEL_COMBINE,
+                [&] { return launch_combine(C, n_comb, csmem, stream); });
     if (rc != CKV_OK) return rc;
-    u0 = u1;
   }
   return CKV_OK;
 }
 
 // ------------------------------------------------------------------ select / gather
-int run_select(const ckv_problem* p, const Info& I, const float* raw, const std::vector<int>& cu_out,
-               int32_t* indices, float* pooled, const Workspace& ws, cudaStream_t stream,
-               const void* k = nullptr, const void* v = nullptr, void* k_out = nullptr,
-               void* v_out = nullptr) {
-  if (!raw && I.p_total > 0) return CKV_ERR_INVALID_ARG;
+// Pooling (unless `pooled_in` holds the pooled scores already), top-k and
+// window append, optionally fused with the K/V gather.
+int run_select(const ckv_problem* p, const Info& I, const float* raw, const float* pooled_in,
+               const std::vector<int>& cu_out, int32_t* indices, float* pooled,
+               const Workspace& ws, cudaStream_t stream, const void* k = nullptr,
+               const void* v = nullptr, void* k_out = nullptr, void* v_out = nullptr) {
+  if (!raw && !pooled_in && I.p_total > 0) return CKV_ERR_INVALID_ARG;
   if (!indices && cu_out[I.B] > 0) return CKV_ERR_INVALID_ARG;
   const bool gather = k != nullptr;
   if (gather && cu_out[I.B] > 0) {
@@ -393,11 +477,12 @@ int run_select(const ckv_problem* p, const Info& I, const float* raw, const std:
   DeviceFacts* F = nullptr;
   int rc = device_facts(&F);
   if (rc != CKV_OK) return rc;
-  if (cu_out[I.B] == 0 && !pooled) return CKV_OK;
+  if (cu_out[I.B] == 0 && (!pooled || pooled_in)) return CKV_OK;
   static thread_local SelectParams P;
   std::memset(&P, 0, sizeof(P));
   P.raw = raw;
-  P.pooled_out = pooled;
+  P.pooled_in = pooled_in;
+  P.pooled_out = pooled_in ? nullptr : pooled;
   P.pooled_ws = ws.pooled;
   P.indices = indices;
   P.status = ws.status;
@@ -504,7 +589,9 @@ int compresskv_score(const ckv_problem* p, const void* q_win, const void* k,
   if (rc != CKV_OK) return rc;
   Workspace ws;
   if ((rc = carve(I, workspace, workspace_bytes, ws)) != CKV_OK) return rc;
-  return run_score(p, I, q_win, k, srh_mask, raw_scores, ws, static_cast<cudaStream_t>(stream));
+  if (!raw_scores) return CKV_ERR_INVALID_ARG;
+  return run_score(p, I, q_win, k, srh_mask, raw_scores, ws.pooled, ws,
+                   static_cast<cudaStream_t>(stream));
 }
 
 int compresskv_select(const ckv_problem* p, const float* raw_scores, const int32_t* budgets,
@@ -519,7 +606,7 @@ int compresskv_select(const ckv_problem* p, const float* raw_scores, const int32
   Workspace ws;
   if ((rc = carve(I, workspace, workspace_bytes, ws)) != CKV_OK) return rc;
   std::copy(co.begin(), co.end(), cu_out);
-  return run_select(p, I, raw_scores, co, indices, pooled_scores, ws,
+  return run_select(p, I, raw_scores, nullptr, co, indices, pooled_scores, ws,
                     static_cast<cudaStream_t>(stream));
 }
 
@@ -560,10 +647,10 @@ int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const voi
   SrhLists S;
   if ((rc = srh_lists(I, srh_mask, S)) != CKV_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  float* raw = raw_scores ? raw_scores : ws.raw;
+  float* pooled = pooled_scores ? pooled_scores : ws.pooled;
   std::copy(co.begin(), co.end(), cu_out);
-  if ((rc = run_score(p, I, q_win, k, srh_mask, raw, ws, st)) != CKV_OK) return rc;
-  return run_select(p, I, raw, co, indices, pooled_scores, ws, st, k, v, k_out, v_out);
+  if ((rc = run_score(p, I, q_win, k, srh_mask, raw_scores, pooled, ws, st)) != CKV_OK) return rc;
+  return run_select(p, I, nullptr, pooled, co, indices, nullptr, ws, st, k, v, k_out, v_out);
 }
 
 int compresskv_read_device_status(const void* workspace, void* stream, int32_t* status) {

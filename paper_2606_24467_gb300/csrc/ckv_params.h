@@ -25,35 +25,57 @@ constexpr int CKV_DEV_ERR_INDEX = -8;
 constexpr int kTileBytes = kTileTokens * kHeadDim * 2;   // 32 KiB
 constexpr int kHalfTileBytes = kTileBytes / 2;           // 64 columns (128 B) of d
 constexpr int kQHalfBytes = kMaxQRows * 128;             // Q rows, one 64-column half
+constexpr int kQuarters = kTileTokens / 32;              // 32-token groups per tile (one warp each)
 
 // One score work item: a contiguous range of K tiles of one unit.  `first`
-// and `count` locate all items of the same unit in the item table (pass 2
-// merges their partial softmax statistics).
+// and `count` locate all items of the same unit in the item table (the
+// combine step merges their partial softmax statistics); `eoff` / `roff` are
+// the unit's offsets in the exponent table (fp16 elements) and in the
+// reference table (floats).
 struct WorkItem {
   uint16_t seq, group, t0, t1, first, count;
+  uint32_t eoff, roff;
 };
 
 struct ScoreParams {
   CUtensorMap tmap_k;          // 3-D map over K: (d, kv head, token)
   const uint16_t* q;           // window queries (f16/bf16 bits)
   float2* partials;            // [n_items][kMaxQRows]: (max z*c, sum 2^(z*c - max))
-  float* raw;                  // score layout [num_kv_heads][p_total]
+  uint16_t* expo;              // fp16 2^(z*c - ref) per prefix token and query row
+  float* refs;                 // per (tile, quarter, query row): the ref used for expo
   int* status;                 // device status word
   long long q_bs, q_hs, q_ws;  // window-query strides, elements
   float c;                     // scale * log2(e)
-  int window, num_kv_heads, p_total, n_items, is_bf16, use_evict_hint;
+  int window, num_kv_heads, n_items, is_bf16, use_evict_hint;
   int q_half_bytes;            // bytes of one 64-column half of the Q rows in shared memory
   int small_n;                 // 1: every unit of the launch has at most 64 query rows
   int stages;                  // K tiles in the shared-memory ring (2..kStages)
   int cu_seqlens[kMaxBatch + 1];
-  int cu_prefix[kMaxBatch + 1];
   uint16_t srh_off[kMaxKvHeads + 1];   // SRH heads of group g: srh_heads[srh_off[g] .. srh_off[g+1])
   uint8_t srh_heads[kMaxQHeads];
   WorkItem items[kMaxItems];
 };
 
+// Combine: normalised scores from the stored exponents, then pooling.
+struct CombineParams {
+  const float2* partials;
+  const uint16_t* expo;
+  const float* refs;
+  float* raw_out;              // optional, score layout
+  float* pooled;               // score layout (caller's buffer or workspace)
+  int window, pool_width, num_kv_heads, p_total, n_items;
+  int cu_seqlens[kMaxBatch + 1];
+  int cu_prefix[kMaxBatch + 1];
+  uint16_t srh_off[kMaxKvHeads + 1];
+  WorkItem items[kMaxItems];
+};
+
+// Row stride (fp16 elements) of the exponent table for `rows` query rows.
+__host__ __device__ constexpr int expo_stride(int rows) { return (rows + 7) & ~7; }
+
 struct SelectParams {
-  const float* raw;            // score layout
+  const float* raw;            // score layout (pooled here when pooled_in is null)
+  const float* pooled_in;      // already pooled scores (score layout), or null
   float* pooled_out;           // optional, score layout
   float* pooled_ws;            // workspace copy of pooled scores, score layout
   int32_t* indices;            // [num_kv_heads][o_total]
@@ -87,12 +109,16 @@ struct GatherParams {
 };
 
 // Host-side launchers (defined next to each kernel).
-cudaError_t launch_score_stats(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s);
-cudaError_t launch_score_accum(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s);
+cudaError_t launch_score(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s);
+cudaError_t launch_combine(const CombineParams& p, int n_items, size_t smem, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, int n_units, size_t smem, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, long long rows, cudaStream_t s);
 size_t score_smem_bytes(int q_half_bytes, int stages);
 cudaError_t score_set_smem_limit(size_t bytes);
+size_t combine_smem_bytes(int chunk_tokens, int pool_width);
+// Sets the combine kernel's dynamic shared-memory limit to what `optin`
+// leaves beside its static shared memory and returns that limit.
+cudaError_t combine_set_smem_limit(size_t optin, size_t* dynamic_max);
 cudaError_t select_set_smem_limit(size_t bytes);
 int select_max_smem_floats();
 

@@ -1,33 +1,35 @@
 // Observation-window scoring (CompressKV Sec. 3.3; SnapKV-style window of
-// Sec. 4) on sm_103a tensor cores.
+// Sec. 4) on sm_103a tensor cores, in one pass over K.
 //
 // For one unit (sequence s, KV group g) let Q_S be the |S_g|*W window-query
 // rows of the group's SRH heads and K the unit's L keys.  With
-// z = <q, k> * scale and c = log2(e):
-//   pass 1 (stats):  m_q = max_j z_qj*c,  Z_q = sum_{j <= p_q} 2^(z_qj*c - m_q)
-//                    over the causal keys j <= p_q = L - W + w(q);
-//   pass 2 (accum):  raw_j = sum_q 2^(z_qj*c - m_q - log2 Z_q)  for j < n = L - W,
-// i.e. the softmax attention of every SRH window query summed over queries,
-// for every prefix token.  The normaliser Z_q needs all keys before any
-// attention weight is final, hence two passes; pass 2 re-reads K while it is
-// still in L2 (the host sizes the units launched together to the L2).
+// z = <q, k> * scale, c = log2(e) and the causal key range j <= p_q:
+//   m_q = max_j z_qj*c,  Z_q = sum_j 2^(z_qj*c - m_q),
+//   raw_j = sum_q 2^(z_qj*c - m_q - log2 Z_q)           (j < n = L - W),
+// i.e. the softmax attention of every SRH window query, summed over the
+// queries, for every prefix token.  Z_q needs every key before any weight is
+// final.  Instead of a second pass over K, this kernel stores for every
+// prefix token and query the exponent e_qj = 2^(z_qj*c - ref_q) in fp16,
+// where ref_q is a running per-warp reference (<= m_q) that is written out
+// per (tile, 32-token quarter).  The combine kernel then forms
+// raw_j = sum_q 2^(ref_q - m_q - log2 Z_q) * e_qj; the weight is <= 1, and the
+// fp16 rounding of e (relative 2^-11) stays inside the score tolerance.
 //
 // Each CTA owns one work item: a contiguous range of 128-token K tiles of one
 // unit.  Warp roles:
 //   warp 0     TMA producer: K tiles (two 64-column halves, 128-byte swizzle)
-//              into a kStages-deep shared-memory ring; it starts streaming
-//              while the other warps stage the query rows;
+//              into a shared-memory ring of up to kStages tiles; it starts
+//              streaming while the other warps stage the query rows;
 //   warp 1     TMEM allocation, then UMMA issue: D[128 tokens x N] =
 //              K_tile . Q_S^T  (tcgen05.mma kind::f16, M=128, N = |S_g|*W
 //              rounded to 16, K = d = 128), fp32 accumulators in TMEM, 2 or 4
-//              buffers;
+//              buffers, each owned by one epilogue warpgroup;
 //   warps 2-9  two epilogue warpgroups (alternate tiles); thread = token
-//              (TMEM lane), it loads its row of N logits from TMEM, hands the
-//              buffer back to the MMA warp at once and works from registers.
+//              (TMEM lane): it reads its row of N logits from TMEM in 32-column
+//              groups, keeps per-warp running references and sums, stores the
+//              exponents, and hands the buffer back when the tile is done.
 // Tokens sit on the MMA's M side so every epilogue lane holds real work for
-// any N; in pass 2 the per-token sum over queries stays inside a thread.
-// Pass 1 keeps, per warp and query, a running reference (raised only when a
-// logit exceeds it by more than 2^kTau) and sums 2^(z*c - ref):
+// any N.  The per-query sums over tokens:
 //   * up to 64 query rows (kSmallN): every lane accumulates its own tokens
 //     in registers; the lanes are combined once per CTA by a 32x32
 //     transpose-reduction (31 shuffles per 32 queries);
@@ -42,20 +44,20 @@ namespace ckv {
 
 namespace {
 
-constexpr float kTau = 8.0f;  // log2 headroom before a running reference is raised
-constexpr int kNumEpiWarps = 8;  // pass-1 epilogue warps (2 warpgroups)
+// Running references R_q are kept kShift below the largest scaled logit seen,
+// so the stored exponents 2^(z*c - R) use the top of the fp16 range; R is
+// raised once an exponent would pass 2^kRaise (< fp16 max 65504).  Any R
+// works: every sum kept against R stands for  sum * 2^R.
+constexpr float kShift = 7.0f;
+constexpr float kRaise = 15.0f;
+constexpr int kNumEpiWarps = 8;  // 2 epilogue warpgroups
 constexpr int kEpiThreads = kNumEpiWarps * 32;
-// Epilogue warpgroups per pass: pass 1 keeps per-lane sums in registers and
-// runs 2; pass 2 needs few registers and runs 4 to hide TMEM-load latency.
-template <bool kAccum>
-struct Roles {
-  static constexpr int kWG = kAccum ? 4 : 2;
-  static constexpr int kThreads = 64 + 128 * kWG;
-  static constexpr int kStaged = kThreads - 32;  // warps 1.. stage the Q rows
-};
-// misc region: barriers (256 B) | refs/bias [8][256] f32 | sums [8][256] f32 |
+constexpr int kWG = 2;
+constexpr int kScoreThreads = 64 + 32 * kNumEpiWarps;
+constexpr int kStagedThreads = kScoreThreads - 32;  // warps 1.. stage the Q rows
+// misc region: barriers (256 B) | refs [8][256] f32 | sums [8][256] f32 |
 // rescale factors [8][256] f32 | window position of each query row [256] i32 |
-// per-warp logit scratch [8][32 lanes][33] f32 (pass 1, rare path)
+// per-warp logit scratch [8][32 lanes][33] f32 (rare path)
 constexpr int kZScratchFloats = 32 * 33;
 constexpr int kMiscBytes =
     256 + 3 * kNumEpiWarps * kMaxQRows * 4 + kMaxQRows * 4 + kNumEpiWarps * kZScratchFloats * 4;
@@ -69,8 +71,8 @@ __device__ __forceinline__ void wait_plain(uint32_t bar, uint32_t parity, uint64
   mbar_wait_bounded(bar, parity, &never, nullptr, timeout_ns);
 }
 
-template <bool kAccum, bool kSmallN>
-__global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
+template <bool kSmallN>
+__global__ void __launch_bounds__(kScoreThreads, 1)
     score_kernel(const __grid_constant__ ScoreParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -83,7 +85,7 @@ __global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
   uint64_t* bars = reinterpret_cast<uint64_t*>(sMisc);  // full[4] empty[4] tfull[4] tempty[4]
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(sMisc + 192);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(sMisc + 196);
-  float* sRef = reinterpret_cast<float*>(sMisc + 256);   // [8][kMaxQRows] refs / pass-2 bias
+  float* sRef = reinterpret_cast<float*>(sMisc + 256);   // [8][kMaxQRows] running references
   float* sAcc = sRef + kNumEpiWarps * kMaxQRows;         // [8][kMaxQRows] sums
   float* sFac = sAcc + kNumEpiWarps * kMaxQRows;         // [8][kMaxQRows] rescale factors
   int* sWpos = reinterpret_cast<int*>(sFac + kNumEpiWarps * kMaxQRows);  // [kMaxQRows]
@@ -106,19 +108,14 @@ __global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
   const int h0 = p.srh_off[g];
   const int N = (p.srh_off[g + 1] - h0) * W;
   const int Npad = (N + 15) & ~15;
+  const int Nr = expo_stride(N);  // row stride of the exponent table
   const int tstride = Npad <= 64 ? 64 : (Npad <= 128 ? 128 : 256);
   const int nbuf = (4 * tstride <= 512) ? 4 : 2;
   const uint32_t tcols = static_cast<uint32_t>(nbuf * tstride);
   const int t0 = it.t0;
-  int t1 = it.t1;
-  if (kAccum) t1 = min(t1, (n + kTileTokens - 1) / kTileTokens);
-  const int ntiles = max(t1 - t0, 0);
+  const int ntiles = it.t1 - t0;  // >= 1 by construction
 
   pdl_launch_dependents();
-  if (ntiles == 0) {  // uniform over the CTA: nothing allocated yet
-    pdl_wait();
-    return;
-  }
 
   // ------------------------------------------------------------ set-up
   if (threadIdx.x == 0) {
@@ -146,8 +143,7 @@ __global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
   if (warp == 0) {
     // ---------------------------------------------------------- TMA producer
     if (lane == 0) {
-      const uint64_t pol =
-          (kAccum || !p.use_evict_hint) ? l2_policy_evict_first() : l2_policy_evict_last();
+      const uint64_t pol = p.use_evict_hint ? l2_policy_evict_first() : l2_policy_evict_last();
       int issued = 0;
       for (int i = 0; i < ntiles; ++i) {
         const int st = i % nst;
@@ -173,7 +169,6 @@ __global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
     // 128-byte-swizzle layout (row r, 16-byte chunk ch of each 64-column half
     // lands at chunk ch ^ (r & 7)); rows N..Npad-1 are zero.
     const int st_tid = threadIdx.x - 32;
-    constexpr int kStagedThreads = Roles<kAccum>::kStaged;
     for (int idx = st_tid; idx < Npad * 16; idx += kStagedThreads) {
       const int r = idx >> 4;
       const int ch = idx & 15;
@@ -192,22 +187,7 @@ __global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
     }
     fence_proxy_async_smem();
     for (int q = st_tid; q < kMaxQRows; q += kStagedThreads) sWpos[q] = q < N ? q % W : 0;
-    if (kAccum) {
-      pdl_wait();  // the partials come from the pass-1 kernel
-      // Merge the unit's pass-1 partials (fixed order => deterministic) into
-      // the per-query bias m_q + log2 Z_q.
-      for (int q = st_tid; q < N; q += kStagedThreads) {
-        float m = kNegInf;
-        for (int i = 0; i < it.count; ++i)
-          m = fmaxf(m, p.partials[static_cast<long long>(it.first + i) * kMaxQRows + q].x);
-        float z = 0.f;
-        for (int i = 0; i < it.count; ++i) {
-          const float2 pr = p.partials[static_cast<long long>(it.first + i) * kMaxQRows + q];
-          if (pr.x != kNegInf) z += pr.y * ex2_approx(pr.x - m);
-        }
-        sRef[q] = m + log2f(z);
-      }
-    } else {
+    {
       const int ew = warp - kFirstEpiWarp;
       if (ew >= 0) {
         for (int q = lane; q < kMaxQRows; q += 32) {
@@ -259,37 +239,41 @@ __global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
     } else {
       // -------------------------------------------------------- epilogue
       const int ew = warp - kFirstEpiWarp;  // 0..7
-      constexpr int kWG = Roles<kAccum>::kWG;
-      const int wg = ew >> 2;   // epilogue warpgroup: tiles i with i % kWG == wg
-      const int qd = warp & 3;  // TMEM lane quarter this warp may access
+      const int wg = ew >> 2;               // epilogue warpgroup: tiles i % nwg == wg
+      const int qd = warp & 3;              // TMEM lane quarter this warp may access
       const float c = p.c;
       float* ref = sRef + ew * kMaxQRows;
       float* acc_s = sAcc + ew * kMaxQRows;
-      float acc[kSmallN ? 64 : 1];  // pass 1, kSmallN: this lane's sums per query
+      float* fac = sFac + ew * kMaxQRows;
+      float* zs = sZ + ew * kZScratchFloats;
+      float acc[kSmallN ? 64 : 1];  // kSmallN: this lane's sums per query
 #pragma unroll
       for (int j = 0; j < (kSmallN ? 64 : 1); ++j) acc[j] = 0.f;
       const int nhalf = (N + 31) >> 5;  // 32-column groups per tile
-      float* zs = sZ + ew * kZScratchFloats;
-      float* fac = sFac + ew * kMaxQRows;
-
+      uint16_t* erow_base = p.expo + it.eoff;
+      float* rtile_base = p.refs + it.roff;
       // Every TMEM buffer must belong to one warpgroup: an mbarrier parity
       // wait cannot tell phase k from phase k+2, so warpgroups sharing a
-      // buffer could read it early.  With fewer buffers than warpgroups the
-      // extra warpgroups stay idle.
+      // buffer could read it early.
       const int nwg = kWG < nbuf ? kWG : nbuf;
+      // The exponent and reference tables are reused: an earlier kernel of the
+      // stream may still read them, so wait for it before the first store.
+      pdl_wait();
+
       for (int i = wg; wg < nwg && i < ntiles; i += nwg) {
         const int b = i % nbuf;
         const uint32_t use = static_cast<uint32_t>(i / nbuf) & 1u;
         const bool got = mbar_wait_bounded(tfull0 + 8 * b, use, abort_flag, p.status);
         if (!__all_sync(0xffffffffu, got)) break;  // warp-uniform exit on abort
         tc_fence_after();
-        const int tok = (t0 + i) * kTileTokens + qd * 32 + lane;  // position in the sequence
+        const int tile = t0 + i;                                // tile index in the unit
+        const int tok = tile * kTileTokens + qd * 32 + lane;    // position in the sequence
         const uint32_t taddr =
             tbase + (static_cast<uint32_t>(qd * 32) << 16) + static_cast<uint32_t>(b * tstride);
         // tiles that reach the window (causal mask) or pass the sequence end
-        const bool edge = (t0 + i + 1) * kTileTokens > n;
+        const bool edge = (tile + 1) * kTileTokens > n;
         const int vis = n - tok;  // query row q sees this key iff tok < L and wpos(q) >= -vis
-        float s_tok = 0.f;        // pass 2: this token's score
+        uint16_t* erow = erow_base + static_cast<long long>(tok) * Nr;
 
 #pragma unroll
         for (int hh = 0; hh < (kSmallN ? 2 : 1); ++hh) {
@@ -300,12 +284,6 @@ __global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
             uint32_t r[32];
             tmem_load32_async(taddr + c0, r);
             tmem_wait_ld(r);
-            if (kAccum && h == nhalf - 1) {
-              // every column of this tile is in registers: hand the buffer back
-              tc_fence_before();
-              __syncwarp();
-              if (lane == 0) mbar_arrive(tempty0 + 8 * b);
-            }
             const int lim = min(32, N - c0);  // valid columns in this group
             const bool masked = edge || lim < 32;
             float z[32];  // raw logits (scaled by c inside the FFMA below)
@@ -323,151 +301,150 @@ __global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
                 }
               }
             }
-
-            if constexpr (kAccum) {
-              // ---------------------------------------------- pass 2
-              const float* bias = sRef + c0;
-              float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+            float* rf = ref + c0;
+            // t = z*c - ref, computed once; -inf where masked
+            float t[32];
+            float tmax = kNegInf;
+            if (masked) {
 #pragma unroll
               for (int j = 0; j < 32; j += 4) {
-                const float4 bq = *reinterpret_cast<const float4*>(bias + j);
-                a0 += ex2_approx(fmaf(z[j + 0], c, -bq.x));
-                a1 += ex2_approx(fmaf(z[j + 1], c, -bq.y));
-                a2 += ex2_approx(fmaf(z[j + 2], c, -bq.z));
-                a3 += ex2_approx(fmaf(z[j + 3], c, -bq.w));
+                const float4 rq = *reinterpret_cast<const float4*>(rf + j);
+                const float rv[4] = {rq.x, rq.y, rq.z, rq.w};
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                  t[j + u] = z[j + u] == kNegInf ? kNegInf : fmaf(z[j + u], c, -rv[u]);
+                  tmax = fmaxf(tmax, t[j + u]);
+                }
               }
-              s_tok += (a0 + a1) + (a2 + a3);
             } else {
-              // ---------------------------------------------- pass 1
-              float* rf = ref + c0;
-              // t = z*c - ref, computed once; -inf where masked
-              float t[32];
-              float tmax = kNegInf;
-              if (masked) {
 #pragma unroll
-                for (int j = 0; j < 32; j += 4) {
-                  const float4 rq = *reinterpret_cast<const float4*>(rf + j);
-                  const float rv[4] = {rq.x, rq.y, rq.z, rq.w};
+              for (int j = 0; j < 32; j += 4) {
+                const float4 rq = *reinterpret_cast<const float4*>(rf + j);
+                t[j + 0] = fmaf(z[j + 0], c, -rq.x);
+                t[j + 1] = fmaf(z[j + 1], c, -rq.y);
+                t[j + 2] = fmaf(z[j + 2], c, -rq.z);
+                t[j + 3] = fmaf(z[j + 3], c, -rq.w);
+                tmax = fmaxf(fmaxf(tmax, fmaxf(t[j], t[j + 1])), fmaxf(t[j + 2], t[j + 3]));
+              }
+            }
+            if (__any_sync(0xffffffffu, tmax > kRaise)) {
+              // Rare: raise each query's reference to kShift below its column
+              // max over the warp and rescale the sums kept so far by
+              // 2^(old - new).  The scaled logits are re-read from TMEM (the
+              // buffer is still held) into shared memory, so this path stays
+              // small; t == -inf marks the masked entries.
 #pragma unroll
-                  for (int u = 0; u < 4; ++u) {
-                    t[j + u] = z[j + u] == kNegInf ? kNegInf : fmaf(z[j + u], c, -rv[u]);
-                    tmax = fmaxf(tmax, t[j + u]);
-                  }
-                }
-              } else {
+              for (int j = 0; j < 32; ++j) zs[lane * 33 + j] = t[j];
+              {
+                uint32_t r2[32];
+                tmem_load32_async(taddr + c0, r2);
+                tmem_wait_ld(r2);
 #pragma unroll
-                for (int j = 0; j < 32; j += 4) {
-                  const float4 rq = *reinterpret_cast<const float4*>(rf + j);
-                  t[j + 0] = fmaf(z[j + 0], c, -rq.x);
-                  t[j + 1] = fmaf(z[j + 1], c, -rq.y);
-                  t[j + 2] = fmaf(z[j + 2], c, -rq.z);
-                  t[j + 3] = fmaf(z[j + 3], c, -rq.w);
-                  tmax = fmaxf(fmaxf(tmax, fmaxf(t[j], t[j + 1])), fmaxf(t[j + 2], t[j + 3]));
+                for (int j = 0; j < 32; ++j) {
+                  const float tj = zs[lane * 33 + j];
+                  zs[lane * 33 + j] = tj == kNegInf ? kNegInf : __uint_as_float(r2[j]) * c;
                 }
               }
-              if (__any_sync(0xffffffffu, tmax > kTau)) {
-                // Rare: raise each query's reference to its column max over
-                // the warp and rescale the sums kept so far by 2^(old - new).
-                // The scaled logits go through shared memory so this path
-                // stays small.
-                {
-                  // re-read this group's logits (the buffer is still held)
-                  uint32_t r2[32];
-                  tmem_load32_async(taddr + c0, r2);
-                  tmem_wait_ld(r2);
+              __syncwarp();
+              float m = kNegInf;
+              for (int rr = 0; rr < 32; ++rr) m = fmaxf(m, zs[rr * 33 + lane]);
+              const float old = rf[lane];
+              const float nw = fmaxf(old, m - kShift);
+              const float f = (nw == old) ? 1.f : ((old == kNegInf) ? 0.f : ex2_approx(old - nw));
+              rf[lane] = nw;
+              if constexpr (kSmallN) {
+                fac[c0 + lane] = f;
+              } else {
+                acc_s[c0 + lane] *= f;
+              }
+              __syncwarp();
 #pragma unroll
-                  for (int j = 0; j < 32; ++j)
-                    zs[lane * 33 + j] = t[j] == kNegInf ? kNegInf : __uint_as_float(r2[j]) * c;
-                }
-                __syncwarp();
-                float m = kNegInf;
-                for (int rr = 0; rr < 32; ++rr) m = fmaxf(m, zs[rr * 33 + lane]);
-                const float old = rf[lane];
-                const float nw = fmaxf(old, m);
-                const float f =
-                    (nw == old) ? 1.f : ((old == kNegInf) ? 0.f : ex2_approx(old - nw));
-                rf[lane] = nw;
-                if constexpr (kSmallN) {
-                  fac[c0 + lane] = f;
-                } else {
-                  acc_s[c0 + lane] *= f;
-                }
-                __syncwarp();
+              for (int j = 0; j < 32; j += 4) {
+                const float4 rq = *reinterpret_cast<const float4*>(rf + j);
+                const float rv[4] = {rq.x, rq.y, rq.z, rq.w};
 #pragma unroll
-                for (int j = 0; j < 32; j += 4) {
-                  const float4 rq = *reinterpret_cast<const float4*>(rf + j);
-                  const float rv[4] = {rq.x, rq.y, rq.z, rq.w};
-#pragma unroll
-                  for (int u = 0; u < 4; ++u) {
-                    const float zc = zs[lane * 33 + j + u];
-                    t[j + u] = zc == kNegInf ? kNegInf : zc - rv[u];
-                  }
-                }
-                if constexpr (kSmallN) {
-#pragma unroll
-                  for (int j = 0; j < 32; j += 4) {
-                    const float4 fq = *reinterpret_cast<const float4*>(fac + c0 + j);
-                    acc[32 * hh + j + 0] *= fq.x;
-                    acc[32 * hh + j + 1] *= fq.y;
-                    acc[32 * hh + j + 2] *= fq.z;
-                    acc[32 * hh + j + 3] *= fq.w;
-                  }
+                for (int u = 0; u < 4; ++u) {
+                  const float zc = zs[lane * 33 + j + u];
+                  t[j + u] = zc == kNegInf ? kNegInf : zc - rv[u];
                 }
               }
               if constexpr (kSmallN) {
 #pragma unroll
-                for (int j = 0; j < 32; ++j) acc[32 * hh + j] += ex2_approx(t[j]);
-              } else {
-#pragma unroll
-                for (int j = 0; j < 32; ++j) t[j] = ex2_approx(t[j]);
-                const float colsum = warp_transpose_sum32(t, lane);
-                acc_s[c0 + lane] += colsum;
+                for (int j = 0; j < 32; j += 4) {
+                  const float4 fq = *reinterpret_cast<const float4*>(fac + c0 + j);
+                  acc[32 * hh + j + 0] *= fq.x;
+                  acc[32 * hh + j + 1] *= fq.y;
+                  acc[32 * hh + j + 2] *= fq.z;
+                  acc[32 * hh + j + 3] *= fq.w;
+                }
               }
-              __syncwarp();
             }
+            // exponents: summed per query, and stored (fp16) for the prefix,
+            // eight at a time to keep few registers live
+            const bool store = tok < n;
+            const int ncols = min(32, Nr - c0);  // 8, 16, 24 or 32 (a multiple of 8)
+            uint4* dst = reinterpret_cast<uint4*>(erow + c0);
+            float e[32];
+#pragma unroll
+            for (int v = 0; v < 4; ++v) {
+#pragma unroll
+              for (int u = 0; u < 8; ++u) e[8 * v + u] = ex2_approx(t[8 * v + u]);
+              if (store && 8 * v < ncols) {
+                uint4 pk;
+                pk.x = pack_half2(e[8 * v + 0], e[8 * v + 1]);
+                pk.y = pack_half2(e[8 * v + 2], e[8 * v + 3]);
+                pk.z = pack_half2(e[8 * v + 4], e[8 * v + 5]);
+                pk.w = pack_half2(e[8 * v + 6], e[8 * v + 7]);
+                dst[v] = pk;
+              }
+              if constexpr (kSmallN) {
+#pragma unroll
+                for (int u = 0; u < 8; ++u) acc[32 * hh + 8 * v + u] += e[8 * v + u];
+              }
+            }
+            if constexpr (!kSmallN) {
+              const float colsum = warp_transpose_sum32(e, lane);
+              acc_s[c0 + lane] += colsum;
+            }
+            __syncwarp();
           }
         }
-        if (!kAccum) {
-          // pass 1 keeps the buffer until the tile is done (the rare path re-reads it)
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(tempty0 + 8 * b);
+        // the references this tile quarter's exponents are relative to
+        {
+          float* rt = rtile_base + (static_cast<long long>(tile) * kQuarters + qd) * Nr;
+          for (int q = lane; q < N; q += 32) rt[q] = ref[q];
         }
-        if (kAccum && tok < n) {
-          p.raw[static_cast<long long>(g) * p.p_total + p.cu_prefix[s] + tok] = s_tok;
-        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(tempty0 + 8 * b);
       }
 
-      if (!kAccum) {
-        if constexpr (kSmallN) {
-          // one cross-lane reduction of the per-lane sums per CTA
+      if constexpr (kSmallN) {
+        // one cross-lane reduction of the per-lane sums per CTA
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            if (h * 32 < N) {
-              float v[32];
+        for (int h = 0; h < 2; ++h) {
+          if (h * 32 < N) {
+            float v[32];
 #pragma unroll
-              for (int j = 0; j < 32; ++j) v[j] = acc[32 * h + j];
-              const float colsum = warp_transpose_sum32(v, lane);
-              acc_s[32 * h + lane] = colsum;
-            }
+            for (int j = 0; j < 32; ++j) v[j] = acc[32 * h + j];
+            const float colsum = warp_transpose_sum32(v, lane);
+            acc_s[32 * h + lane] = colsum;
           }
-          __syncwarp();
         }
-        // combine the 8 epilogue warps' (reference, sum) pairs per query
-        named_bar_sync(kBarEpi, kEpiThreads);
-        // the previous kernels of the stream may still read the partials
-        pdl_wait();
-        const int te = static_cast<int>(threadIdx.x) - kFirstEpiWarp * 32;
-        if (te < N && !*abort_flag) {
-          float m = kNegInf;
-          for (int w = 0; w < kNumEpiWarps; ++w) m = fmaxf(m, sRef[w * kMaxQRows + te]);
-          float z = 0.f;
-          for (int w = 0; w < kNumEpiWarps; ++w) {
-            const float r = sRef[w * kMaxQRows + te];
-            if (r != kNegInf) z += sAcc[w * kMaxQRows + te] * ex2_approx(r - m);
-          }
-          p.partials[static_cast<long long>(blockIdx.x) * kMaxQRows + te] = make_float2(m, z);
+        __syncwarp();
+      }
+      // combine the 8 epilogue warps' (reference, sum) pairs per query
+      named_bar_sync(kBarEpi, kEpiThreads);
+      const int te = static_cast<int>(threadIdx.x) - kFirstEpiWarp * 32;
+      if (te < N && !*abort_flag) {
+        float m = kNegInf;
+        for (int w = 0; w < kNumEpiWarps; ++w) m = fmaxf(m, sRef[w * kMaxQRows + te]);
+        float z = 0.f;
+        for (int w = 0; w < kNumEpiWarps; ++w) {
+          const float r = sRef[w * kMaxQRows + te];
+          if (r != kNegInf) z += sAcc[w * kMaxQRows + te] * ex2_approx(r - m);
         }
+        p.partials[static_cast<long long>(blockIdx.x) * kMaxQRows + te] = make_float2(m, z);
       }
     }
   }
@@ -482,11 +459,11 @@ __global__ void __launch_bounds__(Roles<kAccum>::kThreads, 1)
   }
 }
 
-template <bool kAccum, bool kSmallN>
+template <bool kSmallN>
 cudaError_t launch(const ScoreParams& p, int n_items, size_t smem, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(n_items));
-  cfg.blockDim = dim3(Roles<kAccum>::kThreads);
+  cfg.blockDim = dim3(kScoreThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
@@ -494,7 +471,7 @@ cudaError_t launch(const ScoreParams& p, int n_items, size_t smem, cudaStream_t 
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, score_kernel<kAccum, kSmallN>, p);
+  return cudaLaunchKernelEx(&cfg, score_kernel<kSmallN>, p);
 }
 
 }  // namespace
@@ -506,27 +483,14 @@ size_t score_smem_bytes(int q_half_bytes, int stages) {
 
 cudaError_t score_set_smem_limit(size_t bytes) {
   const int b = static_cast<int>(bytes);
-  cudaError_t e;
-  if ((e = cudaFuncSetAttribute(score_kernel<false, false>,
-                                cudaFuncAttributeMaxDynamicSharedMemorySize, b)) != cudaSuccess)
-    return e;
-  if ((e = cudaFuncSetAttribute(score_kernel<true, false>,
-                                cudaFuncAttributeMaxDynamicSharedMemorySize, b)) != cudaSuccess)
-    return e;
-  if ((e = cudaFuncSetAttribute(score_kernel<false, true>,
-                                cudaFuncAttributeMaxDynamicSharedMemorySize, b)) != cudaSuccess)
-    return e;
-  return cudaFuncSetAttribute(score_kernel<true, true>,
-                              cudaFuncAttributeMaxDynamicSharedMemorySize, b);
+  cudaError_t e = cudaFuncSetAttribute(score_kernel<false>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, b);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(score_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, b);
 }
 
-cudaError_t launch_score_stats(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s) {
-  return p.small_n ? launch<false, true>(p, n_items, smem, s)
-                   : launch<false, false>(p, n_items, smem, s);
-}
-cudaError_t launch_score_accum(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s) {
-  return p.small_n ? launch<true, true>(p, n_items, smem, s)
-                   : launch<true, false>(p, n_items, smem, s);
+cudaError_t launch_score(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s) {
+  return p.small_n ? launch<true>(p, n_items, smem, s) : launch<false>(p, n_items, smem, s);
 }
 
 }  // namespace ckv

@@ -145,14 +145,35 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   const int len = hi - lo;
   const bool in_smem = p.smem_slice;
   float* raw_s = s_dyn;                                  // [S + 2r] when in_smem
-  float* pooled = in_smem ? s_dyn + S + 2 * r : p.pooled_ws + soff + lo;  // [len]
+  const float* pin = p.pooled_in ? p.pooled_in + soff + lo : nullptr;
+  // pooled scores of the slice: shared memory, else the workspace copy (or,
+  // when they arrive already pooled, the caller's buffer, read only)
+  const float* pooled = in_smem ? s_dyn + S + 2 * r
+                                : (pin ? pin : p.pooled_ws + soff + lo);  // [len]
+  float* pooled_w = in_smem ? s_dyn + S + 2 * r : p.pooled_ws + soff + lo;
 
   pdl_launch_dependents();
-  pdl_wait();  // raw scores come from the scoring kernel
+  pdl_wait();  // scores come from the previous kernel
 
   // 1. pooling ---------------------------------------------------------------
   const float fP = static_cast<float>(p.pool_width);
-  if (len > 0) {
+  if (len > 0 && pin) {
+    if (in_smem) {  // already pooled: stage the slice
+      for (int base = 0; base < len; base += 8 * kSelThreads) {
+        float v[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int li = base + i * kSelThreads + tid;
+          v[i] = li < len ? pin[li] : 0.f;
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int li = base + i * kSelThreads + tid;
+          if (li < len) pooled_w[li] = v[i];
+        }
+      }
+    }
+  } else if (len > 0) {
     if (in_smem) {
       const int span = len + 2 * r;
       for (int base = 0; base < span; base += 8 * kSelThreads) {
@@ -174,7 +195,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
         float a = 0.f;
         for (int t = 0; t <= 2 * r; ++t) a += raw_s[i + t];
         const float pv = a / fP;
-        pooled[i] = pv;
+        pooled_w[i] = pv;
         if (pout) pout[lo + i] = pv;
       }
     } else {
@@ -186,7 +207,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
           a += (jj >= 0 && jj < n) ? raw[jj] : 0.f;
         }
         const float pv = a / fP;
-        pooled[i] = pv;
+        pooled_w[i] = pv;
         if (pout) pout[j] = pv;
       }
     }

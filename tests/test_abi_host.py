@@ -108,4 +108,5 @@ def test_compress_layer_host_errors():
     big = np.ones(8, np.uint8)          # 4 heads x W=32 = 128 rows: fine
     prob.struct.window = 80             # 4 x 80 = 320 rows > 256: unsupported
     b3, bp3 = B._i32([100, 100])
-    assert call(big, budgets_ptr=bp3) == B.CKV_ERR_UNSUPPORTED
+    # the workspace bound grows with the window (exponent rows of G*W)
+    assert call(big, budgets_ptr=bp3, wsn=ckv.workspace_size(prob)) == B.CKV_ERR_UNSUPPORTED

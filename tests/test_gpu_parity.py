@@ -1,9 +1,10 @@
 """CUDA path vs. the float64 oracle, through the C ABI (needs a GB300).
 
-Tolerances (spec acceptance, see oracle/compare.py): raw and pooled
-scores within 1e-3 relative + 1e-5 absolute; retained index sets identical
-except for near-ties within 1e-3 of the k-th pooled score; K/V rows
-bit-exact at the device's indices; device results deterministic.
+Tolerances (acceptance, see oracle/compare.py): raw and pooled scores within
+1e-3 relative + 1e-5 absolute (and, as a guard on the device's arithmetic,
+within 2^-11 relative: the fp16 exponent table's rounding); retained index
+sets identical except for near-ties within 1e-3 of the k-th pooled score;
+K/V rows bit-exact at the device's indices; device results deterministic.
 """
 import math
 
@@ -17,6 +18,8 @@ import workloads as wl
 from oracle import compare
 
 pytestmark = pytest.mark.gpu
+
+EXPO_RTOL = 2.0 ** -11 + 2e-5
 
 
 def _bits(t):
@@ -54,8 +57,14 @@ def check(d, window, pool_width, dev, mask=None, budgets=None, scale=None, **kw)
     res = run_oracle(d, window, pool_width, mask=mask, budgets=budgets, scale=scale)
     assert np.array_equal(cu_out, res.cu_out)
     idx = out.indices.cpu().numpy()
-    ties = compare.check_layer(res, out.raw.cpu().numpy(), out.pooled.cpu().numpy(), idx,
-                               d["cu_seqlens"], window)
+    raw_gpu, pooled_gpu = out.raw.cpu().numpy(), out.pooled.cpu().numpy()
+    ties = compare.check_layer(res, raw_gpu, pooled_gpu, idx, d["cu_seqlens"], window)
+    # Tighter than the acceptance tolerance: the device's only coarse rounding
+    # is the fp16 exponent table (relative 2^-11 per term, all terms >= 0);
+    # the rest is fp32 arithmetic.
+    compare.check_scores("raw (fp16 table bound)", raw_gpu, res.raw, rtol=EXPO_RTOL, atol=1e-8)
+    compare.check_scores("pooled (fp16 table bound)", pooled_gpu, res.pooled, rtol=EXPO_RTOL,
+                         atol=1e-8)
     compare.check_gather_bits(_bits(d["k"]), _bits(d["v"]), _bits(out.k_out), _bits(out.v_out),
                               idx, d["cu_seqlens"], cu_out)
     return out, res, ties
@@ -66,8 +75,7 @@ def test_llama8b_4k_single_layer(cuda_device):
     """The 1-layer L=4096 fp16 workload, in full."""
     cfg = wl.get("c1")
     d = wl.make_layer(cfg, 0)
-    _, res, ties = check(d, cfg.window, cfg.pool_width, cuda_device)
-    assert ties <= 2
+    check(d, cfg.window, cfg.pool_width, cuda_device)
 
 
 @pytest.mark.parametrize("dtype", ["fp16", "bf16"])
@@ -196,9 +204,7 @@ def test_gather_reports_bad_index(cuda_device):
 def test_full_size_layer(cuda_device, name, layer):
     cfg = wl.get(name)
     d = wl.make_layer(cfg, layer)
-    _, res, ties = check(d, cfg.window, cfg.pool_width, cuda_device)
-    n_units = len(res.units)
-    assert ties <= max(4, n_units)
+    check(d, cfg.window, cfg.pool_width, cuda_device)
 
 
 def test_graph_captured_multilayer_step_matches(cuda_device):
