@@ -406,8 +406,13 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
     long long quarters = 0;
     for (int u = 0; u < nu; ++u) quarters += units[u0 + u].quarters;
     const long long ctarget = std::max(1, std::min(kMaxItems - nu, 4 * F->sms));
-    const int chunk_q = static_cast<int>(std::max(8LL, (quarters + ctarget - 1) / ctarget));
-    const size_t csmem = combine_smem_bytes(chunk_q * 32, I.P);
+    int chunk_q = static_cast<int>(std::max(8LL, (quarters + ctarget - 1) / ctarget));
+    int max_nr = 8;
+    for (int u = 0; u < nu; ++u) max_nr = std::max(max_nr, expo_stride(S.rows[units[u0 + u].g]));
+    // a chunk's weight table and raw scores must fit the shared memory
+    while (chunk_q > 1 && combine_smem_bytes(chunk_q, max_nr, I.P) > F->combine_smem_max)
+      chunk_q = (chunk_q + 1) / 2;
+    const size_t csmem = combine_smem_bytes(chunk_q, max_nr, I.P);
     if (csmem > F->combine_smem_max) return CKV_ERR_UNSUPPORTED;
 
     int n_items = 0, n_comb = 0;
@@ -444,7 +449,6 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
     P.n_items = n_items;
     C.n_items = n_comb;
     P.q_half_bytes = ((max_rows * 128) + 1023) & ~1023;
-    P.small_n = max_rows <= 64 ? 1 : 0;
     P.stages = kStages;
     while (P.stages > 2 &&
            score_smem_bytes(P.q_half_bytes, P.stages) > static_cast<size_t>(F->smem_optin))

@@ -220,9 +220,10 @@ __device__ __forceinline__ void tmem_order_after_wait(uint32_t (&r)[32]) {
 }
 
 // ---------------------------------------------------------------- PDL
-// Programmatic dependent launch: let the next kernel of the stream start its
-// prologue now, and wait for the previous kernel's results before reading or
-// overwriting anything it may touch.  Without the launch attribute both are
+// Programmatic dependent launch: allow the next kernel of the stream to be
+// launched (once every CTA of this grid has issued the trigger or exited),
+// and wait for the previous kernel's results before reading or overwriting
+// anything it may touch.  Without the launch attribute both are
 // no-ops.  Every kernel executes pdl_wait() before it exits, so completion of
 // a kernel implies completion of all kernels before it.
 __device__ __forceinline__ void pdl_launch_dependents() {
@@ -237,6 +238,22 @@ __device__ __forceinline__ uint32_t pack_half2(float lo, float hi) {
   uint32_t r;
   asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
   return r;
+}
+
+// 32-byte and 16-byte global stores with an L2 eviction-priority policy
+// (from l2_policy_*); the address must be aligned to the store size.
+__device__ __forceinline__ void st_global_v8_hint(void* ptr, const uint32_t (&v)[8], uint64_t pol) {
+  asm volatile(
+      "st.global.L2::cache_hint.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8}, %9;" ::"l"(ptr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+      "l"(pol)
+      : "memory");
+}
+__device__ __forceinline__ void st_global_v4_hint(void* ptr, uint32_t a, uint32_t b, uint32_t c,
+                                                  uint32_t d, uint64_t pol) {
+  asm volatile("st.global.L2::cache_hint.v4.b32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(ptr), "r"(a),
+               "r"(b), "r"(c), "r"(d), "l"(pol)
+               : "memory");
 }
 
 // Hardware base-2 exponential (MUFU); ex2(-inf) = +0.

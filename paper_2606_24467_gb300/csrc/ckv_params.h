@@ -10,7 +10,7 @@ namespace ckv {
 
 constexpr int kHeadDim = 128;       // d: one 256-byte K row per token and group (16-bit types)
 constexpr int kTileTokens = 128;    // tokens per K tile = UMMA M = TMEM lanes
-constexpr int kStages = 4;          // most K tiles in flight per CTA (fewer when Q rows are large)
+constexpr int kStages = 6;          // most K tiles in flight per CTA (fewer when Q rows are large)
 constexpr int kMaxQRows = 256;      // |S_g| * W rows per unit (UMMA N limit)
 constexpr int kMaxBatch = 512;
 constexpr int kMaxQHeads = 256;
@@ -27,11 +27,11 @@ constexpr int kHalfTileBytes = kTileBytes / 2;           // 64 columns (128 B) o
 constexpr int kQHalfBytes = kMaxQRows * 128;             // Q rows, one 64-column half
 constexpr int kQuarters = kTileTokens / 32;              // 32-token groups per tile (one warp each)
 
-// One score work item: a contiguous range of K tiles of one unit.  `first`
-// and `count` locate all items of the same unit in the item table (the
-// combine step merges their partial softmax statistics); `eoff` / `roff` are
-// the unit's offsets in the exponent table (fp16 elements) and in the
-// reference table (floats).
+// One work item: a contiguous range [t0, t1) of one unit -- 128-key tiles
+// for the scoring kernel, 32-key quarters for the combine kernel.  `first` /
+// `count` locate the unit's scoring items (whose softmax pairs the combine
+// kernel merges); `eoff` / `roff` are the unit's offsets in the exponent
+// table (fp16 elements) and in the reference table (floats).
 struct WorkItem {
   uint16_t seq, group, t0, t1, first, count;
   uint32_t eoff, roff;
@@ -40,15 +40,14 @@ struct WorkItem {
 struct ScoreParams {
   CUtensorMap tmap_k;          // 3-D map over K: (d, kv head, token)
   const uint16_t* q;           // window queries (f16/bf16 bits)
-  float2* partials;            // [n_items][kMaxQRows]: (max z*c, sum 2^(z*c - max))
-  uint16_t* expo;              // fp16 2^(z*c - ref) per prefix token and query row
-  float* refs;                 // per (tile, quarter, query row): the ref used for expo
+  float2* partials;            // [n_items][kMaxQRows]: (M, S) with sum 2^(z*c) = S * 2^M
+  uint16_t* expo;              // fp16 2^(z*c - R) per prefix key and query row (Nr per key)
+  float* refs;                 // per (tile, quarter, query row): the R used for expo
   int* status;                 // device status word
   long long q_bs, q_hs, q_ws;  // window-query strides, elements
   float c;                     // scale * log2(e)
   int window, num_kv_heads, n_items, is_bf16, use_evict_hint;
   int q_half_bytes;            // bytes of one 64-column half of the Q rows in shared memory
-  int small_n;                 // 1: every unit of the launch has at most 64 query rows
   int stages;                  // K tiles in the shared-memory ring (2..kStages)
   int cu_seqlens[kMaxBatch + 1];
   uint16_t srh_off[kMaxKvHeads + 1];   // SRH heads of group g: srh_heads[srh_off[g] .. srh_off[g+1])
@@ -70,8 +69,14 @@ struct CombineParams {
   WorkItem items[kMaxItems];
 };
 
-// Row stride (fp16 elements) of the exponent table for `rows` query rows.
-__host__ __device__ constexpr int expo_stride(int rows) { return (rows + 7) & ~7; }
+// Row length (fp16 elements) of the exponent table for `rows` query rows:
+// the next power of two >= max(rows, 8), so that a row is a whole number of
+// 16-byte chunks and their count divides 32 when rows <= 256.
+__host__ __device__ constexpr int expo_stride(int rows) {
+  int r = 8;
+  while (r < rows) r <<= 1;
+  return r;
+}
 
 struct SelectParams {
   const float* raw;            // score layout (pooled here when pooled_in is null)
@@ -115,7 +120,9 @@ cudaError_t launch_select(const SelectParams& p, int n_units, size_t smem, cudaS
 cudaError_t launch_gather(const GatherParams& p, long long rows, cudaStream_t s);
 size_t score_smem_bytes(int q_half_bytes, int stages);
 cudaError_t score_set_smem_limit(size_t bytes);
-size_t combine_smem_bytes(int chunk_tokens, int pool_width);
+// Dynamic shared memory of a combine CTA that covers `quarters` 32-key
+// quarters with exponent rows of `nr` columns and pooling width P.
+size_t combine_smem_bytes(int quarters, int nr, int pool_width);
 // Sets the combine kernel's dynamic shared-memory limit to what `optin`
 // leaves beside its static shared memory and returns that limit.
 cudaError_t combine_set_smem_limit(size_t optin, size_t* dynamic_max);

@@ -1,23 +1,26 @@
 // Normalised window scores and pooling (CompressKV Sec. 3.3 scores summed over
-// the SRH window queries; Sec. 4 average pooling over tokens) from the
-// exponent table the scoring kernel leaves behind.
+// the SRH window queries; Sec. 4 average pooling over tokens) from the tables
+// the scoring kernel leaves behind.
 //
-// For unit (s, g) the scoring kernel stored, per prefix token j and query row
-// q, e_qj = 2^(z_qj*c - R) in fp16, where R = refs[tile, quarter, q] is the
-// reference its warp used for that 32-token quarter, and per work item the
+// For unit (s, g) the scoring kernel stored, per prefix key j and query row
+// q, e_qj = 2^(z_qj*c - R) in fp16, where R = refs[quarter(j), q] is the
+// reference its warp used for that 32-key quarter, and per work item i the
 // pair (M_i, S_i) with  sum over the item's keys of 2^(z*c) = S_i * 2^M_i.
 // This kernel
-//   1. merges the pairs of the unit's items: M = max M_i,
-//      S = sum S_i 2^(M_i - M), bias_q = M + log2 S  (= log2 of the softmax
-//      denominator of query q);
+//   1. merges the pairs of the unit's items into bias_q = log2 D_q, the log2
+//      of query q's softmax denominator (merged in item order);
 //   2. raw_j = sum_q e_qj * 2^(R - bias_q)   (every weight is <= 1);
 //   3. pooled_j = (sum_{t=-h..h} raw_{j+t}) / P with zeros outside [0, n),
 //      summed in a fixed order.
-// One CTA per chunk of 32-token quarters of one unit; the chunk's raw values
-// and an h-token halo on each side live in shared memory.  Warps take whole
-// quarters: the quarter's exponent block (32 x Nr fp16, contiguous) is read
-// with coalesced 16-byte loads, and each lane's 8 columns are weighted with
-// the quarter's weights (one shared-memory row per warp).
+// One CTA per chunk of 32-key quarters of one unit.  It first tabulates the
+// weights 2^(R - bias_q) of every quarter it touches (the chunk plus an
+// h-key halo on each side) in shared memory, then streams the exponent rows
+// of those keys -- one contiguous region -- with the whole block, kLoadBatch
+// 16-byte loads in flight per thread.  Thread tid always meets the same
+// 8-column chunk of a row (tid % cpr, where cpr = Nr / 8 divides 32); the
+// cpr threads of a row are adjacent lanes and add their dot products by
+// shuffles.  Raw scores of the chunk and halo stay in shared memory for the
+// pooling.
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
@@ -28,8 +31,9 @@ namespace ckv {
 namespace {
 
 constexpr int kCombThreads = 256;
-constexpr int kCombWarps = kCombThreads / 32;
-constexpr int kLoadBatch = 4;  // 16-byte loads in flight per lane
+constexpr int kLoadBatch = 8;  // 16-byte loads in flight per thread
+constexpr int kPairSlots = 2048;  // softmax pairs staged per round
+static_assert(kMaxQRows <= kCombThreads, "one thread per query row");
 
 __device__ __forceinline__ float dot8(const uint4 v, const float* w) {
   const __half2* h = reinterpret_cast<const __half2*>(&v);
@@ -52,14 +56,11 @@ __device__ __forceinline__ float dot8(const uint4 v, const float* w) {
 
 __global__ void __launch_bounds__(kCombThreads)
     combine_kernel(const __grid_constant__ CombineParams p) {
-  extern __shared__ float s_raw[];  // [chunk + 2h]: raw over [a - h, b + h)
+  extern __shared__ __align__(16) float s_dyn[];  // weights [nqt][Nr] | raw [span]
   __shared__ float s_bias[kMaxQRows];
-  __shared__ __align__(16) float s_w[kCombWarps][kMaxQRows];
-  __shared__ float s_row[kCombWarps][32];
+  __shared__ float2 s_pairs[kPairSlots];
 
   const int tid = threadIdx.x;
-  const int warp = tid >> 5;
-  const int lane = tid & 31;
   const WorkItem it = p.items[blockIdx.x];
   const int s = it.seq;
   const int g = it.group;
@@ -68,7 +69,8 @@ __global__ void __launch_bounds__(kCombThreads)
   const int n = L - W;
   const int N = (p.srh_off[g + 1] - p.srh_off[g]) * W;
   const int Nr = expo_stride(N);
-  const int cpr = Nr >> 3;  // 16-byte chunks per token row
+  const int cpr = Nr >> 3;  // 16-byte chunks per key row (a power of two <= 32)
+  const int col = tid & (cpr - 1);
   const int h = (p.pool_width - 1) >> 1;
   const int a = it.t0 * 32;
   const int b = min(it.t1 * 32, n);
@@ -76,72 +78,79 @@ __global__ void __launch_bounds__(kCombThreads)
   const int span = b - a + 2 * h;
   const int ea = max(base, 0);
   const int eb = min(b + h, n);
+  const int q0 = ea >> 5;
+  const int nqt = ((eb + 31) >> 5) - q0;  // quarters touched
+  float* s_w = s_dyn;
+  float* s_raw = s_dyn + nqt * Nr;
 
-  pdl_launch_dependents();
   for (int i = tid; i < span; i += kCombThreads) s_raw[i] = 0.f;
-  pdl_wait();  // partials, exponents and references come from the scoring kernel
+  pdl_wait();  // pairs and tables come from the scoring kernel
 
-  // 1. per-query log2 softmax denominators
-  for (int q = tid; q < N; q += kCombThreads) {
-    float m = -INFINITY;
-    for (int i = 0; i < it.count; ++i)
-      m = fmaxf(m, p.partials[static_cast<long long>(it.first + i) * kMaxQRows + q].x);
-    float z = 0.f;
-    for (int i = 0; i < it.count; ++i) {
-      const float2 pr = p.partials[static_cast<long long>(it.first + i) * kMaxQRows + q];
-      if (pr.x != -INFINITY) z = fmaf(pr.y, ex2_approx(pr.x - m), z);
-    }
-    s_bias[q] = m + __log2f(z);
-  }
-  __syncthreads();
-
-  // 2. raw scores, one 32-token quarter per warp at a time
-  const bool pow2 = (32 % cpr) == 0;
-  float* w = s_w[warp];
-  for (int qi = (ea >> 5) + warp; qi < ((eb + 31) >> 5); qi += kCombWarps) {
-    const float* rq = p.refs + it.roff + static_cast<long long>(qi) * Nr;
-    for (int q = lane; q < Nr; q += 32) w[q] = q < N ? ex2_approx(rq[q] - s_bias[q]) : 0.f;
-    if (!pow2) s_row[warp][lane] = 0.f;
-    __syncwarp();
-    const int r0 = max(ea, qi * 32) - qi * 32;
-    const int r1 = min(eb, qi * 32 + 32) - qi * 32;
-    const uint4* E = reinterpret_cast<const uint4*>(p.expo + it.eoff +
-                                                    static_cast<long long>(qi) * 32 * Nr);
-    const int fend = r1 * cpr;
-    for (int f0 = r0 * cpr; f0 < fend; f0 += 32 * kLoadBatch) {
-      uint4 ev[kLoadBatch];
-#pragma unroll
-      for (int u = 0; u < kLoadBatch; ++u) {
-        const int f = f0 + 32 * u + lane;
-        ev[u] = f < fend ? __ldg(E + f) : make_uint4(0u, 0u, 0u, 0u);
+  // 1. per-query log2 softmax denominators: the unit's item pairs are staged
+  //    in shared memory (all loads in flight at once), then merged in item
+  //    order by one thread per query
+  {
+    const int per = kPairSlots / N;  // items per staging round
+    float m = -INFINITY, z = 0.f;    // thread tid < N: query tid
+    for (int i0 = 0; i0 < it.count; i0 += per) {
+      const int ni = min(per, it.count - i0);
+      for (int i = tid; i < ni * N; i += kCombThreads) {
+        const int ii = i / N;
+        const int q = i - ii * N;
+        s_pairs[i] = p.partials[static_cast<long long>(it.first + i0 + ii) * kMaxQRows + q];
       }
-#pragma unroll
-      for (int u = 0; u < kLoadBatch; ++u) {
-        const int f0u = f0 + 32 * u;
-        if (f0u >= fend) break;  // uniform over the warp
-        const int f = f0u + lane;
-        const int row = f / cpr;
-        const int col = f - row * cpr;
-        float v = f < fend ? dot8(ev[u], w + 8 * col) : 0.f;
-        if (pow2) {
-          // the cpr lanes of one row are adjacent and aligned
-          for (int off = cpr >> 1; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-          if (f < fend && col == 0) s_raw[qi * 32 + row - base] = v;
-        } else if (f < fend) {
-          atomicAdd(&s_row[warp][row], v);
+      __syncthreads();
+      for (int q = tid; q < N; q += kCombThreads) {  // N <= kCombThreads: one query per thread
+        for (int ii = 0; ii < ni; ++ii) {
+          const float2 pr = s_pairs[ii * N + q];
+          if (pr.x == -INFINITY) continue;
+          if (pr.x > m) {
+            z = fmaf(z, ex2_approx(m - pr.x), pr.y);
+            m = pr.x;
+          } else {
+            z = fmaf(pr.y, ex2_approx(pr.x - m), z);
+          }
         }
       }
+      __syncthreads();
     }
-    __syncwarp();
-    if (!pow2) {
-      const int t = qi * 32 + lane;
-      if (lane >= r0 && lane < r1) s_raw[t - base] = s_row[warp][lane];
-      __syncwarp();  // s_row is cleared for the next quarter only after this read
+    if (tid < N) s_bias[tid] = m + __log2f(z);
+  }
+  __syncthreads();
+
+  // 2. weights 2^(R - bias_q) of the quarters touched
+  const float* R = p.refs + it.roff + static_cast<long long>(q0) * Nr;
+  for (int i = tid; i < nqt * Nr; i += kCombThreads) {
+    const int qq = i / Nr;
+    const int cc = i - qq * Nr;
+    s_w[i] = cc < N ? ex2_approx(R[i] - s_bias[cc]) : 0.f;
+  }
+  __syncthreads();
+
+  // 3. raw scores of the keys [ea, eb): one contiguous run of exponent rows
+  const uint4* E4 = reinterpret_cast<const uint4*>(p.expo + it.eoff);
+  const int f_lo = ea * cpr;
+  const int f_hi = eb * cpr;
+  for (int f0 = f_lo; f0 < f_hi; f0 += kLoadBatch * kCombThreads) {
+    uint4 ev[kLoadBatch];
+#pragma unroll
+    for (int u = 0; u < kLoadBatch; ++u) {
+      const int f = f0 + u * kCombThreads + tid;
+      ev[u] = f < f_hi ? __ldg(E4 + f) : make_uint4(0u, 0u, 0u, 0u);
+    }
+#pragma unroll
+    for (int u = 0; u < kLoadBatch; ++u) {
+      const int f = f0 + u * kCombThreads + tid;
+      const int row = f / cpr;  // key position
+      const int qq = min((row >> 5) - q0, nqt - 1);
+      float v = dot8(ev[u], s_w + qq * Nr + 8 * col);
+      for (int off = cpr >> 1; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+      if (f < f_hi && col == 0) s_raw[row - base] = v;
     }
   }
   __syncthreads();
 
-  // 3. pooling (and the raw scores, when asked for)
+  // 4. pooling (and the raw scores, when asked for)
   const long long soff = static_cast<long long>(g) * p.p_total + p.cu_prefix[s];
   const float fP = static_cast<float>(p.pool_width);
   for (int j = a + tid; j < b; j += kCombThreads) {
@@ -151,12 +160,17 @@ __global__ void __launch_bounds__(kCombThreads)
     p.pooled[soff + j] = acc / fP;
     if (p.raw_out) p.raw_out[soff + j] = s_raw[i + h];
   }
+  pdl_launch_dependents();  // late: the select kernel needs every chunk anyway
 }
 
 }  // namespace
 
-size_t combine_smem_bytes(int chunk_tokens, int pool_width) {
-  return static_cast<size_t>(chunk_tokens + pool_width) * sizeof(float);
+size_t combine_smem_bytes(int quarters, int nr, int pool_width) {
+  // the chunk's quarters plus one halo quarter on each side, and its raw
+  // scores with the halo
+  return (static_cast<size_t>(quarters + 2) * nr + static_cast<size_t>(quarters) * 32 +
+          pool_width) *
+         sizeof(float);
 }
 
 cudaError_t combine_set_smem_limit(size_t optin, size_t* dynamic_max) {

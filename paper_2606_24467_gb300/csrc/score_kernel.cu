@@ -1,39 +1,44 @@
 // Observation-window scoring (CompressKV Sec. 3.3; SnapKV-style window of
 // Sec. 4) on sm_103a tensor cores, in one pass over K.
 //
-// For one unit (sequence s, KV group g) let Q_S be the |S_g|*W window-query
-// rows of the group's SRH heads and K the unit's L keys.  With
-// z = <q, k> * scale, c = log2(e) and the causal key range j <= p_q:
-//   m_q = max_j z_qj*c,  Z_q = sum_j 2^(z_qj*c - m_q),
-//   raw_j = sum_q 2^(z_qj*c - m_q - log2 Z_q)           (j < n = L - W),
-// i.e. the softmax attention of every SRH window query, summed over the
-// queries, for every prefix token.  Z_q needs every key before any weight is
-// final.  Instead of a second pass over K, this kernel stores for every
-// prefix token and query the exponent e_qj = 2^(z_qj*c - ref_q) in fp16,
-// where ref_q is a running per-warp reference (<= m_q) that is written out
-// per (tile, 32-token quarter).  The combine kernel then forms
-// raw_j = sum_q 2^(ref_q - m_q - log2 Z_q) * e_qj; the weight is <= 1, and the
-// fp16 rounding of e (relative 2^-11) stays inside the score tolerance.
+// For one unit (sequence s, KV group g) let Q_S be the N = |S_g|*W
+// window-query rows of the group's SRH heads and K the unit's L keys.  With
+// z = <q, k> * scale and c = log2(e), the attention of query q (window
+// position p_q) on key j <= p_q is 2^(z_qj*c) / D_q with
+// D_q = sum_{j <= p_q} 2^(z_qj*c).  This kernel computes every logit once
+// and leaves
+//   * for every prefix key j < n = L - W and query row q, the exponent
+//     e_qj = 2^(z_qj*c - R) in an fp16 table (Nr = N rounded up to a power of
+//     two >= 8 columns per key; columns N..Nr-1 are 0), where R is a
+//     per-query reference kept by the warp that owns the key's 32-token
+//     quarter of its tile; the R used for every (tile, quarter, q) goes to a
+//     float table;
+//   * per work item and query row the pair (M, S) with
+//     sum over the item's keys of 2^(z*c) = S * 2^M.
+// R stays kShift below the largest scaled logit the warp has seen and is
+// raised whenever an exponent would pass 2^kRaise, so every stored exponent
+// is at most 2^kRaise (below the fp16 maximum 65504) and keeps a relative
+// rounding error <= 2^-11.  The combine kernel forms D_q from the pairs and
+// the normalised, pooled scores from the tables.
 //
 // Each CTA owns one work item: a contiguous range of 128-token K tiles of one
 // unit.  Warp roles:
-//   warp 0     TMA producer: K tiles (two 64-column halves, 128-byte swizzle)
-//              into a shared-memory ring of up to kStages tiles; it starts
-//              streaming while the other warps stage the query rows;
-//   warp 1     TMEM allocation, then UMMA issue: D[128 tokens x N] =
-//              K_tile . Q_S^T  (tcgen05.mma kind::f16, M=128, N = |S_g|*W
-//              rounded to 16, K = d = 128), fp32 accumulators in TMEM, 2 or 4
-//              buffers, each owned by one epilogue warpgroup;
-//   warps 2-9  two epilogue warpgroups (alternate tiles); thread = token
-//              (TMEM lane): it reads its row of N logits from TMEM in 32-column
-//              groups, keeps per-warp running references and sums, stores the
-//              exponents, and hands the buffer back when the tile is done.
+//   warp 0      TMA producer: K tiles (two 64-column halves, 128-byte swizzle)
+//               into a shared-memory ring of up to kStages tiles; it starts
+//               streaming while the other warps stage the query rows;
+//   warp 1      TMEM allocation, then UMMA issue: D[128 tokens x N] =
+//               K_tile . Q_S^T  (tcgen05.mma kind::f16, M=128, N rounded to 16,
+//               K = d = 128), fp32 accumulators in TMEM, 2 or 4 buffers, each
+//               owned by one epilogue warpgroup;
+//   warps 2-17  four epilogue warpgroups (tiles i % 4; with 2 buffers only
+//               the first two work); thread = token (TMEM lane): it reads its
+//               row of logits from TMEM 32 columns at a time, keeps the
+//               warp's running references, writes its exponent row with
+//               32-byte stores that ask L2 to keep the table, and adds the
+//               exponents into the warp's per-query sums by a 32x32
+//               transpose-reduction.
 // Tokens sit on the MMA's M side so every epilogue lane holds real work for
-// any N.  The per-query sums over tokens:
-//   * up to 64 query rows (kSmallN): every lane accumulates its own tokens
-//     in registers; the lanes are combined once per CTA by a 32x32
-//     transpose-reduction (31 shuffles per 32 queries);
-//   * more rows: the transpose-reduction runs per tile.
+// any N.
 #include <cuda_runtime.h>
 
 #include <cfloat>
@@ -44,26 +49,18 @@ namespace ckv {
 
 namespace {
 
-// Running references R_q are kept kShift below the largest scaled logit seen,
-// so the stored exponents 2^(z*c - R) use the top of the fp16 range; R is
-// raised once an exponent would pass 2^kRaise (< fp16 max 65504).  Any R
-// works: every sum kept against R stands for  sum * 2^R.
-constexpr float kShift = 7.0f;
-constexpr float kRaise = 15.0f;
-constexpr int kNumEpiWarps = 8;  // 2 epilogue warpgroups
-constexpr int kEpiThreads = kNumEpiWarps * 32;
-constexpr int kWG = 2;
+constexpr float kShift = 7.0f;   // R sits this far below the warp's largest logit (log2 units)
+constexpr float kRaise = 15.0f;  // exponents stay <= 2^kRaise
+constexpr int kNumEpiWarps = 16;  // 4 epilogue warpgroups
+constexpr int kWG = kNumEpiWarps / 4;
 constexpr int kScoreThreads = 64 + 32 * kNumEpiWarps;
 constexpr int kStagedThreads = kScoreThreads - 32;  // warps 1.. stage the Q rows
-// misc region: barriers (256 B) | refs [8][256] f32 | sums [8][256] f32 |
-// rescale factors [8][256] f32 | window position of each query row [256] i32 |
-// per-warp logit scratch [8][32 lanes][33] f32 (rare path)
-constexpr int kZScratchFloats = 32 * 33;
-constexpr int kMiscBytes =
-    256 + 3 * kNumEpiWarps * kMaxQRows * 4 + kMaxQRows * 4 + kNumEpiWarps * kZScratchFloats * 4;
+// misc region: barriers (256 B) | running references [16][256] f32 |
+// sums [16][256] f32 | window position of each query row [256] i32
+constexpr int kMiscBytes = 256 + 2 * kNumEpiWarps * kMaxQRows * 4 + kMaxQRows * 4;
 constexpr float kNegInf = -INFINITY;
-constexpr int kBarEpi = 1;       // named barrier: the 8 epilogue warps
-constexpr int kBarStaged = 2;    // named barrier: warps 1..9 after staging Q
+constexpr int kBarStaged = 2;  // named barrier: warps 1.. after staging Q
+constexpr int kBarEpi = 1;     // named barrier: the epilogue warps
 constexpr int kFirstEpiWarp = 2;
 
 __device__ __forceinline__ void wait_plain(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
@@ -71,7 +68,6 @@ __device__ __forceinline__ void wait_plain(uint32_t bar, uint32_t parity, uint64
   mbar_wait_bounded(bar, parity, &never, nullptr, timeout_ns);
 }
 
-template <bool kSmallN>
 __global__ void __launch_bounds__(kScoreThreads, 1)
     score_kernel(const __grid_constant__ ScoreParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -82,14 +78,12 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
   uint8_t* sQ = base + nst * kTileBytes;
   const int qh = p.q_half_bytes;
   uint8_t* sMisc = sQ + 2 * qh;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sMisc);  // full[4] empty[4] tfull[4] tempty[4]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sMisc);  // full[6] empty[6] tfull[4] tempty[4]
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(sMisc + 192);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(sMisc + 196);
-  float* sRef = reinterpret_cast<float*>(sMisc + 256);   // [8][kMaxQRows] running references
-  float* sAcc = sRef + kNumEpiWarps * kMaxQRows;         // [8][kMaxQRows] sums
-  float* sFac = sAcc + kNumEpiWarps * kMaxQRows;         // [8][kMaxQRows] rescale factors
-  int* sWpos = reinterpret_cast<int*>(sFac + kNumEpiWarps * kMaxQRows);  // [kMaxQRows]
-  float* sZ = reinterpret_cast<float*>(sWpos + kMaxQRows);               // [8][32][33]
+  float* sRef = reinterpret_cast<float*>(sMisc + 256);                  // [16][kMaxQRows]
+  float* sAcc = sRef + kNumEpiWarps * kMaxQRows;                         // [16][kMaxQRows]
+  int* sWpos = reinterpret_cast<int*>(sAcc + kNumEpiWarps * kMaxQRows);  // [kMaxQRows]
 
   const uint32_t full0 = smem_u32(bars);
   const uint32_t empty0 = full0 + 8 * kStages;
@@ -108,14 +102,12 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
   const int h0 = p.srh_off[g];
   const int N = (p.srh_off[g + 1] - h0) * W;
   const int Npad = (N + 15) & ~15;
-  const int Nr = expo_stride(N);  // row stride of the exponent table
+  const int Nr = expo_stride(N);  // row length of the exponent table
   const int tstride = Npad <= 64 ? 64 : (Npad <= 128 ? 128 : 256);
   const int nbuf = (4 * tstride <= 512) ? 4 : 2;
   const uint32_t tcols = static_cast<uint32_t>(nbuf * tstride);
   const int t0 = it.t0;
   const int ntiles = it.t1 - t0;  // >= 1 by construction
-
-  pdl_launch_dependents();
 
   // ------------------------------------------------------------ set-up
   if (threadIdx.x == 0) {
@@ -191,8 +183,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
       const int ew = warp - kFirstEpiWarp;
       if (ew >= 0) {
         for (int q = lane; q < kMaxQRows; q += 32) {
-          // padded rows (q >= N) never see a masked value, so they start at 0
-          sRef[ew * kMaxQRows + q] = q < N ? kNegInf : 0.f;
+          sRef[ew * kMaxQRows + q] = kNegInf;
           sAcc[ew * kMaxQRows + q] = 0.f;
         }
       }
@@ -238,20 +229,14 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
       __syncwarp();  // reconverge before the CTA-wide (aligned) barrier below
     } else {
       // -------------------------------------------------------- epilogue
-      const int ew = warp - kFirstEpiWarp;  // 0..7
+      const int ew = warp - kFirstEpiWarp;  // 0..15
       const int wg = ew >> 2;               // epilogue warpgroup: tiles i % nwg == wg
       const int qd = warp & 3;              // TMEM lane quarter this warp may access
       const float c = p.c;
       float* ref = sRef + ew * kMaxQRows;
       float* acc_s = sAcc + ew * kMaxQRows;
-      float* fac = sFac + ew * kMaxQRows;
-      float* zs = sZ + ew * kZScratchFloats;
-      float acc[kSmallN ? 64 : 1];  // kSmallN: this lane's sums per query
-#pragma unroll
-      for (int j = 0; j < (kSmallN ? 64 : 1); ++j) acc[j] = 0.f;
-      const int nhalf = (N + 31) >> 5;  // 32-column groups per tile
-      uint16_t* erow_base = p.expo + it.eoff;
-      float* rtile_base = p.refs + it.roff;
+      const int ngrp = (Nr + 31) >> 5;  // 32-column groups of an exponent row
+      const uint64_t keep = l2_policy_evict_last();
       // Every TMEM buffer must belong to one warpgroup: an mbarrier parity
       // wait cannot tell phase k from phase k+2, so warpgroups sharing a
       // buffer could read it early.
@@ -266,183 +251,144 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         const bool got = mbar_wait_bounded(tfull0 + 8 * b, use, abort_flag, p.status);
         if (!__all_sync(0xffffffffu, got)) break;  // warp-uniform exit on abort
         tc_fence_after();
-        const int tile = t0 + i;                                // tile index in the unit
-        const int tok = tile * kTileTokens + qd * 32 + lane;    // position in the sequence
+        const int tile = t0 + i;                              // tile index in the unit
+        const int tok = tile * kTileTokens + qd * 32 + lane;  // position in the sequence
         const uint32_t taddr =
             tbase + (static_cast<uint32_t>(qd * 32) << 16) + static_cast<uint32_t>(b * tstride);
         // tiles that reach the window (causal mask) or pass the sequence end
         const bool edge = (tile + 1) * kTileTokens > n;
         const int vis = n - tok;  // query row q sees this key iff tok < L and wpos(q) >= -vis
-        uint16_t* erow = erow_base + static_cast<long long>(tok) * Nr;
+        const bool key = tok < L;    // a key of the sequence (the last tile may run past L)
+        const bool store = tok < n;  // the table holds prefix keys only
+        uint16_t* erow = p.expo + it.eoff + static_cast<long long>(tok) * Nr;
 
+        for (int grp = 0; grp < ngrp; ++grp) {
+          const int c0 = 32 * grp;
+          const int ncols = min(32, Nr - c0);  // 8, 16 or 32 (Nr is a power of two)
+          if (c0 >= N) {
+            // padding columns of the table
+            if (store) {
+              if (ncols == 32) {
+                const uint32_t zz[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+                st_global_v8_hint(erow + c0, zz, keep);
+                st_global_v8_hint(erow + c0 + 16, zz, keep);
+              } else {
+                for (int v = 0; v < ncols; v += 8) st_global_v4_hint(erow + c0 + v, 0u, 0u, 0u, 0u, keep);
+              }
+            }
+            continue;
+          }
+          uint32_t r[32];
+          tmem_load32_async(taddr + c0, r);
+          tmem_wait_ld(r);
+          const int lim = min(32, N - c0);  // valid columns in this group
+          const bool masked = edge || lim < 32;
+          float* rf = ref + c0;
+          // t = z*c - R, -inf where the key is masked for that query
+          float t[32];
+          float tmax = kNegInf;
+          if (masked) {
 #pragma unroll
-        for (int hh = 0; hh < (kSmallN ? 2 : 1); ++hh) {
-          for (int hr = 0; hr < (kSmallN ? 1 : nhalf); ++hr) {
-            const int h = kSmallN ? hh : hr;
-            if (kSmallN && h >= nhalf) break;  // uniform: N <= 32
-            const int c0 = 32 * h;
-            uint32_t r[32];
+            for (int j = 0; j < 32; j += 4) {
+              const int4 wq = *reinterpret_cast<const int4*>(sWpos + c0 + j);
+              const float4 rq = *reinterpret_cast<const float4*>(rf + j);
+              const int wv[4] = {wq.x, wq.y, wq.z, wq.w};
+              const float rv[4] = {rq.x, rq.y, rq.z, rq.w};
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                const bool ok = (j + u) < lim && (!edge || (key && wv[u] >= -vis));
+                t[j + u] = ok ? fmaf(__uint_as_float(r[j + u]), c, -rv[u]) : kNegInf;
+                tmax = fmaxf(tmax, t[j + u]);
+              }
+            }
+          } else {
+#pragma unroll
+            for (int j = 0; j < 32; j += 4) {
+              const float4 rq = *reinterpret_cast<const float4*>(rf + j);
+              t[j + 0] = fmaf(__uint_as_float(r[j + 0]), c, -rq.x);
+              t[j + 1] = fmaf(__uint_as_float(r[j + 1]), c, -rq.y);
+              t[j + 2] = fmaf(__uint_as_float(r[j + 2]), c, -rq.z);
+              t[j + 3] = fmaf(__uint_as_float(r[j + 3]), c, -rq.w);
+              tmax = fmaxf(fmaxf(tmax, fmaxf(t[j], t[j + 1])), fmaxf(t[j + 2], t[j + 3]));
+            }
+          }
+          if (__any_sync(0xffffffffu, tmax > kRaise)) {
+            // Rare (always on a warp's first tile, where R = -inf): raise
+            // each query's R to kShift below its largest scaled logit in this
+            // warp's 32 tokens.  Logits are re-read from TMEM (the buffer is
+            // still held) and reduced across lanes in registers.
+            uint32_t valid = 0u;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) valid |= (t[j] != kNegInf ? 1u : 0u) << j;
+            float v[32];
             tmem_load32_async(taddr + c0, r);
             tmem_wait_ld(r);
-            const int lim = min(32, N - c0);  // valid columns in this group
-            const bool masked = edge || lim < 32;
-            float z[32];  // raw logits (scaled by c inside the FFMA below)
 #pragma unroll
-            for (int j = 0; j < 32; ++j) z[j] = __uint_as_float(r[j]);
-            if (masked) {
-#pragma unroll
-              for (int j = 0; j < 32; j += 4) {
-                const int4 wq = *reinterpret_cast<const int4*>(sWpos + c0 + j);
-                const int wv[4] = {wq.x, wq.y, wq.z, wq.w};
-#pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                  const bool ok = (j + u) < lim && (!edge || (tok < L && wv[u] >= -vis));
-                  z[j + u] = ok ? z[j + u] : kNegInf;
-                }
-              }
-            }
-            float* rf = ref + c0;
-            // t = z*c - ref, computed once; -inf where masked
-            float t[32];
-            float tmax = kNegInf;
-            if (masked) {
-#pragma unroll
-              for (int j = 0; j < 32; j += 4) {
-                const float4 rq = *reinterpret_cast<const float4*>(rf + j);
-                const float rv[4] = {rq.x, rq.y, rq.z, rq.w};
-#pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                  t[j + u] = z[j + u] == kNegInf ? kNegInf : fmaf(z[j + u], c, -rv[u]);
-                  tmax = fmaxf(tmax, t[j + u]);
-                }
-              }
-            } else {
-#pragma unroll
-              for (int j = 0; j < 32; j += 4) {
-                const float4 rq = *reinterpret_cast<const float4*>(rf + j);
-                t[j + 0] = fmaf(z[j + 0], c, -rq.x);
-                t[j + 1] = fmaf(z[j + 1], c, -rq.y);
-                t[j + 2] = fmaf(z[j + 2], c, -rq.z);
-                t[j + 3] = fmaf(z[j + 3], c, -rq.w);
-                tmax = fmaxf(fmaxf(tmax, fmaxf(t[j], t[j + 1])), fmaxf(t[j + 2], t[j + 3]));
-              }
-            }
-            if (__any_sync(0xffffffffu, tmax > kRaise)) {
-              // Rare: raise each query's reference to kShift below its column
-              // max over the warp and rescale the sums kept so far by
-              // 2^(old - new).  The scaled logits are re-read from TMEM (the
-              // buffer is still held) into shared memory, so this path stays
-              // small; t == -inf marks the masked entries.
-#pragma unroll
-              for (int j = 0; j < 32; ++j) zs[lane * 33 + j] = t[j];
-              {
-                uint32_t r2[32];
-                tmem_load32_async(taddr + c0, r2);
-                tmem_wait_ld(r2);
-#pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                  const float tj = zs[lane * 33 + j];
-                  zs[lane * 33 + j] = tj == kNegInf ? kNegInf : __uint_as_float(r2[j]) * c;
-                }
-              }
-              __syncwarp();
-              float m = kNegInf;
-              for (int rr = 0; rr < 32; ++rr) m = fmaxf(m, zs[rr * 33 + lane]);
-              const float old = rf[lane];
-              const float nw = fmaxf(old, m - kShift);
-              const float f = (nw == old) ? 1.f : ((old == kNegInf) ? 0.f : ex2_approx(old - nw));
-              rf[lane] = nw;
-              if constexpr (kSmallN) {
-                fac[c0 + lane] = f;
-              } else {
-                acc_s[c0 + lane] *= f;
-              }
-              __syncwarp();
-#pragma unroll
-              for (int j = 0; j < 32; j += 4) {
-                const float4 rq = *reinterpret_cast<const float4*>(rf + j);
-                const float rv[4] = {rq.x, rq.y, rq.z, rq.w};
-#pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                  const float zc = zs[lane * 33 + j + u];
-                  t[j + u] = zc == kNegInf ? kNegInf : zc - rv[u];
-                }
-              }
-              if constexpr (kSmallN) {
-#pragma unroll
-                for (int j = 0; j < 32; j += 4) {
-                  const float4 fq = *reinterpret_cast<const float4*>(fac + c0 + j);
-                  acc[32 * hh + j + 0] *= fq.x;
-                  acc[32 * hh + j + 1] *= fq.y;
-                  acc[32 * hh + j + 2] *= fq.z;
-                  acc[32 * hh + j + 3] *= fq.w;
-                }
-              }
-            }
-            // exponents: summed per query, and stored (fp16) for the prefix,
-            // eight at a time to keep few registers live
-            const bool store = tok < n;
-            const int ncols = min(32, Nr - c0);  // 8, 16, 24 or 32 (a multiple of 8)
-            uint4* dst = reinterpret_cast<uint4*>(erow + c0);
-            float e[32];
-#pragma unroll
-            for (int v = 0; v < 4; ++v) {
-#pragma unroll
-              for (int u = 0; u < 8; ++u) e[8 * v + u] = ex2_approx(t[8 * v + u]);
-              if (store && 8 * v < ncols) {
-                uint4 pk;
-                pk.x = pack_half2(e[8 * v + 0], e[8 * v + 1]);
-                pk.y = pack_half2(e[8 * v + 2], e[8 * v + 3]);
-                pk.z = pack_half2(e[8 * v + 4], e[8 * v + 5]);
-                pk.w = pack_half2(e[8 * v + 6], e[8 * v + 7]);
-                dst[v] = pk;
-              }
-              if constexpr (kSmallN) {
-#pragma unroll
-                for (int u = 0; u < 8; ++u) acc[32 * hh + 8 * v + u] += e[8 * v + u];
-              }
-            }
-            if constexpr (!kSmallN) {
-              const float colsum = warp_transpose_sum32(e, lane);
-              acc_s[c0 + lane] += colsum;
-            }
+            for (int j = 0; j < 32; ++j)
+              v[j] = ((valid >> j) & 1u) ? __uint_as_float(r[j]) * c : kNegInf;
+            const float m = warp_transpose_max32(v, lane);  // column c0 + lane
+            const float old = rf[lane];
+            const float nw = fmaxf(old, m - kShift);
+            // the sums kept against the old R shrink by 2^(old - new)
+            acc_s[c0 + lane] *= (nw == old) ? 1.f : ((old == kNegInf) ? 0.f : ex2_approx(old - nw));
             __syncwarp();
+            rf[lane] = nw;
+            __syncwarp();
+            tmem_load32_async(taddr + c0, r);
+            tmem_wait_ld(r);
+#pragma unroll
+            for (int j = 0; j < 32; j += 4) {
+              const float4 rq = *reinterpret_cast<const float4*>(rf + j);
+              const float rv[4] = {rq.x, rq.y, rq.z, rq.w};
+#pragma unroll
+              for (int u = 0; u < 4; ++u)
+                t[j + u] = ((valid >> (j + u)) & 1u) ? fmaf(__uint_as_float(r[j + u]), c, -rv[u])
+                                                      : kNegInf;
+            }
           }
+          // exponents: stored as fp16 (prefix keys), 16 per 32-byte store, and
+          // summed per query over the warp's 32 keys
+          float e[32];
+#pragma unroll
+          for (int j = 0; j < 32; ++j) e[j] = ex2_approx(t[j]);
+          if (store) {
+#pragma unroll
+            for (int v = 0; v < 2; ++v) {
+              if (16 * v < ncols) {
+                uint32_t pk[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) pk[u] = pack_half2(e[16 * v + 2 * u], e[16 * v + 2 * u + 1]);
+                if (ncols >= 16) {
+                  st_global_v8_hint(erow + c0 + 16 * v, pk, keep);
+                } else {  // ncols == 8
+                  st_global_v4_hint(erow + c0, pk[0], pk[1], pk[2], pk[3], keep);
+                }
+              }
+            }
+          }
+          const float colsum = warp_transpose_sum32(e, lane);
+          acc_s[c0 + lane] += colsum;
+          __syncwarp();
         }
         // the references this tile quarter's exponents are relative to
         {
-          float* rt = rtile_base + (static_cast<long long>(tile) * kQuarters + qd) * Nr;
+          float* rt = p.refs + it.roff + (static_cast<long long>(tile) * kQuarters + qd) * Nr;
           for (int q = lane; q < N; q += 32) rt[q] = ref[q];
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(tempty0 + 8 * b);
       }
-
-      if constexpr (kSmallN) {
-        // one cross-lane reduction of the per-lane sums per CTA
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          if (h * 32 < N) {
-            float v[32];
-#pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] = acc[32 * h + j];
-            const float colsum = warp_transpose_sum32(v, lane);
-            acc_s[32 * h + lane] = colsum;
-          }
-        }
-        __syncwarp();
-      }
-      // combine the 8 epilogue warps' (reference, sum) pairs per query
-      named_bar_sync(kBarEpi, kEpiThreads);
+      // merge the epilogue warps' (R, sum) pairs per query into the item's pair
+      named_bar_sync(kBarEpi, 32 * kNumEpiWarps);
       const int te = static_cast<int>(threadIdx.x) - kFirstEpiWarp * 32;
       if (te < N && !*abort_flag) {
         float m = kNegInf;
         for (int w = 0; w < kNumEpiWarps; ++w) m = fmaxf(m, sRef[w * kMaxQRows + te]);
         float z = 0.f;
         for (int w = 0; w < kNumEpiWarps; ++w) {
-          const float r = sRef[w * kMaxQRows + te];
-          if (r != kNegInf) z += sAcc[w * kMaxQRows + te] * ex2_approx(r - m);
+          const float rw = sRef[w * kMaxQRows + te];
+          if (rw != kNegInf) z += sAcc[w * kMaxQRows + te] * ex2_approx(rw - m);
         }
         p.partials[static_cast<long long>(blockIdx.x) * kMaxQRows + te] = make_float2(m, z);
       }
@@ -450,6 +396,9 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
   }
 
   // ------------------------------------------------------------ teardown
+  // The next kernel is launched once every CTA has reached this point, so its
+  // CTAs spread over all SMs instead of packing the ones that freed first.
+  pdl_launch_dependents();
   pdl_wait();
   tc_fence_before();
   __syncthreads();
@@ -457,21 +406,6 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     tc_fence_after();
     tmem_dealloc(tbase, tcols);
   }
-}
-
-template <bool kSmallN>
-cudaError_t launch(const ScoreParams& p, int n_items, size_t smem, cudaStream_t stream) {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(n_items));
-  cfg.blockDim = dim3(kScoreThreads);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, score_kernel<kSmallN>, p);
 }
 
 }  // namespace
@@ -482,15 +416,22 @@ size_t score_smem_bytes(int q_half_bytes, int stages) {
 }
 
 cudaError_t score_set_smem_limit(size_t bytes) {
-  const int b = static_cast<int>(bytes);
-  cudaError_t e = cudaFuncSetAttribute(score_kernel<false>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, b);
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(score_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, b);
+  return cudaFuncSetAttribute(score_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(bytes));
 }
 
-cudaError_t launch_score(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s) {
-  return p.small_n ? launch<true>(p, n_items, smem, s) : launch<false>(p, n_items, smem, s);
+cudaError_t launch_score(const ScoreParams& p, int n_items, size_t smem, cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(n_items));
+  cfg.blockDim = dim3(kScoreThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, score_kernel, p);
 }
 
 }  // namespace ckv
