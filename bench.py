@@ -56,6 +56,8 @@ def parse_args():
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--streams", type=int, default=3,
+                    help="layers in flight: layer l runs on stream l %% S with its own workspace")
     return ap.parse_args()
 
 
@@ -240,15 +242,39 @@ def run_ours(args):
                          trace=counter) for lay in layers]
     tprobs = [ckv.Problem(lay["q_win"], lay["k"], lay["cu_seqlens"], cfg.window, cfg.pool_width,
                           trace=trace) for lay in layers]
-    ws = ckv.workspace(probs[0], dev)
+    # Layers are independent: with S streams, layer l is compressed on stream
+    # l % S with that stream's workspace, so one layer's latency-bound select
+    # overlaps the next layer's K stream.  Each stream's kernels still chain
+    # through programmatic dependent launch.
+    n_streams = max(1, args.streams)
+    wss = [ckv.workspace(probs[0], dev) for _ in range(n_streams)]
+    ws = wss[0]
+    lanes = [torch.cuda.Stream() for _ in range(n_streams)]
     outs = [ckv.LayerOutputs(probs[l], budgets[l], cfg.head_dim, layers[l]["k"].dtype, dev,
                              scores=False) for l in range(cfg.n_layers)]
 
-    def step(pr):
+    def step(pr, streams=n_streams):
+        if streams == 1:
+            for l, lay in enumerate(layers):
+                o = outs[l]
+                ckv.compress_layer(pr[l], lay["q_win"], lay["k"], lay["v"], lay["srh_mask"],
+                                   lay["budgets"], o.indices, o.k_out, o.v_out, ws)
+            return
+        cur = torch.cuda.current_stream()
+        fork = torch.cuda.Event()
+        fork.record(cur)
+        for st in lanes[:streams]:
+            st.wait_event(fork)
         for l, lay in enumerate(layers):
             o = outs[l]
+            st = lanes[l % streams]
             ckv.compress_layer(pr[l], lay["q_win"], lay["k"], lay["v"], lay["srh_mask"],
-                               lay["budgets"], o.indices, o.k_out, o.v_out, ws)
+                               lay["budgets"], o.indices, o.k_out, o.v_out, wss[l % streams],
+                               stream=st)
+        for st in lanes[:streams]:
+            done = torch.cuda.Event()
+            done.record(st)
+            cur.wait_event(done)
 
     side = torch.cuda.Stream()
     side.wait_stream(torch.cuda.current_stream())
@@ -265,7 +291,7 @@ def run_ours(args):
     traced = torch.cuda.CUDAGraph()
     trace.reset()
     with torch.cuda.graph(traced, capture_error_mode="thread_local"):
-        step(tprobs)
+        step(tprobs, streams=1)
     torch.cuda.synchronize()
 
     for _ in range(max(args.warmup, 3)):
@@ -288,7 +314,8 @@ def run_ours(args):
     elapsed_ms = reduce_max(dist, t0.elapsed_time(t1), dev)
     ms_per_step = elapsed_ms / args.steps
     value = world * tokens * args.steps / (elapsed_ms / 1e3)
-    assert ckv.read_device_status(ws) == 0, "device status set during the bench"
+    for w in wss:
+        assert ckv.read_device_status(w) == 0, "device status set during the bench"
 
     # per-kernel durations: a second timed region replaying the traced graph
     for _ in range(3):
@@ -341,6 +368,7 @@ def run_ours(args):
                    "l2": f"inputs larger than L2: {sum(l['k'].numel() * 2 * 2 for l in layers) / 1e9:.2f} GB "
                          "of K/V per step, each layer's K read cold; no flush",
                    "cuda_graph": True, "parallelism": f"replicas x{world}",
+                   "layer_streams": n_streams,
                    "l2_bytes": torch.cuda.get_device_properties(dev).L2_cache_size,
                    "sms": torch.cuda.get_device_properties(dev).multi_processor_count},
         "roofline": roofline,
