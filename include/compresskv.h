@@ -215,6 +215,25 @@ int compresskv_compress_layer_noalloc(const ckv_problem* p, const void* q_win, c
 int compresskv_read_device_status(const void* workspace, void* stream, int32_t* status);
 
 /* Static text for a status code. */
+/* Error-aware layer budgets (Sec. 3.4: the offline per-layer eviction
+ * errors, normalised as in Eq. 4, share the total budget after every layer
+ * gets a minimum m, no layer above a maximum M; Sec. 4 uses m = 32 and
+ * M = 3 * B_total / L).  Host only: no device work, no stream.
+ * layer_errors: host double [n_layers], e^(l) >= 0 in any common scale.
+ * total_budget: B_total, retained KV pairs summed over the layers.
+ * min_budget, max_budget: m and M; max_budget <= 0 selects 3*B_total/L.
+ * budgets: host int32 [n_layers], written: m plus the water-filled share
+ *   (a layer whose proportional share would pass M - m is capped and the
+ *   rest is shared again), rounded by largest remainder with ties to the
+ *   lower layer, so the budgets sum to B_total exactly.
+ * Returns CKV_ERR_BUDGET when n_layers*m > B_total or B_total > n_layers*M
+ * (or m > M), CKV_ERR_INVALID_ARG for a null pointer, n_layers < 1 or an
+ * error that is negative, NaN or infinite.  The layer budgets feed
+ * compresskv_compress_layer's `budgets` (one value per sequence). */
+int compresskv_allocate_layer_budgets(const double* layer_errors, int32_t n_layers,
+                                      int64_t total_budget, int32_t min_budget,
+                                      int32_t max_budget, int32_t* budgets);
+
 const char* compresskv_status_string(int status);
 
 #ifdef __cplusplus

@@ -11,6 +11,7 @@ from .compresskv import (  # noqa: F401
     LayerOutputs,
     Problem,
     Trace,
+    allocate_layer_budgets,
     compress_layer,
     compress_layer_noalloc,
     gather,

@@ -17,7 +17,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB_PATH = os.path.join(OUT_DIR, "libcompresskv.so")
-SOURCES = ["api.cu", "score_kernel.cu", "combine_kernel.cu", "select_kernel.cu", "gather_kernel.cu"]
+SOURCES = ["api.cu", "score_kernel.cu", "combine_kernel.cu", "select_kernel.cu", "gather_kernel.cu",
+           "budget_alloc.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -56,8 +57,9 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | N
     objs = []
 
     def compile_one(src: str) -> str:
-        obj = os.path.join(OUT_DIR, src.replace(".cu", ".o"))
-        cmd = [*common, "-c", os.path.join(CSRC, src), "-o", obj]
+        obj = os.path.join(OUT_DIR, os.path.splitext(src)[0] + ".o")
+        # host floating point in IEEE order (no contraction into fused multiply-adds)
+        cmd = [*common, "-Xcompiler", "-ffp-contract=off", "-c", os.path.join(CSRC, src), "-o", obj]
         res = subprocess.run(cmd, capture_output=True, text=True)
         if res.returncode != 0:
             raise RuntimeError(f"nvcc failed on {src}:\n{res.stdout}\n{res.stderr}")

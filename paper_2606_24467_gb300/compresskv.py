@@ -42,6 +42,7 @@ EXPORTED = (
     "compresskv_compress_layer",
     "compresskv_compress_layer_noalloc",
     "compresskv_read_device_status",
+    "compresskv_allocate_layer_budgets",
     "compresskv_status_string",
 )
 
@@ -99,6 +100,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         "compresskv_compress_layer_noalloc": (c_int32, [pp, vp, vp, vp, vp, i32p, vp, i32p, vp,
                                                          vp, vp, vp, vp, vp]),
         "compresskv_read_device_status": (c_int32, [vp, vp, i32p]),
+        "compresskv_allocate_layer_budgets": (c_int32, [POINTER(ctypes.c_double), c_int32,
+                                                        c_int64, c_int32, c_int32, i32p]),
         "compresskv_status_string": (ctypes.c_char_p, [c_int32]),
     }
     for name, (res, args) in sig.items():
@@ -286,6 +289,19 @@ def compress_layer_noalloc(problem: Problem, q_win, k, v, srh_mask, budgets, ind
         cu_out.ctypes.data_as(POINTER(c_int32)), _ptr(k_out), _ptr(v_out), _ptr(raw),
         _ptr(pooled), _ptr(device_status), _stream(stream)), "compresskv_compress_layer_noalloc")
     return cu_out
+
+
+def allocate_layer_budgets(layer_errors, total_budget: int, min_budget: int = 32,
+                           max_budget: int = 0) -> np.ndarray:
+    """Per-layer budgets from offline layer errors (Sec. 3.4); host only.
+    `max_budget` <= 0 selects 3 * total_budget / n_layers."""
+    err = np.ascontiguousarray(np.asarray(layer_errors, dtype=np.float64))
+    out = np.zeros(err.size, dtype=np.int32)
+    _check(load().compresskv_allocate_layer_budgets(
+        err.ctypes.data_as(POINTER(ctypes.c_double)), int(err.size), int(total_budget),
+        int(min_budget), int(max_budget), out.ctypes.data_as(POINTER(c_int32))),
+        "compresskv_allocate_layer_budgets")
+    return out
 
 
 def read_device_status(ws, stream=None) -> int:

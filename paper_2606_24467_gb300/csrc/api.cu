@@ -510,15 +510,18 @@ int run_select(const ckv_problem* p, const Info& I, const float* raw, const floa
     P.cu_out[s] = cu_out[s];
     if (s < I.B) max_n = std::max(max_n, I.n[s]);
   }
-  // A cluster of up to 8 CTAs per unit, about 4096 prefix tokens per CTA.
+  // A cluster of up to 8 CTAs per unit, about 4096 prefix tokens per CTA
+  // (one CTA per unit is several times slower: the four radix passes over a
+  // whole unit's keys serialise in one block).
+  const int r = (I.P - 1) / 2;
   const int C = std::min(8, std::max(1, (max_n + 4095) / 4096));
   const int S = std::max(32, ((max_n + C - 1) / C + 31) / 32 * 32);
-  const int r = (I.P - 1) / 2;
-  const bool fits = 2 * S + 2 * r <= select_max_smem_floats();
+  const int need = pooled_in ? S : 2 * S + 2 * r;  // floats of shared memory
+  const bool fits = need <= select_max_smem_floats();
   P.cluster = C;
   P.slice = S;
   P.smem_slice = fits ? 1 : 0;
-  const size_t smem = fits ? static_cast<size_t>(2 * S + 2 * r) * 4 : 0;
+  const size_t smem = fits ? static_cast<size_t>(need) * 4 : 0;
   Tracer tr{p->trace, stream};
   return traced(tr, CKV_KERNEL_SELECT, [&] { return launch_select(P, I.B * I.Hkv, smem, stream); });
 }

@@ -148,9 +148,10 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   const float* pin = p.pooled_in ? p.pooled_in + soff + lo : nullptr;
   // pooled scores of the slice: shared memory, else the workspace copy (or,
   // when they arrive already pooled, the caller's buffer, read only)
-  const float* pooled = in_smem ? s_dyn + S + 2 * r
-                                : (pin ? pin : p.pooled_ws + soff + lo);  // [len]
-  float* pooled_w = in_smem ? s_dyn + S + 2 * r : p.pooled_ws + soff + lo;
+  // (already pooled scores need no raw staging area in front of them)
+  float* const s_pooled = s_dyn + (pin ? 0 : S + 2 * r);
+  const float* pooled = in_smem ? s_pooled : (pin ? pin : p.pooled_ws + soff + lo);  // [len]
+  float* pooled_w = in_smem ? s_pooled : p.pooled_ws + soff + lo;
 
   pdl_launch_dependents();
   pdl_wait();  // scores come from the previous kernel
