@@ -86,6 +86,14 @@ enum {
 
 enum { CKV_DTYPE_F16 = 0, CKV_DTYPE_BF16 = 1 };
 enum { CKV_POOL_AVG = 0 };
+/* Selection scope.  PER_GROUP: every KV group keeps the tokens its own SRH
+ * heads rank highest, and a group without an SRH head is an error.
+ * PER_LAYER (Sec. 3.3 read literally: all heads of a layer share one set of
+ * retained tokens chosen by the layer's SRH heads, whose pooled scores are
+ * averaged): per sequence, the pooled scores of all groups are summed (a
+ * group without an SRH head adds nothing), one top-k is taken and every KV
+ * group keeps the same positions. */
+enum { CKV_SELECT_PER_GROUP = 0, CKV_SELECT_PER_LAYER = 1 };
 
 /* Kernel kinds reported through ckv_trace. */
 enum {
@@ -120,7 +128,7 @@ typedef struct ckv_problem {
   int32_t dtype;            /* CKV_DTYPE_F16 | CKV_DTYPE_BF16 for Q, K and V */
   int32_t pool_kind;        /* CKV_POOL_AVG */
   float scale;              /* softmax scale; 0 selects 1/sqrt(head_dim) */
-  int32_t reserved;         /* must be 0 */
+  int32_t selection;        /* CKV_SELECT_PER_GROUP or CKV_SELECT_PER_LAYER */
   const int32_t* cu_seqlens;/* host [batch+1] */
   int64_t kv_token_stride;  /* elements between consecutive tokens of K/V */
   int64_t kv_head_stride;   /* elements between KV heads of K/V */
@@ -161,7 +169,11 @@ int compresskv_score(const ckv_problem* p, const void* q_win, const void* k,
  * budgets: host int32 [batch] (per sequence, including the W window tokens).
  * indices: device int32 [num_kv_heads][O_total] (output layout).
  * cu_out: host int32 [batch+1], written.
- * pooled_scores: optional device float in score layout (NULL for none). */
+ * pooled_scores: optional device float in score layout (NULL for none;
+ *   must be NULL under CKV_SELECT_PER_LAYER, whose keys are the pooled sum
+ *   of all groups' raw scores).
+ * Under CKV_SELECT_PER_LAYER every group's row of `indices` receives the
+ * sequence's shared selection. */
 int compresskv_select(const ckv_problem* p, const float* raw_scores,
                       const int32_t* budgets, int32_t* indices, int32_t* cu_out,
                       float* pooled_scores, void* workspace, size_t workspace_bytes,
@@ -178,7 +190,10 @@ int compresskv_gather(const ckv_problem* p, const int32_t* indices, const int32_
 
 /* Steps 1-4 fused for one layer: score, select, gather.
  * raw_scores / pooled_scores are optional outputs in score layout (NULL: raw
- * scores are not materialised, pooled scores stay in the workspace).
+ * scores are not materialised, pooled scores stay in the workspace); they are
+ * per group in both selection scopes (a group without an SRH head gets
+ * zeros under CKV_SELECT_PER_LAYER), and the per-layer selection ranks their
+ * sum over the groups.
  * cu_out: host int32 [batch+1], written. */
 int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const void* k,
                               const void* v, const uint8_t* srh_mask, const int32_t* budgets,

@@ -49,3 +49,29 @@ def brute_unit(q_heads, k_unit, window, pool_width, budget, scale):
     ranked = sorted(range(n), key=lambda j: (-pooled[j], j))
     chosen = sorted(ranked[:k])
     return raw, pooled, chosen + list(range(n, L))
+
+
+def brute_layer_shared(q_heads_per_group, k_per_group, window, pool_width, budget, scale):
+    """Layer-shared selection (Sec. 3.3 read literally) by brute force: every
+    group's SRH heads are scored against that group's keys, the pooled
+    vectors of all groups are added (math.fsum, group order) and one top-k
+    with ties to the lower position is kept for the whole layer.
+    q_heads_per_group: per group, a list over its SRH heads (possibly empty)
+    of W lists of d floats; k_per_group: per group, L lists of d floats.
+    Returns (pooled_sum, indices)."""
+    L = len(k_per_group[0])
+    W = window
+    if budget < W:
+        raise ValueError("budget smaller than window")
+    if L <= W:
+        return [], list(range(L))
+    n = L - W
+    pooled_per_group = []
+    for heads, keys in zip(q_heads_per_group, k_per_group):
+        if heads:
+            _, pooled, _ = brute_unit(heads, keys, window, pool_width, budget, scale)
+            pooled_per_group.append(pooled)
+    total = [math.fsum(pg[j] for pg in pooled_per_group) for j in range(n)]
+    k = min(budget, L) - W
+    ranked = sorted(range(n), key=lambda j: (-total[j], j))
+    return total, sorted(ranked[:k]) + list(range(n, L))

@@ -34,9 +34,19 @@ for every sequence ``s`` and GQA KV group ``g`` (a *unit*):
 Every step is written with plain numpy on float64 copies of the inputs; the
 only library primitives are a dot product, ``exp`` and a sort.
 
-Readings where the paper is silent (each also listed in the design notes):
-per-group selection with the group's own SRH heads; a group with no SRH head
-is an error; the softmax of window query ``w`` spans all causal keys
+Two selection scopes:
+
+* per group (the default): steps 3-6 run per unit with the group's own SRH
+  heads; a group with no SRH head is an error;
+* per layer (Sec. 3.3 read literally: all heads of a layer share one set of
+  retained indices chosen by the layer's SRH heads, whose pooled window
+  scores are averaged): per sequence, every SRH head's attention (against
+  its own group's keys) is summed over the window and pooled, the pooled
+  vectors are summed over all SRH heads of the layer (the average times the
+  fixed head count), the top ``k`` are kept and every KV group retains the
+  same positions; groups without an SRH head are allowed.
+
+Readings where the paper is silent (each also listed in the design notes): the softmax of window query ``w`` spans all causal keys
 including earlier window keys, only prefix columns are scored; the budget
 ``B`` counts the window tokens; ``B < W`` is an error and ``B >= L`` keeps
 everything; retained tokens are listed in ascending position.
@@ -195,6 +205,15 @@ def compress_unit(q_heads: np.ndarray, k_unit: np.ndarray, window: int, pool_wid
 # One layer over a packed (cu_seqlens) batch, in the library's output layout
 # ---------------------------------------------------------------------------
 @dataclass
+class SharedSelection:
+    """Per-layer (shared) selection of one sequence."""
+    pooled: np.ndarray       # [n] pooled scores summed over the layer's SRH heads
+    k: int
+    tau: float
+    indices: np.ndarray      # [min(B, L)] ascending positions, the same for every group
+
+
+@dataclass
 class LayerResult:
     units: dict              # (s, g) -> UnitResult
     raw: np.ndarray          # [H_kv, sum_s n_s] float64
@@ -204,6 +223,7 @@ class LayerResult:
     cu_prefix: np.ndarray    # [B+1] offsets of the prefix scores
     k_out: np.ndarray        # [sum_s kept_s, H_kv, d]  (input dtype)
     v_out: np.ndarray
+    shared: dict = field(default_factory=dict)  # s -> SharedSelection (layer scope)
 
 
 def default_scale(head_dim: int) -> float:
@@ -212,14 +232,17 @@ def default_scale(head_dim: int) -> float:
 
 def compress_layer(q_win, k, v, cu_seqlens, srh_mask, budgets, window: int,
                    pool_width: int, scale: float | None = None,
-                   keep_attn: bool = False) -> LayerResult:
+                   keep_attn: bool = False, selection: str = "group") -> LayerResult:
     """Oracle of one layer's compression.
 
     q_win: ``[B, H_q, W, d]`` window queries (position ``L_s - W + w``).
     k, v:  ``[T, H_kv, d]`` packed keys/values, sequence ``s`` at rows
            ``cu_seqlens[s] : cu_seqlens[s+1]``.
     srh_mask: ``[H_q]`` booleans; budgets: ``[B]`` ints (per sequence).
+    selection: ``"group"`` or ``"layer"`` (see the module docstring).
     """
+    if selection not in ("group", "layer"):
+        raise OracleError("selection must be 'group' or 'layer'")
     q_win = np.asarray(q_win)
     k = np.asarray(k)
     v = np.asarray(v)
@@ -245,6 +268,48 @@ def compress_layer(q_win, k, v, cu_seqlens, srh_mask, budgets, window: int,
     q64 = q_win.astype(np.float64)
     k64 = k.astype(np.float64)
     units = {}
+    shared = {}
+    if selection == "layer":
+        if not any(srh_heads(srh_mask, g, G) for g in range(H_kv)) and any(
+                Ls > window for Ls in lengths):
+            raise OracleError("the layer has no SRH head")
+        for s in range(B):
+            Ls, n, kept = lengths[s], n_s[s], kept_s[s]
+            layer_pooled = np.zeros(n, dtype=np.float64)
+            for g in range(H_kv):
+                heads = srh_heads(srh_mask, g, G)
+                ku = k64[cu[s]:cu[s + 1], g]
+                if heads and Ls > window:
+                    # Sec. 3.3: each head's window-summed attention is pooled,
+                    # then the heads' vectors are combined
+                    attn = [window_attention(q64[s, h], ku, scale) for h in heads]
+                    for A in attn:
+                        layer_pooled += pool_avg(raw_scores([A], n), pool_width)
+                    g_raw = raw_scores(attn, n)
+                    g_pooled = pool_avg(g_raw, pool_width)
+                else:
+                    attn, g_raw, g_pooled = [], np.zeros(n), np.zeros(n)
+                units[(s, g)] = UnitResult(heads, g_raw, g_pooled, 0, float("nan"),
+                                           np.zeros(0, dtype=np.int64),
+                                           attn if keep_attn else [])
+                raw[g, cu_prefix[s]:cu_prefix[s + 1]] = g_raw
+                pooled[g, cu_prefix[s]:cu_prefix[s + 1]] = g_pooled
+            if Ls <= window:
+                idx = np.arange(Ls, dtype=np.int64)
+                kk, tau = 0, float("nan")
+            else:
+                kk = kept - window
+                sel = select_top(layer_pooled, kk)
+                idx = np.concatenate([sel, np.arange(n, Ls, dtype=np.int64)])
+                tau = kth_value(layer_pooled, kk)
+            shared[s] = SharedSelection(layer_pooled, kk, tau, idx)
+            for g in range(H_kv):
+                units[(s, g)].k, units[(s, g)].tau, units[(s, g)].indices = kk, tau, idx
+                indices[g, cu_out[s]:cu_out[s + 1]] = idx
+                rows = cu[s] + idx
+                k_out[cu_out[s]:cu_out[s + 1], g] = k[rows, g]
+                v_out[cu_out[s]:cu_out[s + 1], g] = v[rows, g]
+        return LayerResult(units, raw, pooled, indices, cu_out, cu_prefix, k_out, v_out, shared)
     for s in range(B):
         for g in range(H_kv):
             heads = srh_heads(srh_mask, g, G)

@@ -30,6 +30,8 @@ STATIC_SCRATCH_BYTES = 16 * 1024 * 1024
 CKV_DTYPE_F16 = 0
 CKV_DTYPE_BF16 = 1
 CKV_POOL_AVG = 0
+CKV_SELECT_PER_GROUP = 0
+CKV_SELECT_PER_LAYER = 1
 KERNEL_KINDS = {1: "score", 2: "combine", 3: "select", 4: "gather"}
 
 EXPORTED = (
@@ -56,7 +58,7 @@ class CkvProblem(ctypes.Structure):
     _fields_ = [("batch", c_int32), ("num_q_heads", c_int32), ("num_kv_heads", c_int32),
                 ("head_dim", c_int32), ("window", c_int32), ("pool_width", c_int32),
                 ("dtype", c_int32), ("pool_kind", c_int32), ("scale", c_float),
-                ("reserved", c_int32), ("cu_seqlens", POINTER(c_int32)),
+                ("selection", c_int32), ("cu_seqlens", POINTER(c_int32)),
                 ("kv_token_stride", c_int64), ("kv_head_stride", c_int64),
                 ("q_batch_stride", c_int64), ("q_head_stride", c_int64),
                 ("q_win_stride", c_int64), ("trace", POINTER(CkvTrace))]
@@ -146,7 +148,10 @@ class Problem:
     """
 
     def __init__(self, q_win: torch.Tensor, k: torch.Tensor, cu_seqlens, window: int,
-                 pool_width: int, scale: float = 0.0, trace: "Trace | None" = None):
+                 pool_width: int, scale: float = 0.0, trace: "Trace | None" = None,
+                 selection: str = "group"):
+        """``selection``: "group" (each KV group keeps its own SRH heads'
+        choice) or "layer" (one choice per sequence shared by every group)."""
         if k.dtype not in (torch.float16, torch.bfloat16) or q_win.dtype != k.dtype:
             raise CompressKVError(CKV_ERR_INVALID_ARG, "Q and K must share an f16/bf16 dtype")
         self._cu, cu_ptr = _i32(cu_seqlens)
@@ -161,7 +166,9 @@ class Problem:
         s.dtype = CKV_DTYPE_BF16 if k.dtype == torch.bfloat16 else CKV_DTYPE_F16
         s.pool_kind = CKV_POOL_AVG
         s.scale = float(scale)
-        s.reserved = 0
+        if selection not in ("group", "layer"):
+            raise CompressKVError(CKV_ERR_INVALID_ARG, "selection must be 'group' or 'layer'")
+        s.selection = CKV_SELECT_PER_LAYER if selection == "layer" else CKV_SELECT_PER_GROUP
         s.cu_seqlens = cu_ptr
         s.kv_token_stride = k.stride(0)
         s.kv_head_stride = k.stride(1)

@@ -87,6 +87,7 @@ int device_facts(DeviceFacts** out) {
 struct Info {
   int B = 0, Hq = 0, Hkv = 0, G = 0, W = 0, P = 0;
   bool bf16 = false;
+  bool layer = false;  // CKV_SELECT_PER_LAYER
   float scale = 0.f;
   std::vector<int> cu, len, n, cu_prefix;
   long long T = 0, p_total = 0;
@@ -105,7 +106,8 @@ int validate(const ckv_problem* p, Info& I) {
   if (p->pool_width < 1 || p->pool_width % 2 == 0 || p->pool_width > 63) return CKV_ERR_INVALID_ARG;
   if (p->dtype != CKV_DTYPE_F16 && p->dtype != CKV_DTYPE_BF16) return CKV_ERR_INVALID_ARG;
   if (p->pool_kind != CKV_POOL_AVG) return CKV_ERR_UNSUPPORTED;
-  if (p->reserved != 0) return CKV_ERR_INVALID_ARG;
+  if (p->selection != CKV_SELECT_PER_GROUP && p->selection != CKV_SELECT_PER_LAYER)
+    return CKV_ERR_INVALID_ARG;
   if (!(p->scale >= 0.f) || std::isinf(p->scale)) return CKV_ERR_INVALID_ARG;
   if (p->kv_token_stride <= 0 || p->kv_head_stride <= 0 || p->kv_token_stride % 8 ||
       p->kv_head_stride % 8)
@@ -120,6 +122,7 @@ int validate(const ckv_problem* p, Info& I) {
   I.W = p->window;
   I.P = p->pool_width;
   I.bf16 = p->dtype == CKV_DTYPE_BF16;
+  I.layer = p->selection == CKV_SELECT_PER_LAYER;
   I.scale = p->scale > 0.f ? p->scale : 1.0f / std::sqrt(static_cast<float>(kHeadDim));
   I.cu.assign(p->cu_seqlens, p->cu_seqlens + I.B + 1);
   if (I.cu[0] != 0) return CKV_ERR_INVALID_ARG;
@@ -191,10 +194,11 @@ struct Workspace {
   float* pooled = nullptr;   // score layout
   uint16_t* expo = nullptr;  // one set's exponent table
   float* refs = nullptr;     // one set's reference table
+  float* shared = nullptr;   // per-layer selection: summed scores [sum_s n_s]
 };
 
 struct WorkspaceLayout {
-  size_t pooled, expo, refs, total;
+  size_t pooled, expo, refs, shared, total;
 };
 
 WorkspaceLayout workspace_layout(const Info& I) {
@@ -209,7 +213,8 @@ WorkspaceLayout workspace_layout(const Info& I) {
   W.pooled = kStatusBytes + kPartialBytes;
   W.expo = W.pooled + align256(static_cast<size_t>(I.Hkv) * I.p_total * sizeof(float));
   W.refs = W.expo + align256(static_cast<size_t>(e) * sizeof(uint16_t));
-  W.total = W.refs + align256(static_cast<size_t>(r) * sizeof(float));
+  W.shared = W.refs + align256(static_cast<size_t>(r) * sizeof(float));
+  W.total = W.shared + (I.layer ? align256(static_cast<size_t>(I.p_total) * sizeof(float)) : 0);
   return W;
 }
 
@@ -224,6 +229,7 @@ int carve(const Info& I, void* ws, size_t bytes, Workspace& out) {
   out.pooled = reinterpret_cast<float*>(b + W.pooled);
   out.expo = reinterpret_cast<uint16_t*>(b + W.expo);
   out.refs = reinterpret_cast<float*>(b + W.refs);
+  out.shared = reinterpret_cast<float*>(b + W.shared);
   return CKV_OK;
 }
 
@@ -298,10 +304,13 @@ int srh_lists(const Info& I, const uint8_t* mask, SrhLists& S) {
       if (mask[h]) S.heads.push_back(static_cast<uint8_t>(h));
     S.off[g + 1] = static_cast<uint16_t>(S.heads.size());
     const int cnt = S.off[g + 1] - S.off[g];
-    if (cnt == 0 && any_scored) return CKV_ERR_EMPTY_SRH_GROUP;
+    // per-group selection needs an SRH head in every group; per-layer
+    // selection only somewhere in the layer
+    if (cnt == 0 && any_scored && !I.layer) return CKV_ERR_EMPTY_SRH_GROUP;
     S.rows[g] = cnt * I.W;
     if (S.rows[g] > kMaxQRows) return CKV_ERR_UNSUPPORTED;
   }
+  if (I.layer && S.heads.empty() && any_scored) return CKV_ERR_EMPTY_SRH_GROUP;
   return CKV_OK;
 }
 
@@ -379,6 +388,17 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
   std::vector<UnitSet> sets;
   plan_sets(I, sets);
   Tracer tr{p->trace, stream};
+  // Per-layer selection sums the groups' scores: a group without an SRH head
+  // contributes zeros.
+  for (int g = 0; g < I.Hkv; ++g) {
+    if (S.rows[g] > 0) continue;
+    const size_t row = static_cast<size_t>(I.p_total) * sizeof(float);
+    if (cudaMemsetAsync(pooled + static_cast<size_t>(g) * I.p_total, 0, row, stream) != cudaSuccess)
+      return CKV_ERR_CUDA;
+    if (raw && cudaMemsetAsync(raw + static_cast<size_t>(g) * I.p_total, 0, row, stream) !=
+                   cudaSuccess)
+      return CKV_ERR_CUDA;
+  }
   for (const UnitSet& set : sets) {
     const int u0 = set.u0;
     const int nu = set.u1 - set.u0;
@@ -387,16 +407,23 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
     // rows); every unit gets one item, the remaining items go one at a time
     // to the unit with the largest work per item, then each unit's tiles are
     // split into balanced ranges.
+    // (Units of a group without an SRH head -- per-layer selection only --
+    // get no items.)
     auto cost = [&](const Unit& U) { return 64LL + ((S.rows[U.g] + 15) & ~15); };
     std::vector<int> cnt(nu, 1);
     std::vector<long long> uw(nu);
-    for (int u = 0; u < nu; ++u)
+    int active = 0;
+    for (int u = 0; u < nu; ++u) {
       uw[u] = static_cast<long long>(units[u0 + u].tiles) * cost(units[u0 + u]);
-    const int target = std::min(kMaxItems, std::max(nu, F->sms));
-    for (int extra = target - nu; extra > 0; --extra) {
+      cnt[u] = S.rows[units[u0 + u].g] > 0 ? 1 : 0;
+      active += cnt[u];
+    }
+    if (active == 0) continue;
+    const int target = std::min(kMaxItems, std::max(active, F->sms));
+    for (int extra = target - active; extra > 0; --extra) {
       int best = -1;
       for (int u = 0; u < nu; ++u) {
-        if (cnt[u] >= units[u0 + u].tiles) continue;
+        if (cnt[u] == 0 || cnt[u] >= units[u0 + u].tiles) continue;
         if (best < 0 || uw[u] * cnt[best] > uw[best] * cnt[u]) best = u;
       }
       if (best < 0) break;
@@ -404,7 +431,8 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
     }
     // Combine items: chunks of 32-token quarters, about four CTAs per SM.
     long long quarters = 0;
-    for (int u = 0; u < nu; ++u) quarters += units[u0 + u].quarters;
+    for (int u = 0; u < nu; ++u)
+      if (cnt[u] > 0) quarters += units[u0 + u].quarters;
     const long long ctarget = std::max(1, std::min(kMaxItems - nu, 4 * F->sms));
     int chunk_q = static_cast<int>(std::max(8LL, (quarters + ctarget - 1) / ctarget));
     int max_nr = 8;
@@ -421,6 +449,7 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
     for (int u = 0; u < nu; ++u) {
       const Unit& U = units[u0 + u];
       const int c_u = cnt[u];
+      if (c_u == 0) continue;
       const int nr = expo_stride(S.rows[U.g]);
       if (n_items + c_u > kMaxItems) return CKV_ERR_UNSUPPORTED;
       for (int c = 0; c < c_u; ++c) {
@@ -487,6 +516,8 @@ int run_select(const ckv_problem* p, const Info& I, const float* raw, const floa
   P.raw = raw;
   P.pooled_in = pooled_in;
   P.pooled_out = pooled_in ? nullptr : pooled;
+  P.layer_scope = I.layer ? 1 : 0;
+  P.shared_ws = ws.shared;
   P.pooled_ws = ws.pooled;
   P.indices = indices;
   P.status = ws.status;
@@ -523,7 +554,8 @@ int run_select(const ckv_problem* p, const Info& I, const float* raw, const floa
   P.smem_slice = fits ? 1 : 0;
   const size_t smem = fits ? static_cast<size_t>(need) * 4 : 0;
   Tracer tr{p->trace, stream};
-  return traced(tr, CKV_KERNEL_SELECT, [&] { return launch_select(P, I.B * I.Hkv, smem, stream); });
+  const int n_units = I.layer ? I.B : I.B * I.Hkv;
+  return traced(tr, CKV_KERNEL_SELECT, [&] { return launch_select(P, n_units, smem, stream); });
 }
 
 int run_gather(const ckv_problem* p, const Info& I, const int32_t* indices,
@@ -610,6 +642,9 @@ int compresskv_select(const ckv_problem* p, const float* raw_scores, const int32
   std::vector<int> co;
   if ((rc = output_layout(I, budgets, co)) != CKV_OK) return rc;
   if (!cu_out) return CKV_ERR_INVALID_ARG;
+  // per-layer selection pools the groups' summed raw scores: there is no
+  // per-group pooled output to write
+  if (I.layer && pooled_scores) return CKV_ERR_INVALID_ARG;
   Workspace ws;
   if ((rc = carve(I, workspace, workspace_bytes, ws)) != CKV_OK) return rc;
   std::copy(co.begin(), co.end(), cu_out);

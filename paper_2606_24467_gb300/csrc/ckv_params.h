@@ -95,6 +95,8 @@ struct SelectParams {
   int slice;                   // prefix tokens per CTA (multiple of 32)
   int smem_slice;              // 1: raw and pooled slices live in shared memory
   int gather;                  // 1: also copy the retained K/V rows
+  int layer_scope;             // 1: one selection per sequence, shared by every KV group
+  float* shared_ws;            // layer scope: workspace row for the summed scores [p_total]
   int cu_seqlens[kMaxBatch + 1];
   int cu_prefix[kMaxBatch + 1];
   int cu_out[kMaxBatch + 1];

@@ -12,11 +12,13 @@
 //   2. raw_j = sum_q e_qj * 2^(R - bias_q)   (every weight is <= 1);
 //   3. pooled_j = (sum_{t=-h..h} raw_{j+t}) / P with zeros outside [0, n),
 //      summed in a fixed order.
-// One CTA per chunk of 32-key quarters of one unit.  It first tabulates the
-// weights 2^(R - bias_q) of every quarter it touches (the chunk plus an
-// h-key halo on each side) in shared memory, then streams the exponent rows
-// of those keys -- one contiguous region -- with the whole block, kLoadBatch
-// 16-byte loads in flight per thread.  Thread tid always meets the same
+// One CTA per chunk of 32-key quarters of one unit.  The unit's pairs, the
+// references of every quarter the chunk touches (the chunk plus an h-key
+// halo on each side) and the first exponent rows are requested together;
+// the weights 2^(R - bias_q) are then tabulated in shared memory and the
+// exponent rows of those keys -- one contiguous region -- are streamed by the
+// whole block, two batches of kLoadBatch 16-byte loads in flight per thread.
+// Thread tid always meets the same
 // 8-column chunk of a row (tid % cpr, where cpr = Nr / 8 divides 32); the
 // cpr threads of a row are adjacent lanes and add their dot products by
 // shuffles.  Raw scores of the chunk and halo stay in shared memory for the
@@ -31,7 +33,7 @@ namespace ckv {
 namespace {
 
 constexpr int kCombThreads = 256;
-constexpr int kLoadBatch = 8;  // 16-byte loads in flight per thread
+constexpr int kLoadBatch = 4;  // 16-byte loads per batch (two batches in flight per thread)
 constexpr int kPairSlots = 2048;  // softmax pairs staged per round
 static_assert(kMaxQRows <= kCombThreads, "one thread per query row");
 
@@ -61,6 +63,8 @@ __global__ void __launch_bounds__(kCombThreads)
   __shared__ float2 s_pairs[kPairSlots];
 
   const int tid = threadIdx.x;
+  const int warp = tid >> 5;
+  const int lane = tid & 31;
   const WorkItem it = p.items[blockIdx.x];
   const int s = it.seq;
   const int g = it.group;
@@ -70,6 +74,7 @@ __global__ void __launch_bounds__(kCombThreads)
   const int N = (p.srh_off[g + 1] - p.srh_off[g]) * W;
   const int Nr = expo_stride(N);
   const int cpr = Nr >> 3;  // 16-byte chunks per key row (a power of two <= 32)
+  const int lg_cpr = __ffs(cpr) - 1;
   const int col = tid & (cpr - 1);
   const int h = (p.pool_width - 1) >> 1;
   const int a = it.t0 * 32;
@@ -86,23 +91,48 @@ __global__ void __launch_bounds__(kCombThreads)
   for (int i = tid; i < span; i += kCombThreads) s_raw[i] = 0.f;
   pdl_wait();  // pairs and tables come from the scoring kernel
 
-  // 1. per-query log2 softmax denominators: the unit's item pairs are staged
-  //    in shared memory (all loads in flight at once), then merged in item
-  //    order by one thread per query
+  // Everything below depends on three independent reads -- the unit's
+  // softmax pairs, the references of the quarters touched and the exponent
+  // rows -- so all three are issued before any of them is waited on.
+  const uint4* E4 = reinterpret_cast<const uint4*>(p.expo + it.eoff);
+  const int f_lo = ea * cpr;
+  const int f_hi = eb * cpr;
+  uint4 ev[kLoadBatch];
+  auto load_batch = [&](int f0, uint4 (&dst)[kLoadBatch]) {
+#pragma unroll
+    for (int u = 0; u < kLoadBatch; ++u) {
+      const int f = f0 + u * kCombThreads + tid;
+      dst[u] = f < f_hi ? __ldg(E4 + f) : make_uint4(0u, 0u, 0u, 0u);
+    }
+  };
+  load_batch(f_lo, ev);
+  const float* R = p.refs + it.roff + static_cast<long long>(q0) * Nr;
+  for (int i = tid; i < nqt * Nr; i += kCombThreads) s_w[i] = R[i];
+  const int per = kPairSlots / N;  // items staged per round
+  const int ni0 = min(per, static_cast<int>(it.count));
+  auto stage_pairs = [&](int i0, int ni) {
+    for (int ii = warp; ii < ni; ii += kCombThreads / 32) {
+      const float2* src = p.partials + static_cast<long long>(it.first + i0 + ii) * kMaxQRows;
+      for (int q = lane; q < N; q += 32) s_pairs[ii * N + q] = src[q];
+    }
+  };
+  stage_pairs(0, ni0);
+  __syncthreads();
+
+  // 1. per-query log2 softmax denominators, item pairs merged in order (one
+  //    thread per query; units with many items take several staging rounds)
   {
-    const int per = kPairSlots / N;  // items per staging round
-    float m = -INFINITY, z = 0.f;    // thread tid < N: query tid
+    float m = -INFINITY, z = 0.f;
     for (int i0 = 0; i0 < it.count; i0 += per) {
       const int ni = min(per, it.count - i0);
-      for (int i = tid; i < ni * N; i += kCombThreads) {
-        const int ii = i / N;
-        const int q = i - ii * N;
-        s_pairs[i] = p.partials[static_cast<long long>(it.first + i0 + ii) * kMaxQRows + q];
+      if (i0 > 0) {
+        __syncthreads();
+        stage_pairs(i0, ni);
+        __syncthreads();
       }
-      __syncthreads();
-      for (int q = tid; q < N; q += kCombThreads) {  // N <= kCombThreads: one query per thread
+      if (tid < N) {
         for (int ii = 0; ii < ni; ++ii) {
-          const float2 pr = s_pairs[ii * N + q];
+          const float2 pr = s_pairs[ii * N + tid];
           if (pr.x == -INFINITY) continue;
           if (pr.x > m) {
             z = fmaf(z, ex2_approx(m - pr.x), pr.y);
@@ -112,40 +142,36 @@ __global__ void __launch_bounds__(kCombThreads)
           }
         }
       }
-      __syncthreads();
     }
     if (tid < N) s_bias[tid] = m + __log2f(z);
   }
   __syncthreads();
 
-  // 2. weights 2^(R - bias_q) of the quarters touched
-  const float* R = p.refs + it.roff + static_cast<long long>(q0) * Nr;
+  // 2. weights 2^(R - bias_q) of the quarters touched, in place
   for (int i = tid; i < nqt * Nr; i += kCombThreads) {
-    const int qq = i / Nr;
-    const int cc = i - qq * Nr;
-    s_w[i] = cc < N ? ex2_approx(R[i] - s_bias[cc]) : 0.f;
+    const int cc = i & (Nr - 1);
+    s_w[i] = cc < N ? ex2_approx(s_w[i] - s_bias[cc]) : 0.f;
   }
   __syncthreads();
 
-  // 3. raw scores of the keys [ea, eb): one contiguous run of exponent rows
-  const uint4* E4 = reinterpret_cast<const uint4*>(p.expo + it.eoff);
-  const int f_lo = ea * cpr;
-  const int f_hi = eb * cpr;
+  // 3. raw scores of the keys [ea, eb): one contiguous run of exponent rows,
+  //    the next batch in flight while the current one is reduced
   for (int f0 = f_lo; f0 < f_hi; f0 += kLoadBatch * kCombThreads) {
-    uint4 ev[kLoadBatch];
+    uint4 nx[kLoadBatch];
+    const int f1 = f0 + kLoadBatch * kCombThreads;
+    if (f1 < f_hi) load_batch(f1, nx);
 #pragma unroll
     for (int u = 0; u < kLoadBatch; ++u) {
       const int f = f0 + u * kCombThreads + tid;
-      ev[u] = f < f_hi ? __ldg(E4 + f) : make_uint4(0u, 0u, 0u, 0u);
-    }
-#pragma unroll
-    for (int u = 0; u < kLoadBatch; ++u) {
-      const int f = f0 + u * kCombThreads + tid;
-      const int row = f / cpr;  // key position
+      const int row = f >> lg_cpr;  // key position
       const int qq = min((row >> 5) - q0, nqt - 1);
       float v = dot8(ev[u], s_w + qq * Nr + 8 * col);
       for (int off = cpr >> 1; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
       if (f < f_hi && col == 0) s_raw[row - base] = v;
+    }
+    if (f1 < f_hi) {
+#pragma unroll
+      for (int u = 0; u < kLoadBatch; ++u) ev[u] = nx[u];
     }
   }
   __syncthreads();

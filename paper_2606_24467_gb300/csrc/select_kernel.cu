@@ -126,8 +126,13 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   const int warp = tid >> 5;
   const int lane = tid & 31;
   const int u = blockIdx.x / C;
-  const int s = u / p.num_kv_heads;
-  const int g = u - s * p.num_kv_heads;
+  // per-layer selection: one unit per sequence whose keys are the pooled
+  // scores summed over the KV groups, and whose indices every group keeps
+  const bool layer = p.layer_scope != 0;
+  const int s = layer ? u : u / p.num_kv_heads;
+  const int g = layer ? 0 : u - s * p.num_kv_heads;
+  const int nrows = layer ? p.num_kv_heads : 1;  // score rows summed into the keys
+  const long long rstride = p.p_total;
   const int seq0 = p.cu_seqlens[s];
   const int L = p.cu_seqlens[s + 1] - seq0;
   const int W = p.window;
@@ -135,6 +140,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   const int out0 = p.cu_out[s];
   const int kept = p.cu_out[s + 1] - out0;
   int32_t* out = p.indices + static_cast<long long>(g) * p.o_total + out0;
+  const long long ostride = p.o_total;  // index rows of the groups (layer scope writes all)
   const long long soff = static_cast<long long>(g) * p.p_total + p.cu_prefix[s];
   const float* raw = p.raw + soff;
   float* pout = p.pooled_out ? p.pooled_out + soff : nullptr;
@@ -150,8 +156,9 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   // when they arrive already pooled, the caller's buffer, read only)
   // (already pooled scores need no raw staging area in front of them)
   float* const s_pooled = s_dyn + (pin ? 0 : S + 2 * r);
-  const float* pooled = in_smem ? s_pooled : (pin ? pin : p.pooled_ws + soff + lo);  // [len]
-  float* pooled_w = in_smem ? s_pooled : p.pooled_ws + soff + lo;
+  float* pooled_w =
+      in_smem ? s_pooled : (layer ? p.shared_ws + p.cu_prefix[s] + lo : p.pooled_ws + soff + lo);
+  const float* pooled = in_smem || layer || !pin ? pooled_w : pin;  // [len]
 
   pdl_launch_dependents();
   pdl_wait();  // scores come from the previous kernel
@@ -159,13 +166,20 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   // 1. pooling ---------------------------------------------------------------
   const float fP = static_cast<float>(p.pool_width);
   if (len > 0 && pin) {
-    if (in_smem) {  // already pooled: stage the slice
+    if (in_smem || layer) {  // already pooled: stage (and sum) the slice
       for (int base = 0; base < len; base += 8 * kSelThreads) {
         float v[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
           const int li = base + i * kSelThreads + tid;
           v[i] = li < len ? pin[li] : 0.f;
+        }
+        for (int rr = 1; rr < nrows; ++rr) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int li = base + i * kSelThreads + tid;
+            if (li < len) v[i] += pin[rr * rstride + li];
+          }
         }
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
@@ -184,6 +198,14 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
           const int li = base + i * kSelThreads + tid;
           const int j = lo - r + li;
           v[i] = (li < span && j >= 0 && j < n) ? raw[j] : 0.f;
+        }
+        for (int rr = 1; rr < nrows; ++rr) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int li = base + i * kSelThreads + tid;
+            const int j = lo - r + li;
+            if (li < span && j >= 0 && j < n) v[i] += raw[rr * rstride + j];
+          }
         }
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
@@ -205,7 +227,11 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
         float a = 0.f;
         for (int t = -r; t <= r; ++t) {
           const int jj = j + t;
-          a += (jj >= 0 && jj < n) ? raw[jj] : 0.f;
+          if (jj >= 0 && jj < n) {
+            float x = raw[jj];
+            for (int rr = 1; rr < nrows; ++rr) x += raw[rr * rstride + jj];
+            a += x;
+          }
         }
         const float pv = a / fP;
         pooled_w[i] = pv;
@@ -219,21 +245,23 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
     const int per = (L + C - 1) / C;
     const int a0 = min(L, crank * per);
     const int a1 = min(L, a0 + per);
-    for (int i = a0 + tid; i < a1; i += kSelThreads) out[i] = i;
+    for (int i = a0 + tid; i < a1; i += kSelThreads)
+      for (int rr = 0; rr < nrows; ++rr) out[rr * ostride + i] = i;
     if (p.gather && a1 > a0) {
       __syncthreads();  // the indices written above are read back by the copy
-      copy_kv_rows(p, seq0, g, out, out0, a0, a1 - a0);
+      for (int rr = 0; rr < nrows; ++rr) copy_kv_rows(p, seq0, g + rr, out, out0, a0, a1 - a0);
     }
     return;  // uniform over the cluster: no cluster barrier is pending
   }
   const int k = kept - W;  // 0 <= k < n
   if (crank == C - 1) {
-    for (int w = tid; w < W; w += kSelThreads) out[k + w] = n + w;
+    for (int w = tid; w < W; w += kSelThreads)
+      for (int rr = 0; rr < nrows; ++rr) out[rr * ostride + k + w] = n + w;
   }
   if (k == 0) {  // window only (uniform over the cluster)
     if (p.gather && crank == C - 1) {
       __syncthreads();
-      copy_kv_rows(p, seq0, g, out, out0, k, W);
+      for (int rr = 0; rr < nrows; ++rr) copy_kv_rows(p, seq0, g + rr, out, out0, k, W);
     }
     return;
   }
@@ -370,7 +398,8 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
         in && key == tau && (eq_seen + __popc(meq & lanemask_lt(lane))) < need_eq;
     const uint32_t msel = mgt | __ballot_sync(0xffffffffu, take_eq);
     const int o = pos + __popc(msel & lanemask_lt(lane));
-    if ((msel & (1u << lane)) && o < k) out[o] = lo + i;
+    if ((msel & (1u << lane)) && o < k)
+      for (int rr = 0; rr < nrows; ++rr) out[rr * ostride + o] = lo + i;
     pos += __popc(msel);
     eq_seen += __popc(meq);
   }
@@ -379,8 +408,10 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
     __syncthreads();  // the indices written above are read back by the copy
     const int cta_first = s_cta_first;
     const int cta_count = min(k - cta_first, s_cta_count);
-    if (cta_count > 0) copy_kv_rows(p, seq0, g, out, out0, cta_first, cta_count);
-    if (crank == C - 1) copy_kv_rows(p, seq0, g, out, out0, k, W);
+    for (int rr = 0; rr < nrows; ++rr) {
+      if (cta_count > 0) copy_kv_rows(p, seq0, g + rr, out, out0, cta_first, cta_count);
+      if (crank == C - 1) copy_kv_rows(p, seq0, g + rr, out, out0, k, W);
+    }
   }
 }
 

@@ -110,3 +110,35 @@ def test_compress_layer_host_errors():
     b3, bp3 = B._i32([100, 100])
     # the workspace bound grows with the window (exponent rows of G*W)
     assert call(big, budgets_ptr=bp3, wsn=ckv.workspace_size(prob)) == B.CKV_ERR_UNSUPPORTED
+
+
+def test_selection_scope_validation():
+    lib = ckv.load()
+    prob, q, k = _problem()
+    prob.struct.selection = 2
+    assert lib.compresskv_workspace_size(prob.ref) == 0
+    assert lib.compresskv_output_layout(prob.ref, None, None, None) == B.CKV_ERR_INVALID_ARG
+    with pytest.raises(ckv.CompressKVError):
+        _problem(selection="heads")
+    # the per-layer scope keeps an extra row of summed scores in the workspace
+    g, _, _ = _problem()
+    lay, _, _ = _problem(selection="layer")
+    assert ckv.workspace_size(lay) >= ckv.workspace_size(g) + (268 + 8) * 4
+
+
+def test_layer_scope_host_errors():
+    lib = ckv.load()
+    prob, q, k = _problem(selection="layer")
+    vp = ctypes.c_void_p
+    n = ckv.workspace_size(prob)
+    bud, bp = B._i32([64, 64])
+    cu_out = (ctypes.c_int32 * 3)()
+    no_srh = np.zeros(8, np.uint8)  # no SRH head anywhere in the layer
+    rc = lib.compresskv_compress_layer(
+        prob.ref, vp(1 << 30), vp(1 << 30), vp(1 << 30), vp(no_srh.ctypes.data), bp,
+        vp(1 << 30), cu_out, vp(1 << 30), vp(1 << 30), None, None, vp(1 << 30), n, None)
+    assert rc == B.CKV_ERR_EMPTY_SRH_GROUP
+    # per-layer selection has no per-group pooled output in compresskv_select
+    rc = lib.compresskv_select(prob.ref, vp(1 << 30), bp, vp(1 << 30), cu_out, vp(1 << 30),
+                               vp(1 << 30), n, None)
+    assert rc == B.CKV_ERR_INVALID_ARG
