@@ -201,6 +201,25 @@ int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const voi
                               float* raw_scores, float* pooled_scores,
                               void* workspace, size_t workspace_bytes, void* stream);
 
+/* compresskv_compress_layer when the softmax denominators of the window
+ * queries are already known -- a prefill attention kernel has them as its
+ * log-sum-exp (CompressKV's latency study, Sec. 4.4, runs on a
+ * FlashAttention prefill; no separate normaliser pass is then needed).
+ * lse_win: device float, natural-log LSE of each window query's causal
+ *   softmax over keys j <= L_s - W + w with the problem's scale: element
+ *   (s, h, w) at lse_win + s*lse_batch_stride + h*lse_head_stride + w (4-byte
+ *   aligned; only SRH heads are read).  Scores are then exp(z - LSE) summed
+ *   in fp32 straight from the logits (no fp16 table), so their accuracy is
+ *   the given LSE's.  Other arguments as for compresskv_compress_layer
+ *   (pooled_scores must be NULL under CKV_SELECT_PER_LAYER). */
+int compresskv_compress_layer_lse(const ckv_problem* p, const void* q_win, const void* k,
+                                  const void* v, const float* lse_win, int64_t lse_batch_stride,
+                                  int64_t lse_head_stride, const uint8_t* srh_mask,
+                                  const int32_t* budgets, int32_t* indices, int32_t* cu_out,
+                                  void* k_out, void* v_out, float* raw_scores,
+                                  float* pooled_scores, void* workspace, size_t workspace_bytes,
+                                  void* stream);
+
 /* compresskv_compress_layer for callers that cannot allocate device memory
  * (the paper has no counterpart; this is a deployment convenience).  Some
  * hosts own every byte of device memory and give a plugin no allocator (an

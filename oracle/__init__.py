@@ -15,4 +15,5 @@ from .compresskv_oracle import (  # noqa: F401
     select_top,
     srh_heads,
     window_attention,
+    window_lse,
 )

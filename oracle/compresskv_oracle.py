@@ -202,6 +202,36 @@ def compress_unit(q_heads: np.ndarray, k_unit: np.ndarray, window: int, pool_wid
 
 
 # ---------------------------------------------------------------------------
+# Softmax denominators of the window queries (the log-sum-exp a prefill
+# attention kernel returns; the library's given-LSE entry point takes it)
+# ---------------------------------------------------------------------------
+def window_lse(q_win, k, cu_seqlens, window: int, scale: float | None = None) -> np.ndarray:
+    """``[B, H_q, W]`` natural-log ``log sum_{j <= p} exp(z_j)`` of every
+    window query (``p = L_s - W + w``, ``z_j = scale * <q, k_j>``, keys of
+    the head's KV group); 0 where the sequence has no such position."""
+    q_win = np.asarray(q_win, np.float64)
+    k = np.asarray(k, np.float64)
+    cu = [int(x) for x in cu_seqlens]
+    B, H_q, W, d = q_win.shape
+    G = H_q // k.shape[1]
+    if scale is None:
+        scale = default_scale(d)
+    out = np.zeros((B, H_q, W), dtype=np.float64)
+    for s in range(B):
+        L = cu[s + 1] - cu[s]
+        for h in range(H_q):
+            ku = k[cu[s]:cu[s + 1], h // G]
+            for w in range(W):
+                p = L - W + w
+                if p < 0:
+                    continue
+                z = scale * (ku[:p + 1] @ q_win[s, h, w])
+                m = z.max()
+                out[s, h, w] = m + math.log(np.exp(z - m).sum())
+    return out
+
+
+# ---------------------------------------------------------------------------
 # One layer over a packed (cu_seqlens) batch, in the library's output layout
 # ---------------------------------------------------------------------------
 @dataclass

@@ -13,6 +13,7 @@ from .compresskv import (  # noqa: F401
     Trace,
     allocate_layer_budgets,
     compress_layer,
+    compress_layer_lse,
     compress_layer_noalloc,
     gather,
     load,

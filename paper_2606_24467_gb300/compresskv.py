@@ -43,6 +43,7 @@ EXPORTED = (
     "compresskv_gather",
     "compresskv_compress_layer",
     "compresskv_compress_layer_noalloc",
+    "compresskv_compress_layer_lse",
     "compresskv_read_device_status",
     "compresskv_allocate_layer_budgets",
     "compresskv_status_string",
@@ -101,6 +102,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
                                                  vp, vp, vp, c_size_t, vp]),
         "compresskv_compress_layer_noalloc": (c_int32, [pp, vp, vp, vp, vp, i32p, vp, i32p, vp,
                                                          vp, vp, vp, vp, vp]),
+        "compresskv_compress_layer_lse": (c_int32, [pp, vp, vp, vp, vp, c_int64, c_int64, vp, i32p,
+                                                     vp, i32p, vp, vp, vp, vp, vp, c_size_t, vp]),
         "compresskv_read_device_status": (c_int32, [vp, vp, i32p]),
         "compresskv_allocate_layer_budgets": (c_int32, [POINTER(ctypes.c_double), c_int32,
                                                         c_int64, c_int32, c_int32, i32p]),
@@ -309,6 +312,23 @@ def allocate_layer_budgets(layer_errors, total_budget: int, min_budget: int = 32
         int(min_budget), int(max_budget), out.ctypes.data_as(POINTER(c_int32))),
         "compresskv_allocate_layer_budgets")
     return out
+
+
+def compress_layer_lse(problem: Problem, q_win, k, v, lse_win, srh_mask, budgets, indices, k_out,
+                       v_out, ws, raw=None, pooled=None, stream=None) -> np.ndarray:
+    """compress_layer with the window queries' log-sum-exp given:
+    ``lse_win`` is a float32 ``[B, H_q, W]`` tensor (window rows contiguous)."""
+    if lse_win.dtype != torch.float32 or lse_win.stride(2) != 1:
+        raise CompressKVError(CKV_ERR_INVALID_ARG, "lse_win must be float32 with contiguous rows")
+    m, mp = _mask(srh_mask)
+    b, bp = _i32(budgets)
+    cu_out = np.zeros(problem.batch + 1, np.int32)
+    _check(load().compresskv_compress_layer_lse(
+        problem.ref, _ptr(q_win), _ptr(k), _ptr(v), _ptr(lse_win), lse_win.stride(0),
+        lse_win.stride(1), mp, bp, _ptr(indices), cu_out.ctypes.data_as(POINTER(c_int32)),
+        _ptr(k_out), _ptr(v_out), _ptr(raw), _ptr(pooled), _ptr(ws), ws.numel(), _stream(stream)),
+        "compresskv_compress_layer_lse")
+    return cu_out
 
 
 def read_device_status(ws, stream=None) -> int:

@@ -195,10 +195,11 @@ struct Workspace {
   uint16_t* expo = nullptr;  // one set's exponent table
   float* refs = nullptr;     // one set's reference table
   float* shared = nullptr;   // per-layer selection: summed scores [sum_s n_s]
+  float* raw = nullptr;      // raw scores, score layout (given-LSE calls)
 };
 
 struct WorkspaceLayout {
-  size_t pooled, expo, refs, shared, total;
+  size_t pooled, expo, refs, shared, raw, total;
 };
 
 WorkspaceLayout workspace_layout(const Info& I) {
@@ -214,7 +215,8 @@ WorkspaceLayout workspace_layout(const Info& I) {
   W.expo = W.pooled + align256(static_cast<size_t>(I.Hkv) * I.p_total * sizeof(float));
   W.refs = W.expo + align256(static_cast<size_t>(e) * sizeof(uint16_t));
   W.shared = W.refs + align256(static_cast<size_t>(r) * sizeof(float));
-  W.total = W.shared + (I.layer ? align256(static_cast<size_t>(I.p_total) * sizeof(float)) : 0);
+  W.raw = W.shared + (I.layer ? align256(static_cast<size_t>(I.p_total) * sizeof(float)) : 0);
+  W.total = W.raw + align256(static_cast<size_t>(I.Hkv) * I.p_total * sizeof(float));
   return W;
 }
 
@@ -230,6 +232,7 @@ int carve(const Info& I, void* ws, size_t bytes, Workspace& out) {
   out.expo = reinterpret_cast<uint16_t*>(b + W.expo);
   out.refs = reinterpret_cast<float*>(b + W.refs);
   out.shared = reinterpret_cast<float*>(b + W.shared);
+  out.raw = reinterpret_cast<float*>(b + W.raw);
   return CKV_OK;
 }
 
@@ -332,10 +335,17 @@ int make_k_map(const Info& I, const ckv_problem* p, const void* k, CUtensorMap* 
 // Scores every unit: per set, the scoring kernel (one pass over K) and the
 // combine kernel, which leaves pooled scores (and raw scores when `raw` is
 // given) in score layout.
+// Window-query log-sum-exps supplied by the caller (given-LSE mode).
+struct LseInput {
+  const float* lse = nullptr;
+  long long batch_stride = 0, head_stride = 0;
+};
+
 int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void* k,
               const uint8_t* mask, float* raw, float* pooled, const Workspace& ws,
-              cudaStream_t stream) {
-  if (!q_win || !k || !pooled) return CKV_ERR_INVALID_ARG;
+              cudaStream_t stream, const LseInput& lse = LseInput{}) {
+  const bool given_lse = lse.lse != nullptr;
+  if (!q_win || !k || (given_lse ? !raw : !pooled)) return CKV_ERR_INVALID_ARG;
   if (!aligned16(q_win) || !aligned16(k)) return CKV_ERR_INVALID_ARG;
   SrhLists S;
   int rc = srh_lists(I, mask, S);
@@ -362,6 +372,12 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
   P.num_kv_heads = I.Hkv;
   P.is_bf16 = I.bf16 ? 1 : 0;
   P.use_evict_hint = 1;
+  P.lse = lse.lse;
+  P.lse_bs = lse.batch_stride;
+  P.lse_hs = lse.head_stride;
+  P.raw_out = raw;
+  P.p_total = static_cast<int>(I.p_total);
+  for (int s = 0; s <= I.B; ++s) P.cu_prefix[s] = I.cu_prefix[s];
   C.partials = ws.partials;
   C.expo = ws.expo;
   C.refs = ws.refs;
@@ -393,7 +409,8 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
   for (int g = 0; g < I.Hkv; ++g) {
     if (S.rows[g] > 0) continue;
     const size_t row = static_cast<size_t>(I.p_total) * sizeof(float);
-    if (cudaMemsetAsync(pooled + static_cast<size_t>(g) * I.p_total, 0, row, stream) != cudaSuccess)
+    if (pooled &&
+        cudaMemsetAsync(pooled + static_cast<size_t>(g) * I.p_total, 0, row, stream) != cudaSuccess)
       return CKV_ERR_CUDA;
     if (raw && cudaMemsetAsync(raw + static_cast<size_t>(g) * I.p_total, 0, row, stream) !=
                    cudaSuccess)
@@ -483,6 +500,11 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
            score_smem_bytes(P.q_half_bytes, P.stages) > static_cast<size_t>(F->smem_optin))
       --P.stages;
     const size_t smem = score_smem_bytes(P.q_half_bytes, P.stages);
+    if (given_lse) {  // raw scores come straight out of the scoring kernel
+      rc = traced(tr, CKV_KERNEL_SCORE, [&] { return launch_score_lse(P, n_items, smem, stream); });
+      if (rc != CKV_OK) return rc;
+      continue;
+    }
     rc = traced(tr, CKV_KERNEL_SCORE, [&] { return launch_score(P, n_items, smem, stream); });
     if (rc != CKV_OK) return rc;
     rc = traced(tr, CKV_KERNEL_COMBINE,
@@ -693,6 +715,37 @@ int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const voi
   std::copy(co.begin(), co.end(), cu_out);
   if ((rc = run_score(p, I, q_win, k, srh_mask, raw_scores, pooled, ws, st)) != CKV_OK) return rc;
   return run_select(p, I, nullptr, pooled, co, indices, nullptr, ws, st, k, v, k_out, v_out);
+}
+
+int compresskv_compress_layer_lse(const ckv_problem* p, const void* q_win, const void* k,
+                                  const void* v, const float* lse_win, int64_t lse_batch_stride,
+                                  int64_t lse_head_stride, const uint8_t* srh_mask,
+                                  const int32_t* budgets, int32_t* indices, int32_t* cu_out,
+                                  void* k_out, void* v_out, float* raw_scores,
+                                  float* pooled_scores, void* workspace, size_t workspace_bytes,
+                                  void* stream) {
+  Info I;
+  int rc = validate(p, I);
+  if (rc != CKV_OK) return rc;
+  if (!lse_win || lse_batch_stride < 0 || lse_head_stride < 0) return CKV_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(lse_win) & 3u) return CKV_ERR_INVALID_ARG;
+  std::vector<int> co;
+  if ((rc = output_layout(I, budgets, co)) != CKV_OK) return rc;
+  if (!cu_out) return CKV_ERR_INVALID_ARG;
+  if (I.layer && pooled_scores) return CKV_ERR_INVALID_ARG;
+  Workspace ws;
+  if ((rc = carve(I, workspace, workspace_bytes, ws)) != CKV_OK) return rc;
+  SrhLists S;
+  if ((rc = srh_lists(I, srh_mask, S)) != CKV_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  float* raw = raw_scores ? raw_scores : ws.raw;
+  std::copy(co.begin(), co.end(), cu_out);
+  LseInput lse;
+  lse.lse = lse_win;
+  lse.batch_stride = lse_batch_stride;
+  lse.head_stride = lse_head_stride;
+  if ((rc = run_score(p, I, q_win, k, srh_mask, raw, nullptr, ws, st, lse)) != CKV_OK) return rc;
+  return run_select(p, I, raw, nullptr, co, indices, pooled_scores, ws, st, k, v, k_out, v_out);
 }
 
 int compresskv_read_device_status(const void* workspace, void* stream, int32_t* status) {

@@ -43,6 +43,11 @@ struct ScoreParams {
   float2* partials;            // [n_items][kMaxQRows]: (M, S) with sum 2^(z*c) = S * 2^M
   uint16_t* expo;              // fp16 2^(z*c - R) per prefix key and query row (Nr per key)
   float* refs;                 // per (tile, quarter, query row): the R used for expo
+  const float* lse;            // given-LSE mode: natural-log LSE per (sequence, head, window row)
+  float* raw_out;              // given-LSE mode: raw scores, score layout
+  long long lse_bs, lse_hs;    // LSE strides (elements); window rows are contiguous
+  int p_total;
+  int cu_prefix[kMaxBatch + 1];
   int* status;                 // device status word
   long long q_bs, q_hs, q_ws;  // window-query strides, elements
   float c;                     // scale * log2(e)
@@ -117,6 +122,7 @@ struct GatherParams {
 
 // Host-side launchers (defined next to each kernel).
 cudaError_t launch_score(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s);
+cudaError_t launch_score_lse(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s);
 cudaError_t launch_combine(const CombineParams& p, int n_items, size_t smem, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, int n_units, size_t smem, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, long long rows, cudaStream_t s);

@@ -39,6 +39,11 @@
 //               transpose-reduction.
 // Tokens sit on the MMA's M side so every epilogue lane holds real work for
 // any N.
+//
+// With the window queries' log-sum-exp given (kLse: the softmax denominators
+// a prefill attention kernel already has), no table is needed: every lane
+// sums 2^(z*c - LSE_q*log2(e)) over its row -- the normalised attention of all
+// query rows on its key -- and writes the prefix key's raw score directly.
 #include <cuda_runtime.h>
 
 #include <cfloat>
@@ -68,6 +73,7 @@ __device__ __forceinline__ void wait_plain(uint32_t bar, uint32_t parity, uint64
   mbar_wait_bounded(bar, parity, &never, nullptr, timeout_ns);
 }
 
+template <bool kLse>
 __global__ void __launch_bounds__(kScoreThreads, 1)
     score_kernel(const __grid_constant__ ScoreParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -179,7 +185,19 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     }
     fence_proxy_async_smem();
     for (int q = st_tid; q < kMaxQRows; q += kStagedThreads) sWpos[q] = q < N ? q % W : 0;
-    {
+    if constexpr (kLse) {
+      // log2 of every query row's softmax denominator (first rows of sRef)
+      for (int q = st_tid; q < kMaxQRows; q += kStagedThreads) {
+        float l2 = 0.f;
+        if (q < N) {
+          const int head = p.srh_heads[h0 + q / W];
+          const int w = q - (q / W) * W;
+          l2 = p.lse[static_cast<long long>(s) * p.lse_bs + static_cast<long long>(head) * p.lse_hs +
+                     w] * 1.4426950408889634f;
+        }
+        sRef[q] = l2;
+      }
+    } else {
       const int ew = warp - kFirstEpiWarp;
       if (ew >= 0) {
         for (int q = lane; q < kMaxQRows; q += 32) {
@@ -227,6 +245,65 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         }
       }
       __syncwarp();  // reconverge before the CTA-wide (aligned) barrier below
+    } else if constexpr (kLse) {
+      // -------------------------------------------------------- epilogue (given LSE)
+      const int ew = warp - kFirstEpiWarp;  // 0..15
+      const int wg = ew >> 2;
+      const int qd = warp & 3;
+      const float c = p.c;
+      const float* lse2 = sRef;
+      const int nwg = kWG < nbuf ? kWG : nbuf;
+      float* raw_row = p.raw_out + static_cast<long long>(g) * p.p_total + p.cu_prefix[s];
+      // the raw-score buffer may still be read by an earlier kernel of the stream
+      pdl_wait();
+      for (int i = wg; wg < nwg && i < ntiles; i += nwg) {
+        const int b = i % nbuf;
+        const uint32_t use = static_cast<uint32_t>(i / nbuf) & 1u;
+        const bool got = mbar_wait_bounded(tfull0 + 8 * b, use, abort_flag, p.status);
+        if (!__all_sync(0xffffffffu, got)) break;
+        tc_fence_after();
+        const int tile = t0 + i;
+        const int tok = tile * kTileTokens + qd * 32 + lane;
+        const uint32_t taddr =
+            tbase + (static_cast<uint32_t>(qd * 32) << 16) + static_cast<uint32_t>(b * tstride);
+        const bool edge = (tile + 1) * kTileTokens > n;
+        const int vis = n - tok;
+        const bool key = tok < L;
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int c0 = 0; c0 < N; c0 += 32) {
+          uint32_t r[32];
+          tmem_load32_async(taddr + c0, r);
+          tmem_wait_ld(r);
+          const int lim = min(32, N - c0);
+          if (edge || lim < 32) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 4) {
+              const int4 wq = *reinterpret_cast<const int4*>(sWpos + c0 + j);
+              const float4 lq = *reinterpret_cast<const float4*>(lse2 + c0 + j);
+              const int wv[4] = {wq.x, wq.y, wq.z, wq.w};
+              const float lv[4] = {lq.x, lq.y, lq.z, lq.w};
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                const bool ok = (j + u) < lim && (!edge || (key && wv[u] >= -vis));
+                acc[u] += ok ? ex2_approx(fmaf(__uint_as_float(r[j + u]), c, -lv[u])) : 0.f;
+              }
+            }
+          } else {
+#pragma unroll
+            for (int j = 0; j < 32; j += 4) {
+              const float4 lq = *reinterpret_cast<const float4*>(lse2 + c0 + j);
+              acc[0] += ex2_approx(fmaf(__uint_as_float(r[j + 0]), c, -lq.x));
+              acc[1] += ex2_approx(fmaf(__uint_as_float(r[j + 1]), c, -lq.y));
+              acc[2] += ex2_approx(fmaf(__uint_as_float(r[j + 2]), c, -lq.z));
+              acc[3] += ex2_approx(fmaf(__uint_as_float(r[j + 3]), c, -lq.w));
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(tempty0 + 8 * b);
+        if (tok < n) raw_row[tok] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+      }
     } else {
       // -------------------------------------------------------- epilogue
       const int ew = warp - kFirstEpiWarp;  // 0..15
@@ -416,11 +493,18 @@ size_t score_smem_bytes(int q_half_bytes, int stages) {
 }
 
 cudaError_t score_set_smem_limit(size_t bytes) {
-  return cudaFuncSetAttribute(score_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(score_kernel<false>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(bytes));
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(score_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               static_cast<int>(bytes));
 }
 
-cudaError_t launch_score(const ScoreParams& p, int n_items, size_t smem, cudaStream_t stream) {
+namespace {
+
+template <bool kLse>
+cudaError_t launch(const ScoreParams& p, int n_items, size_t smem, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(n_items));
   cfg.blockDim = dim3(kScoreThreads);
@@ -431,7 +515,17 @@ cudaError_t launch_score(const ScoreParams& p, int n_items, size_t smem, cudaStr
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, score_kernel, p);
+  return cudaLaunchKernelEx(&cfg, score_kernel<kLse>, p);
+}
+
+}  // namespace
+
+cudaError_t launch_score(const ScoreParams& p, int n_items, size_t smem, cudaStream_t stream) {
+  return launch<false>(p, n_items, smem, stream);
+}
+
+cudaError_t launch_score_lse(const ScoreParams& p, int n_items, size_t smem, cudaStream_t stream) {
+  return launch<true>(p, n_items, smem, stream);
 }
 
 }  // namespace ckv
