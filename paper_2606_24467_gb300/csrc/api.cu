@@ -436,7 +436,15 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
       active += cnt[u];
     }
     if (active == 0) continue;
-    const int target = std::min(kMaxItems, std::max(active, F->sms));
+    // Two CTAs per SM (8 epilogue warps each, two K rings in flight) when
+    // their shared memory fits; else one CTA per SM with 16 epilogue warps.
+    int max_rows = 16;
+    for (int u = 0; u < nu; ++u)
+      if (cnt[u] > 0) max_rows = std::max(max_rows, (S.rows[units[u0 + u].g] + 15) & ~15);
+    const int q_half = ((max_rows * 128) + 1023) & ~1023;
+    const int per_sm =
+        score_smem_bytes(q_half, 2, 8) <= static_cast<size_t>(F->smem_optin) / 2 - 1024 ? 2 : 1;
+    const int target = std::min(kMaxItems, std::max(active, per_sm * F->sms));
     for (int extra = target - active; extra > 0; --extra) {
       int best = -1;
       for (int u = 0; u < nu; ++u) {
@@ -461,7 +469,6 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
     if (csmem > F->combine_smem_max) return CKV_ERR_UNSUPPORTED;
 
     int n_items = 0, n_comb = 0;
-    int max_rows = 16;
     uint32_t eoff = 0, roff = 0;
     for (int u = 0; u < nu; ++u) {
       const Unit& U = units[u0 + u];
@@ -490,16 +497,17 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
       n_items += c_u;
       eoff += static_cast<uint32_t>(I.n[U.s]) * static_cast<uint32_t>(nr);
       roff += static_cast<uint32_t>(U.tiles * kQuarters * nr);
-      max_rows = std::max(max_rows, (S.rows[U.g] + 15) & ~15);
     }
     P.n_items = n_items;
     C.n_items = n_comb;
-    P.q_half_bytes = ((max_rows * 128) + 1023) & ~1023;
+    P.q_half_bytes = q_half;
     P.stages = kStages;
-    while (P.stages > 2 &&
-           score_smem_bytes(P.q_half_bytes, P.stages) > static_cast<size_t>(F->smem_optin))
+    P.epi_warps = per_sm == 2 ? 8 : 16;
+    const size_t smem_cap = per_sm == 2 ? static_cast<size_t>(F->smem_optin) / 2 - 1024
+                                        : static_cast<size_t>(F->smem_optin);
+    while (P.stages > 2 && score_smem_bytes(P.q_half_bytes, P.stages, P.epi_warps) > smem_cap)
       --P.stages;
-    const size_t smem = score_smem_bytes(P.q_half_bytes, P.stages);
+    const size_t smem = score_smem_bytes(P.q_half_bytes, P.stages, P.epi_warps);
     if (given_lse) {  // raw scores come straight out of the scoring kernel
       rc = traced(tr, CKV_KERNEL_SCORE, [&] { return launch_score_lse(P, n_items, smem, stream); });
       if (rc != CKV_OK) return rc;

@@ -54,6 +54,7 @@ struct ScoreParams {
   int window, num_kv_heads, n_items, is_bf16, use_evict_hint;
   int q_half_bytes;            // bytes of one 64-column half of the Q rows in shared memory
   int stages;                  // K tiles in the shared-memory ring (2..kStages)
+  int epi_warps;               // 8 (two CTAs per SM) or 16 (one CTA per SM)
   int cu_seqlens[kMaxBatch + 1];
   uint16_t srh_off[kMaxKvHeads + 1];   // SRH heads of group g: srh_heads[srh_off[g] .. srh_off[g+1])
   uint8_t srh_heads[kMaxQHeads];
@@ -126,7 +127,9 @@ cudaError_t launch_score_lse(const ScoreParams& p, int n_items, size_t smem, cud
 cudaError_t launch_combine(const CombineParams& p, int n_items, size_t smem, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, int n_units, size_t smem, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, long long rows, cudaStream_t s);
-size_t score_smem_bytes(int q_half_bytes, int stages);
+size_t score_smem_bytes(int q_half_bytes, int stages, int epi_warps);
+// Sets every scoring kernel's shared-memory limit: `bytes` for one CTA per
+// SM, half of it for the two-CTA form.
 cudaError_t score_set_smem_limit(size_t bytes);
 // Dynamic shared memory of a combine CTA that covers `quarters` 32-key
 // quarters with exponent rows of `nr` columns and pooling width P.

@@ -30,8 +30,10 @@
 //               K_tile . Q_S^T  (tcgen05.mma kind::f16, M=128, N rounded to 16,
 //               K = d = 128), fp32 accumulators in TMEM, 2 or 4 buffers, each
 //               owned by one epilogue warpgroup;
-//   warps 2-17  four epilogue warpgroups (tiles i % 4; with 2 buffers only
-//               the first two work); thread = token (TMEM lane): it reads its
+//   warps 2..   two or four epilogue warpgroups (tiles i % #groups; with 2
+//               TMEM buffers only the first two work) -- two warpgroups per CTA
+//               and two CTAs per SM when their shared memory fits, else four
+//               in one CTA per SM; thread = token (TMEM lane): it reads its
 //               row of logits from TMEM 32 columns at a time, keeps the
 //               warp's running references, writes its exponent row with
 //               32-byte stores that ask L2 to keep the table, and adds the
@@ -56,13 +58,18 @@ namespace {
 
 constexpr float kShift = 7.0f;   // R sits this far below the warp's largest logit (log2 units)
 constexpr float kRaise = 15.0f;  // exponents stay <= 2^kRaise
-constexpr int kNumEpiWarps = 16;  // 4 epilogue warpgroups
-constexpr int kWG = kNumEpiWarps / 4;
-constexpr int kScoreThreads = 64 + 32 * kNumEpiWarps;
-constexpr int kStagedThreads = kScoreThreads - 32;  // warps 1.. stage the Q rows
-// misc region: barriers (256 B) | running references [16][256] f32 |
-// sums [16][256] f32 | window position of each query row [256] i32
-constexpr int kMiscBytes = 256 + 2 * kNumEpiWarps * kMaxQRows * 4 + kMaxQRows * 4;
+// Epilogue width: 8 warps (two CTAs per SM, when their shared memory fits)
+// or 16 warps (one CTA per SM).
+template <int kEpi>
+struct Shape {
+  static constexpr int kWG = kEpi / 4;                    // epilogue warpgroups
+  static constexpr int kThreads = 64 + 32 * kEpi;
+  static constexpr int kStagedThreads = kThreads - 32;    // warps 1.. stage the Q rows
+  static constexpr int kCtasPerSm = kEpi == 8 ? 2 : 1;
+  // misc region: barriers (256 B) | running references [kEpi][256] f32 |
+  // sums [kEpi][256] f32 | window position of each query row [256] i32
+  static constexpr int kMiscBytes = 256 + 2 * kEpi * kMaxQRows * 4 + kMaxQRows * 4;
+};
 constexpr float kNegInf = -INFINITY;
 constexpr int kBarStaged = 2;  // named barrier: warps 1.. after staging Q
 constexpr int kBarEpi = 1;     // named barrier: the epilogue warps
@@ -73,9 +80,12 @@ __device__ __forceinline__ void wait_plain(uint32_t bar, uint32_t parity, uint64
   mbar_wait_bounded(bar, parity, &never, nullptr, timeout_ns);
 }
 
-template <bool kLse>
-__global__ void __launch_bounds__(kScoreThreads, 1)
+template <bool kLse, int kEpi>
+__global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm)
     score_kernel(const __grid_constant__ ScoreParams p) {
+  constexpr int kNumEpiWarps = kEpi;
+  constexpr int kWG = Shape<kEpi>::kWG;
+  constexpr int kStagedThreads = Shape<kEpi>::kStagedThreads;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -88,7 +98,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(sMisc + 192);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(sMisc + 196);
   float* sRef = reinterpret_cast<float*>(sMisc + 256);                  // [16][kMaxQRows]
-  float* sAcc = sRef + kNumEpiWarps * kMaxQRows;                         // [16][kMaxQRows]
+  float* sAcc = sRef + kNumEpiWarps * kMaxQRows;                         // [kEpi][kMaxQRows]
   int* sWpos = reinterpret_cast<int*>(sAcc + kNumEpiWarps * kMaxQRows);  // [kMaxQRows]
 
   const uint32_t full0 = smem_u32(bars);
@@ -487,27 +497,36 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
 
 }  // namespace
 
-size_t score_smem_bytes(int q_half_bytes, int stages) {
+size_t score_smem_bytes(int q_half_bytes, int stages, int epi_warps) {
+  const size_t misc = epi_warps == 8 ? Shape<8>::kMiscBytes : Shape<16>::kMiscBytes;
   return 1024 + static_cast<size_t>(stages) * kTileBytes + 2 * static_cast<size_t>(q_half_bytes) +
-         kMiscBytes;
+         misc;
 }
 
 cudaError_t score_set_smem_limit(size_t bytes) {
-  cudaError_t e = cudaFuncSetAttribute(score_kernel<false>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(bytes));
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(score_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(bytes));
+  const int b = static_cast<int>(bytes);
+  const int half = static_cast<int>(bytes / 2 - 1024);  // two CTAs per SM
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(score_kernel<false, 16>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, b)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(score_kernel<true, 16>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, b)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(score_kernel<false, 8>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, half)) != cudaSuccess)
+    return e;
+  return cudaFuncSetAttribute(score_kernel<true, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              half);
 }
 
 namespace {
 
-template <bool kLse>
+template <bool kLse, int kEpi>
 cudaError_t launch(const ScoreParams& p, int n_items, size_t smem, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(n_items));
-  cfg.blockDim = dim3(kScoreThreads);
+  cfg.blockDim = dim3(Shape<kEpi>::kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
@@ -515,17 +534,19 @@ cudaError_t launch(const ScoreParams& p, int n_items, size_t smem, cudaStream_t 
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, score_kernel<kLse>, p);
+  return cudaLaunchKernelEx(&cfg, score_kernel<kLse, kEpi>, p);
 }
 
 }  // namespace
 
 cudaError_t launch_score(const ScoreParams& p, int n_items, size_t smem, cudaStream_t stream) {
-  return launch<false>(p, n_items, smem, stream);
+  return p.epi_warps == 8 ? launch<false, 8>(p, n_items, smem, stream)
+                          : launch<false, 16>(p, n_items, smem, stream);
 }
 
 cudaError_t launch_score_lse(const ScoreParams& p, int n_items, size_t smem, cudaStream_t stream) {
-  return launch<true>(p, n_items, smem, stream);
+  return p.epi_warps == 8 ? launch<true, 8>(p, n_items, smem, stream)
+                          : launch<true, 16>(p, n_items, smem, stream);
 }
 
 }  // namespace ckv
