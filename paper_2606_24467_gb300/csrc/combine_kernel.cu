@@ -22,7 +22,9 @@
 // 8-column chunk of a row (tid % cpr, where cpr = Nr / 8 divides 32); the
 // cpr threads of a row are adjacent lanes and add their dot products by
 // shuffles.  Raw scores of the chunk and halo stay in shared memory for the
-// pooling.
+// pooling.  The table lines only this chunk reads are then discarded from
+// L2 (`discard.global.L2`): the table is dead, so its dirty lines need not be
+// written back to DRAM.
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
@@ -175,6 +177,20 @@ __global__ void __launch_bounds__(kCombThreads)
     }
   }
   __syncthreads();
+
+  // discard the table lines no other chunk reads (rows inside [a + h, b - h)):
+  // every load of them has completed, and they need no write-back to DRAM
+  {
+    const long long row_bytes = static_cast<long long>(Nr) * 2;
+    const long long base_b = static_cast<long long>(it.eoff) * 2;
+    const long long lo_b = ((base_b + static_cast<long long>(a + h + 1) * row_bytes + 127) / 128) * 128;
+    const long long hi_b = ((base_b + static_cast<long long>(b - h - 1) * row_bytes) / 128) * 128;
+    for (long long x = lo_b + static_cast<long long>(tid) * 128; x + 128 <= hi_b;
+         x += static_cast<long long>(kCombThreads) * 128) {
+      const char* line = reinterpret_cast<const char*>(p.expo) + x;
+      asm volatile("discard.global.L2 [%0], 128;" ::"l"(line) : "memory");
+    }
+  }
 
   // 4. pooling (and the raw scores, when asked for)
   const long long soff = static_cast<long long>(g) * p.p_total + p.cu_prefix[s];
