@@ -220,6 +220,29 @@ int compresskv_compress_layer_lse(const ckv_problem* p, const void* q_win, const
                                   float* pooled_scores, void* workspace, size_t workspace_bytes,
                                   void* stream);
 
+/* compresskv_compress_layer with a budget per (sequence, KV group) -- the
+ * head-level allocation CompressKV's token selection combines with (Sec.
+ * 4.6, HeadKV / AdaKV style budgets, computed elsewhere).  Per-group
+ * selection only (CKV_SELECT_PER_LAYER is CKV_ERR_INVALID_ARG).
+ * group_budgets: host int32 [batch][num_kv_heads], each >= W (else
+ *   CKV_ERR_BUDGET); unit (s, g) keeps min(budget, L_s) tokens.
+ * Outputs are packed group-major: group 0's sequences, then group 1's, ...
+ * cu_out: host int32 [num_kv_heads][batch+1], written: cu_out[g][s] is the
+ *   first output row of (s, g) and cu_out[g][batch] the end of group g.
+ * indices: device int32 [rows] (positions within the sequence, ascending
+ *   per unit, window last); k_out / v_out: [rows][head_dim] in the input
+ *   dtype, rows = cu_out[num_kv_heads-1][batch].
+ * At most 2048 (sequence, group) pairs (CKV_ERR_UNSUPPORTED).  Other
+ * arguments as for compresskv_compress_layer. */
+int compresskv_compress_layer_head_budgets(const ckv_problem* p, const void* q_win,
+                                           const void* k, const void* v,
+                                           const uint8_t* srh_mask,
+                                           const int32_t* group_budgets, int32_t* indices,
+                                           int32_t* cu_out, void* k_out, void* v_out,
+                                           float* raw_scores, float* pooled_scores,
+                                           void* workspace, size_t workspace_bytes,
+                                           void* stream);
+
 /* compresskv_compress_layer for callers that cannot allocate device memory
  * (the paper has no counterpart; this is a deployment convenience).  Some
  * hosts own every byte of device memory and give a plugin no allocator (an

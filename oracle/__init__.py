@@ -6,6 +6,7 @@ and reference legs import this package.
 from .compresskv_oracle import (  # noqa: F401
     OracleError,
     compress_layer,
+    compress_layer_head_budgets,
     compress_unit,
     default_scale,
     kept_count,

@@ -357,3 +357,59 @@ def compress_layer(q_win, k, v, cu_seqlens, srh_mask, budgets, window: int,
             k_out[cu_out[s]:cu_out[s + 1], g] = k[rows, g]
             v_out[cu_out[s]:cu_out[s + 1], g] = v[rows, g]
     return LayerResult(units, raw, pooled, indices, cu_out, cu_prefix, k_out, v_out)
+
+
+# ---------------------------------------------------------------------------
+# Head-level budgets (Sec. 4.6: the token selection combined with a budget
+# per head group from a head-level allocator), outputs packed group-major
+# ---------------------------------------------------------------------------
+@dataclass
+class HeadBudgetResult:
+    units: dict              # (s, g) -> UnitResult, each with its own budget
+    cu_out: np.ndarray       # [H_kv, B+1] first output row of (s, g); end of group g
+    indices: np.ndarray      # [rows] int64
+    k_out: np.ndarray        # [rows, d]
+    v_out: np.ndarray
+
+
+def compress_layer_head_budgets(q_win, k, v, cu_seqlens, srh_mask, group_budgets, window: int,
+                                pool_width: int, scale: float | None = None) -> HeadBudgetResult:
+    """Per (sequence, group) selection with budget ``group_budgets[s][g]``;
+    group g's compressed sequences follow each other, then group g+1's."""
+    q_win = np.asarray(q_win)
+    k = np.asarray(k)
+    v = np.asarray(v)
+    cu = [int(x) for x in cu_seqlens]
+    B = len(cu) - 1
+    H_q, H_kv = q_win.shape[1], k.shape[1]
+    G = H_q // H_kv
+    if scale is None:
+        scale = default_scale(k.shape[2])
+    gb = np.asarray(group_budgets).reshape(B, H_kv)
+    q64, k64 = q_win.astype(np.float64), k.astype(np.float64)
+    units, idx_parts, k_parts, v_parts = {}, [], [], []
+    cu_out = np.zeros((H_kv, B + 1), dtype=np.int64)
+    row = 0
+    for g in range(H_kv):
+        heads = srh_heads(srh_mask, g, G)
+        for s in range(B):
+            cu_out[g, s] = row
+            L = cu[s + 1] - cu[s]
+            if not heads and L > window:
+                raise OracleError(f"KV group {g} has no SRH head")
+            qh = q64[s, heads] if heads else np.zeros((0, window, k.shape[2]))
+            res = compress_unit(qh, k64[cu[s]:cu[s + 1], g], window, pool_width, int(gb[s, g]),
+                                scale)
+            res.heads = heads
+            units[(s, g)] = res
+            idx_parts.append(res.indices)
+            k_parts.append(k[cu[s] + res.indices, g])
+            v_parts.append(v[cu[s] + res.indices, g])
+            row += len(res.indices)
+        cu_out[g, B] = row
+    d = k.shape[2]
+    cat = lambda parts, dt: (np.concatenate(parts) if parts else np.zeros((0, d), dt))
+    return HeadBudgetResult(units, cu_out,
+                            np.concatenate(idx_parts) if idx_parts else np.zeros(0, np.int64),
+                            cat(k_parts, k.dtype), cat(v_parts, v.dtype))
+

@@ -13,9 +13,11 @@ from .compresskv import (  # noqa: F401
     Trace,
     allocate_layer_budgets,
     compress_layer,
+    compress_layer_head_budgets,
     compress_layer_lse,
     compress_layer_noalloc,
     gather,
+    head_budget_layout,
     load,
     output_layout,
     read_device_status,

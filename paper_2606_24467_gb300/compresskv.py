@@ -44,6 +44,7 @@ EXPORTED = (
     "compresskv_compress_layer",
     "compresskv_compress_layer_noalloc",
     "compresskv_compress_layer_lse",
+    "compresskv_compress_layer_head_budgets",
     "compresskv_read_device_status",
     "compresskv_allocate_layer_budgets",
     "compresskv_status_string",
@@ -104,6 +105,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
                                                          vp, vp, vp, vp, vp]),
         "compresskv_compress_layer_lse": (c_int32, [pp, vp, vp, vp, vp, c_int64, c_int64, vp, i32p,
                                                      vp, i32p, vp, vp, vp, vp, vp, c_size_t, vp]),
+        "compresskv_compress_layer_head_budgets": (c_int32, [pp, vp, vp, vp, vp, i32p, vp, i32p,
+                                                              vp, vp, vp, vp, vp, c_size_t, vp]),
         "compresskv_read_device_status": (c_int32, [vp, vp, i32p]),
         "compresskv_allocate_layer_budgets": (c_int32, [POINTER(ctypes.c_double), c_int32,
                                                         c_int64, c_int32, c_int32, i32p]),
@@ -328,6 +331,39 @@ def compress_layer_lse(problem: Problem, q_win, k, v, lse_win, srh_mask, budgets
         lse_win.stride(1), mp, bp, _ptr(indices), cu_out.ctypes.data_as(POINTER(c_int32)),
         _ptr(k_out), _ptr(v_out), _ptr(raw), _ptr(pooled), _ptr(ws), ws.numel(), _stream(stream)),
         "compresskv_compress_layer_lse")
+    return cu_out
+
+
+def head_budget_layout(problem: Problem, group_budgets) -> tuple[np.ndarray, int]:
+    """Host-side output layout of compress_layer_head_budgets: cu_out
+    ``[H_kv, B+1]`` (group-major packing) and the total number of rows."""
+    b = np.asarray(group_budgets, dtype=np.int64).reshape(problem.batch, problem.num_kv_heads)
+    lens = np.diff(np.asarray(problem._cu, dtype=np.int64))
+    kept = np.minimum(b, lens[:, None])
+    cu = np.zeros((problem.num_kv_heads, problem.batch + 1), dtype=np.int32)
+    row = 0
+    for g in range(problem.num_kv_heads):
+        for s in range(problem.batch):
+            cu[g, s] = row
+            row += int(kept[s, g])
+        cu[g, problem.batch] = row
+    return cu, row
+
+
+def compress_layer_head_budgets(problem: Problem, q_win, k, v, srh_mask, group_budgets, indices,
+                                k_out, v_out, ws, raw=None, pooled=None,
+                                stream=None) -> np.ndarray:
+    """compress_layer with a budget per (sequence, KV group): ``group_budgets``
+    is ``[B, H_kv]``; outputs are packed group-major (see head_budget_layout);
+    returns cu_out ``[H_kv, B+1]``."""
+    m, mp = _mask(srh_mask)
+    b, bp = _i32(np.asarray(group_budgets).reshape(-1))
+    cu_out = np.zeros((problem.num_kv_heads, problem.batch + 1), np.int32)
+    _check(load().compresskv_compress_layer_head_budgets(
+        problem.ref, _ptr(q_win), _ptr(k), _ptr(v), mp, bp, _ptr(indices),
+        cu_out.ctypes.data_as(POINTER(c_int32)), _ptr(k_out), _ptr(v_out), _ptr(raw),
+        _ptr(pooled), _ptr(ws), ws.numel(), _stream(stream)),
+        "compresskv_compress_layer_head_budgets")
     return cu_out
 
 

@@ -525,10 +525,14 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
 // ------------------------------------------------------------------ select / gather
 // Pooling (unless `pooled_in` holds the pooled scores already), top-k and
 // window append, optionally fused with the K/V gather.
+// With `unit_out` (head-level budgets) every unit (s, g) has its own output
+// rows (first row, count) in a group-major packing, and cu_out[I.B] is the
+// total row count.
 int run_select(const ckv_problem* p, const Info& I, const float* raw, const float* pooled_in,
                const std::vector<int>& cu_out, int32_t* indices, float* pooled,
                const Workspace& ws, cudaStream_t stream, const void* k = nullptr,
-               const void* v = nullptr, void* k_out = nullptr, void* v_out = nullptr) {
+               const void* v = nullptr, void* k_out = nullptr, void* v_out = nullptr,
+               const std::vector<int2>* unit_out = nullptr) {
   if (!raw && !pooled_in && I.p_total > 0) return CKV_ERR_INVALID_ARG;
   if (!indices && cu_out[I.B] > 0) return CKV_ERR_INVALID_ARG;
   const bool gather = k != nullptr;
@@ -563,6 +567,11 @@ int run_select(const ckv_problem* p, const Info& I, const float* raw, const floa
   P.num_kv_heads = I.Hkv;
   P.p_total = static_cast<int>(I.p_total);
   P.o_total = cu_out[I.B];
+  if (unit_out) {
+    if (unit_out->size() > static_cast<size_t>(kMaxBudgetUnits)) return CKV_ERR_UNSUPPORTED;
+    P.head_budgets = 1;
+    for (size_t u = 0; u < unit_out->size(); ++u) P.unit_out[u] = (*unit_out)[u];
+  }
   P.batch = I.B;
   int max_n = 0;
   for (int s = 0; s <= I.B; ++s) {
@@ -754,6 +763,53 @@ int compresskv_compress_layer_lse(const ckv_problem* p, const void* q_win, const
   lse.head_stride = lse_head_stride;
   if ((rc = run_score(p, I, q_win, k, srh_mask, raw, nullptr, ws, st, lse)) != CKV_OK) return rc;
   return run_select(p, I, raw, nullptr, co, indices, pooled_scores, ws, st, k, v, k_out, v_out);
+}
+
+int compresskv_compress_layer_head_budgets(const ckv_problem* p, const void* q_win,
+                                           const void* k, const void* v,
+                                           const uint8_t* srh_mask,
+                                           const int32_t* group_budgets, int32_t* indices,
+                                           int32_t* cu_out, void* k_out, void* v_out,
+                                           float* raw_scores, float* pooled_scores,
+                                           void* workspace, size_t workspace_bytes,
+                                           void* stream) {
+  Info I;
+  int rc = validate(p, I);
+  if (rc != CKV_OK) return rc;
+  if (I.layer) return CKV_ERR_INVALID_ARG;  // one shared selection has one budget
+  if (!group_budgets || !cu_out) return CKV_ERR_INVALID_ARG;
+  if (static_cast<long long>(I.B) * I.Hkv > kMaxBudgetUnits) return CKV_ERR_UNSUPPORTED;
+  // group-major packing: group g's sequences follow each other, then group g+1
+  std::vector<int2> unit_out(static_cast<size_t>(I.B) * I.Hkv);
+  long long row = 0;
+  for (int g = 0; g < I.Hkv; ++g) {
+    for (int s = 0; s < I.B; ++s) {
+      const int b = group_budgets[static_cast<long long>(s) * I.Hkv + g];
+      if (b < I.W) return CKV_ERR_BUDGET;
+      const int kept = std::min(b, I.len[s]);
+      unit_out[static_cast<size_t>(s) * I.Hkv + g] = make_int2(static_cast<int>(row), kept);
+      row += kept;
+    }
+  }
+  if (row > (1LL << 31) - 1) return CKV_ERR_UNSUPPORTED;
+  Workspace ws;
+  if ((rc = carve(I, workspace, workspace_bytes, ws)) != CKV_OK) return rc;
+  SrhLists S;
+  if ((rc = srh_lists(I, srh_mask, S)) != CKV_OK) return rc;
+  for (int g = 0; g < I.Hkv; ++g) {
+    for (int s = 0; s <= I.B; ++s) {
+      cu_out[g * (I.B + 1) + s] =
+          s < I.B ? unit_out[static_cast<size_t>(s) * I.Hkv + g].x
+                  : (g + 1 < I.Hkv ? unit_out[static_cast<size_t>(g + 1)].x : static_cast<int>(row));
+    }
+  }
+  std::vector<int> co(I.B + 1, 0);
+  co[I.B] = static_cast<int>(row);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  float* pooled = pooled_scores ? pooled_scores : ws.pooled;
+  if ((rc = run_score(p, I, q_win, k, srh_mask, raw_scores, pooled, ws, st)) != CKV_OK) return rc;
+  return run_select(p, I, nullptr, pooled, co, indices, nullptr, ws, st, k, v, k_out, v_out,
+                    &unit_out);
 }
 
 int compresskv_read_device_status(const void* workspace, void* stream, int32_t* status) {

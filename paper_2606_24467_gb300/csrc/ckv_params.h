@@ -5,6 +5,7 @@
 
 #include <cstdint>
 #include <cuda.h>
+#include <vector_types.h>
 
 namespace ckv {
 
@@ -16,6 +17,7 @@ constexpr int kMaxBatch = 512;
 constexpr int kMaxQHeads = 256;
 constexpr int kMaxKvHeads = 64;
 constexpr int kMaxItems = 1024;     // score work items per launch
+constexpr int kMaxBudgetUnits = 2048;  // (sequence, group) pairs with their own budget
 constexpr uint64_t kWaitTimeoutNs = 2000000000ull;  // 2 s: far above any legitimate wait
 
 // Device status codes (mirrors of the public CKV_ERR_* values).
@@ -101,11 +103,13 @@ struct SelectParams {
   int slice;                   // prefix tokens per CTA (multiple of 32)
   int smem_slice;              // 1: raw and pooled slices live in shared memory
   int gather;                  // 1: also copy the retained K/V rows
+  int head_budgets;            // 1: a budget per (sequence, group), outputs packed group-major
   int layer_scope;             // 1: one selection per sequence, shared by every KV group
   float* shared_ws;            // layer scope: workspace row for the summed scores [p_total]
   int cu_seqlens[kMaxBatch + 1];
   int cu_prefix[kMaxBatch + 1];
   int cu_out[kMaxBatch + 1];
+  int2 unit_out[kMaxBudgetUnits];  // head budgets: (first output row, rows) of unit s*H_kv + g
 };
 
 struct GatherParams {

@@ -101,7 +101,10 @@ __device__ __forceinline__ void copy_kv_rows(const SelectParams& p, int seq0, in
         const long long src = static_cast<long long>(seq0 + tok) * p.tok_stride_v16 +
                               static_cast<long long>(g) * p.head_stride_v16 + part;
         v[u] = __ldg((is_v[u] ? p.v : p.k) + src);
-        dst[u] = (static_cast<long long>(out0 + first + i) * p.num_kv_heads + g) *
+        // one row per (token, group), or per token of this group when the
+        // output is packed group-major (head-level budgets)
+        dst[u] = (p.head_budgets ? static_cast<long long>(out0 + first + i)
+                                 : static_cast<long long>(out0 + first + i) * p.num_kv_heads + g) *
                      (kHeadDim * 2 / 16) + part;
       }
     }
@@ -137,9 +140,11 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   const int L = p.cu_seqlens[s + 1] - seq0;
   const int W = p.window;
   const int n = max(L - W, 0);
-  const int out0 = p.cu_out[s];
-  const int kept = p.cu_out[s + 1] - out0;
-  int32_t* out = p.indices + static_cast<long long>(g) * p.o_total + out0;
+  // output rows of the unit: per sequence (shared by the groups), or per
+  // (sequence, group) with head-level budgets (packed group-major)
+  const int out0 = p.head_budgets ? p.unit_out[u].x : p.cu_out[s];
+  const int kept = p.head_budgets ? p.unit_out[u].y : p.cu_out[s + 1] - out0;
+  int32_t* out = p.indices + (p.head_budgets ? 0 : static_cast<long long>(g) * p.o_total) + out0;
   const long long ostride = p.o_total;  // index rows of the groups (layer scope writes all)
   const long long soff = static_cast<long long>(g) * p.p_total + p.cu_prefix[s];
   const float* raw = p.raw + soff;

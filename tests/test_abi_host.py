@@ -142,3 +142,24 @@ def test_layer_scope_host_errors():
     rc = lib.compresskv_select(prob.ref, vp(1 << 30), bp, vp(1 << 30), cu_out, vp(1 << 30),
                                vp(1 << 30), n, None)
     assert rc == B.CKV_ERR_INVALID_ARG
+
+
+def test_head_budget_host_errors_and_layout():
+    lib = ckv.load()
+    prob, q, k = _problem()
+    cu, rows = ckv.head_budget_layout(prob, [[100, 50], [300, 40]])
+    assert cu.tolist() == [[0, 100, 140], [140, 190, 230]] and rows == 230
+    vp = ctypes.c_void_p
+    n = ckv.workspace_size(prob)
+    mask = np.ones(8, np.uint8)
+    cu_out = (ctypes.c_int32 * 6)()
+
+    def call(gb, problem=prob):
+        b, bp = B._i32(np.asarray(gb).reshape(-1))
+        return lib.compresskv_compress_layer_head_budgets(
+            problem.ref, vp(1 << 30), vp(1 << 30), vp(1 << 30), vp(mask.ctypes.data), bp,
+            vp(1 << 30), cu_out, vp(1 << 30), vp(1 << 30), None, None, vp(1 << 30), n, None)
+
+    assert call([[100, 31], [100, 100]]) == B.CKV_ERR_BUDGET
+    lay, _, _ = _problem(selection="layer")
+    assert call([[100, 100], [100, 100]], lay) == B.CKV_ERR_INVALID_ARG
