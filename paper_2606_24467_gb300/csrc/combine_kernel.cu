@@ -8,7 +8,7 @@
 // pair (M_i, S_i) with  sum over the item's keys of 2^(z*c) = S_i * 2^M_i.
 // This kernel
 //   1. merges the pairs of the unit's items into bias_q = log2 D_q, the log2
-//      of query q's softmax denominator (merged in item order);
+//      of query q's softmax denominator (merged in a fixed order);
 //   2. raw_j = sum_q e_qj * 2^(R - bias_q)   (every weight is <= 1);
 //   3. pooled_j = (sum_{t=-h..h} raw_{j+t}) / P with zeros outside [0, n),
 //      summed in a fixed order.
@@ -108,23 +108,43 @@ __global__ void __launch_bounds__(kCombThreads)
     }
   };
   load_batch(f_lo, ev);
+  // references (16-byte chunks: nqt * Nr is a multiple of 8 and the rows are
+  // 32-byte aligned) and softmax pairs arrive by asynchronous copies, all in
+  // flight together
   const float* R = p.refs + it.roff + static_cast<long long>(q0) * Nr;
-  for (int i = tid; i < nqt * Nr; i += kCombThreads) s_w[i] = R[i];
+  for (int i = 4 * tid; i < nqt * Nr; i += 4 * kCombThreads) cp_async16(smem_u32(s_w + i), R + i);
   const int per = kPairSlots / N;  // items staged per round
   const int ni0 = min(per, static_cast<int>(it.count));
   auto stage_pairs = [&](int i0, int ni) {
-    for (int ii = warp; ii < ni; ii += kCombThreads / 32) {
-      const float2* src = p.partials + static_cast<long long>(it.first + i0 + ii) * kMaxQRows;
-      for (int q = lane; q < N; q += 32) s_pairs[ii * N + q] = src[q];
+    for (int e = tid; e < ni * N; e += kCombThreads) {
+      const int ii = e / N;
+      const int q = e - ii * N;
+      cp_async8(smem_u32(s_pairs + e),
+                p.partials + static_cast<long long>(it.first + i0 + ii) * kMaxQRows + q);
     }
+    cp_async_wait_all();
   };
   stage_pairs(0, ni0);
   __syncthreads();
 
-  // 1. per-query log2 softmax denominators, item pairs merged in order (one
-  //    thread per query; units with many items take several staging rounds)
+  // 1. per-query log2 softmax denominators.  The item pairs are merged by
+  //    nm = 256 / N threads per query (thread t: query t % N, items
+  //    i = t / N (mod nm)), then the nm partial pairs in that order; units
+  //    with many items take several staging rounds.
   {
+    const int nm = kCombThreads / N;
+    const int q = tid % N;
+    const int sub = tid / N;
     float m = -INFINITY, z = 0.f;
+    auto merge = [&](float pm, float pz) {
+      if (pm == -INFINITY) return;
+      if (pm > m) {
+        z = fmaf(z, ex2_approx(m - pm), pz);
+        m = pm;
+      } else {
+        z = fmaf(pz, ex2_approx(pm - m), z);
+      }
+    };
     for (int i0 = 0; i0 < it.count; i0 += per) {
       const int ni = min(per, it.count - i0);
       if (i0 > 0) {
@@ -132,20 +152,23 @@ __global__ void __launch_bounds__(kCombThreads)
         stage_pairs(i0, ni);
         __syncthreads();
       }
-      if (tid < N) {
-        for (int ii = 0; ii < ni; ++ii) {
-          const float2 pr = s_pairs[ii * N + tid];
-          if (pr.x == -INFINITY) continue;
-          if (pr.x > m) {
-            z = fmaf(z, ex2_approx(m - pr.x), pr.y);
-            m = pr.x;
-          } else {
-            z = fmaf(pr.y, ex2_approx(pr.x - m), z);
-          }
+      if (sub < nm) {
+        for (int ii = sub; ii < ni; ii += nm) {
+          const float2 pr = s_pairs[ii * N + q];
+          merge(pr.x, pr.y);
         }
       }
     }
-    if (tid < N) s_bias[tid] = m + __log2f(z);
+    __syncthreads();  // every round's pairs have been read
+    float2* part = s_pairs;  // [nm][N] partial pairs
+    if (sub < nm) part[sub * N + q] = make_float2(m, z);
+    __syncthreads();
+    if (tid < N) {
+      m = -INFINITY;
+      z = 0.f;
+      for (int j = 0; j < nm; ++j) merge(part[j * N + tid].x, part[j * N + tid].y);
+      s_bias[tid] = m + __log2f(z);
+    }
   }
   __syncthreads();
 

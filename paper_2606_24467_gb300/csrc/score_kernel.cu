@@ -126,6 +126,29 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
   const int ntiles = it.t1 - t0;  // >= 1 by construction
 
   // ------------------------------------------------------------ set-up
+  // Window-query rows of the SRH heads -> shared memory in the UMMA K-major
+  // 128-byte-swizzle layout (row r, 16-byte chunk ch of each 64-column half
+  // lands at chunk ch ^ (r & 7)); rows N..Npad-1 are zero.  The copies are
+  // asynchronous and issued first, so their latency overlaps the set-up.
+  if (warp != 0) {
+    const int st_tid = threadIdx.x - 32;
+    for (int idx = st_tid; idx < Npad * 16; idx += kStagedThreads) {
+      const int r = idx >> 4;
+      const int ch = idx & 15;
+      uint8_t* dst = sQ + (ch >> 3) * qh + r * 128 + (((ch & 7) ^ (r & 7)) << 4);
+      if (r < N) {
+        const int head = p.srh_heads[h0 + r / W];
+        const int w = r - (r / W) * W;
+        cp_async16(smem_u32(dst), p.q + static_cast<long long>(s) * p.q_bs +
+                                      static_cast<long long>(head) * p.q_hs +
+                                      static_cast<long long>(w) * p.q_ws + ch * 8);
+      } else {
+        *reinterpret_cast<uint4*>(dst) = make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
+  }
+  const uint64_t kpol = p.use_evict_hint ? l2_policy_evict_first() : l2_policy_evict_last();
+  const int prefill = min(nst, ntiles);  // ring stages filled before the CTA-wide barrier
   if (threadIdx.x == 0) {
     for (int i = 0; i < nst; ++i) {
       mbar_init(full0 + 8 * i, 1);
@@ -137,8 +160,15 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
     }
     *abort_flag = 0;
     fence_mbar_init();
+    // the ring starts empty: its first tiles need no wait
+    for (int i = 0; i < prefill; ++i) {
+      mbar_arrive_expect_tx(full0 + 8 * i, kTileBytes);
+      const int row = seq0 + (t0 + i) * kTileTokens;
+      const uint32_t dst = smem_u32(sK + i * kTileBytes);
+      tma_load_3d(dst, &p.tmap_k, full0 + 8 * i, 0, g, row, kpol);
+      tma_load_3d(dst + kHalfTileBytes, &p.tmap_k, full0 + 8 * i, 64, g, row, kpol);
+    }
   }
-  if (warp == 0 && lane == 0) tma_prefetch_map(&p.tmap_k);
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_holder), tcols);
     tmem_relinquish();
@@ -151,17 +181,16 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
   if (warp == 0) {
     // ---------------------------------------------------------- TMA producer
     if (lane == 0) {
-      const uint64_t pol = p.use_evict_hint ? l2_policy_evict_first() : l2_policy_evict_last();
-      int issued = 0;
-      for (int i = 0; i < ntiles; ++i) {
+      int issued = prefill;
+      for (int i = prefill; i < ntiles; ++i) {
         const int st = i % nst;
         const uint32_t ph = static_cast<uint32_t>(i / nst) & 1u;
         if (!mbar_wait_bounded(empty0 + 8 * st, ph ^ 1u, abort_flag, p.status)) break;
         mbar_arrive_expect_tx(full0 + 8 * st, kTileBytes);
         const int row = seq0 + (t0 + i) * kTileTokens;
         const uint32_t dst = smem_u32(sK + st * kTileBytes);
-        tma_load_3d(dst, &p.tmap_k, full0 + 8 * st, 0, g, row, pol);
-        tma_load_3d(dst + kHalfTileBytes, &p.tmap_k, full0 + 8 * st, 64, g, row, pol);
+        tma_load_3d(dst, &p.tmap_k, full0 + 8 * st, 0, g, row, kpol);
+        tma_load_3d(dst + kHalfTileBytes, &p.tmap_k, full0 + 8 * st, 64, g, row, kpol);
         ++issued;
       }
       if (*abort_flag) {
@@ -173,26 +202,10 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
     __syncwarp();  // reconverge before the CTA-wide (aligned) barrier below
   } else {
     // ---------------------------------------------------------- staging
-    // Window-query rows of the SRH heads -> shared memory in the UMMA K-major
-    // 128-byte-swizzle layout (row r, 16-byte chunk ch of each 64-column half
-    // lands at chunk ch ^ (r & 7)); rows N..Npad-1 are zero.
+    // the Q-row copies issued at entry have landed: make them visible to the
+    // tensor cores (async proxy)
     const int st_tid = threadIdx.x - 32;
-    for (int idx = st_tid; idx < Npad * 16; idx += kStagedThreads) {
-      const int r = idx >> 4;
-      const int ch = idx & 15;
-      uint4 val = make_uint4(0u, 0u, 0u, 0u);
-      if (r < N) {
-        const int head = p.srh_heads[h0 + r / W];
-        const int w = r - (r / W) * W;
-        const uint16_t* src = p.q + static_cast<long long>(s) * p.q_bs +
-                              static_cast<long long>(head) * p.q_hs +
-                              static_cast<long long>(w) * p.q_ws + ch * 8;
-        val = *reinterpret_cast<const uint4*>(src);
-      }
-      const int half = ch >> 3;
-      const int c8 = ch & 7;
-      *reinterpret_cast<uint4*>(sQ + half * qh + r * 128 + ((c8 ^ (r & 7)) << 4)) = val;
-    }
+    cp_async_wait_all();
     fence_proxy_async_smem();
     for (int q = st_tid; q < kMaxQRows; q += kStagedThreads) sWpos[q] = q < N ? q % W : 0;
     if constexpr (kLse) {
