@@ -38,6 +38,7 @@ struct DeviceFacts {
   int smem_optin = 0;
   long long l2_bytes = 0;
   size_t combine_smem_max = 0;  // dynamic shared memory the combine kernel may use
+  int sampled_cluster = 8;      // largest cluster of the sampled select (16 or 8)
   bool smem_attr_set = false;
 };
 
@@ -68,6 +69,7 @@ int device_facts(DeviceFacts** out) {
       return CKV_ERR_CUDA;
     if (select_set_smem_limit(static_cast<size_t>(select_max_smem_floats()) * 4) != cudaSuccess)
       return CKV_ERR_CUDA;
+    f.sampled_cluster = select_sampled_max_cluster(kScTargetSlice);
     f.smem_attr_set = true;
   }
   if (!g_encode) {
@@ -454,18 +456,29 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
       if (best < 0) break;
       ++cnt[best];
     }
-    // Combine items: chunks of 32-token quarters, about four CTAs per SM.
-    long long quarters = 0;
+    // Combine items: chunks of 32-token quarters, about four CTAs per SM,
+    // balanced by bytes: a quarter of a unit with exponent rows of nr
+    // columns weighs nr + 16 (table bytes plus a fixed share per key).
+    constexpr int kQuarterFixed = 16;
+    long long weight = 0;
     for (int u = 0; u < nu; ++u)
-      if (cnt[u] > 0) quarters += units[u0 + u].quarters;
+      if (cnt[u] > 0)
+        weight += static_cast<long long>(units[u0 + u].quarters) *
+                  (expo_stride(S.rows[units[u0 + u].g]) + kQuarterFixed);
     const long long ctarget = std::max(1, std::min(kMaxItems - nu, 4 * F->sms));
-    int chunk_q = static_cast<int>(std::max(8LL, (quarters + ctarget - 1) / ctarget));
-    int max_nr = 8;
-    for (int u = 0; u < nu; ++u) max_nr = std::max(max_nr, expo_stride(S.rows[units[u0 + u].g]));
-    // a chunk's weight table and raw scores must fit the shared memory
-    while (chunk_q > 1 && combine_smem_bytes(chunk_q, max_nr, I.P) > F->combine_smem_max)
-      chunk_q = (chunk_q + 1) / 2;
-    const size_t csmem = combine_smem_bytes(chunk_q, max_nr, I.P);
+    const long long per_chunk = std::max<long long>(8 * (8 + kQuarterFixed),
+                                                    (weight + ctarget - 1) / ctarget);
+    std::vector<int> chunk_q(nu, 1);
+    size_t csmem = 0;
+    for (int u = 0; u < nu; ++u) {
+      if (cnt[u] == 0) continue;
+      const int nr = expo_stride(S.rows[units[u0 + u].g]);
+      int cq = static_cast<int>(std::max(1LL, per_chunk / (nr + kQuarterFixed)));
+      // a chunk's weight table and raw scores must fit the shared memory
+      while (cq > 1 && combine_smem_bytes(cq, nr, I.P) > F->combine_smem_max) cq = (cq + 1) / 2;
+      chunk_q[u] = cq;
+      csmem = std::max(csmem, combine_smem_bytes(cq, nr, I.P));
+    }
     if (csmem > F->combine_smem_max) return CKV_ERR_UNSUPPORTED;
 
     int n_items = 0, n_comb = 0;
@@ -487,12 +500,12 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
         it.eoff = eoff;
         it.roff = roff;
       }
-      for (int q0 = 0; q0 < U.quarters; q0 += chunk_q) {
+      for (int q0 = 0; q0 < U.quarters; q0 += chunk_q[u]) {
         if (n_comb >= kMaxItems) return CKV_ERR_UNSUPPORTED;
         WorkItem& it = C.items[n_comb++];
         it = P.items[n_items];
         it.t0 = static_cast<uint16_t>(q0);
-        it.t1 = static_cast<uint16_t>(std::min(U.quarters, q0 + chunk_q));
+        it.t1 = static_cast<uint16_t>(std::min(U.quarters, q0 + chunk_q[u]));
       }
       n_items += c_u;
       eoff += static_cast<uint32_t>(I.n[U.s]) * static_cast<uint32_t>(nr);
@@ -579,6 +592,21 @@ int run_select(const ckv_problem* p, const Info& I, const float* raw, const floa
     P.cu_prefix[s] = I.cu_prefix[s];
     P.cu_out[s] = cu_out[s];
     if (s < I.B) max_n = std::max(max_n, I.n[s]);
+  }
+  if (pooled_in && !I.layer) {
+    // fused layer call, per-group selection: sampled select, a cluster of up
+    // to 16 CTAs per unit with about kScTargetSlice positions each
+    const int C = std::min(F->sampled_cluster,
+                           std::max(1, (max_n + kScTargetSlice - 1) / kScTargetSlice));
+    const int S = std::max(32, ((max_n + C - 1) / C + 31) / 32 * 32);
+    if (S <= kScMaxSlice) {
+      P.cluster = C;
+      P.slice = S;
+      Tracer tr{p->trace, stream};
+      const size_t smem = select_sampled_smem_bytes(S);
+      return traced(tr, CKV_KERNEL_SELECT,
+                    [&] { return launch_select_sampled(P, I.B * I.Hkv, smem, stream); });
+    }
   }
   // A cluster of up to 8 CTAs per unit, about 4096 prefix tokens per CTA
   // (one CTA per unit is several times slower: the four radix passes over a

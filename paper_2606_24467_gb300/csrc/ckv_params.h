@@ -130,6 +130,13 @@ cudaError_t launch_score(const ScoreParams& p, int n_items, size_t smem, cudaStr
 cudaError_t launch_score_lse(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s);
 cudaError_t launch_combine(const CombineParams& p, int n_items, size_t smem, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, int n_units, size_t smem, cudaStream_t s);
+// Per-group selection from pooled scores by sampling (clusters of up to 16
+// CTAs, `p.slice` <= kScMaxSlice positions per CTA).
+constexpr int kScMaxSlice = 16384;
+constexpr int kScTargetSlice = 2048;  // positions per CTA when the cluster allows
+cudaError_t launch_select_sampled(const SelectParams& p, int n_units, size_t smem, cudaStream_t s);
+size_t select_sampled_smem_bytes(int slice);
+int select_sampled_max_cluster(int slice);  // 16 when the device takes such clusters, else 8
 cudaError_t launch_gather(const GatherParams& p, long long rows, cudaStream_t s);
 size_t score_smem_bytes(int q_half_bytes, int stages, int epi_warps);
 // Sets every scoring kernel's shared-memory limit: `bytes` for one CTA per

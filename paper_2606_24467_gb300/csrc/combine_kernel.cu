@@ -36,7 +36,7 @@ namespace {
 
 constexpr int kCombThreads = 256;
 constexpr int kLoadBatch = 4;  // 16-byte loads per batch (two batches in flight per thread)
-constexpr int kPairSlots = 2048;  // softmax pairs staged per round
+constexpr int kPairSlots = 4096;  // softmax pairs staged per round
 static_assert(kMaxQRows <= kCombThreads, "one thread per query row");
 
 __device__ __forceinline__ float dot8(const uint4 v, const float* w) {
@@ -65,8 +65,6 @@ __global__ void __launch_bounds__(kCombThreads)
   __shared__ float2 s_pairs[kPairSlots];
 
   const int tid = threadIdx.x;
-  const int warp = tid >> 5;
-  const int lane = tid & 31;
   const WorkItem it = p.items[blockIdx.x];
   const int s = it.seq;
   const int g = it.group;

@@ -79,18 +79,19 @@ __device__ __forceinline__ T* unit_rank_ptr(T* ptr, int rank) {
 // output rows: token i is out[first + i] (a position in the sequence) and goes
 // to output row out0 + first + i.  Each thread moves 16-byte chunks, issuing
 // a batch of loads before the matching stores.
+template <int kThreads = kSelThreads>
 __device__ __forceinline__ void copy_kv_rows(const SelectParams& p, int seq0, int g,
                                              const int32_t* out, int out0, int first, int count) {
   constexpr int kChunks = 2 * kHeadDim * 2 / 16;  // 16 K + 16 V chunks per token
   constexpr int kBatch = 4;
   const int total = count * kChunks;
-  for (int base = 0; base < total; base += kBatch * kSelThreads) {
+  for (int base = 0; base < total; base += kBatch * kThreads) {
     uint4 v[kBatch];
     long long dst[kBatch];
     bool is_v[kBatch];
 #pragma unroll
     for (int u = 0; u < kBatch; ++u) {
-      const int e = base + u * kSelThreads + static_cast<int>(threadIdx.x);
+      const int e = base + u * kThreads + static_cast<int>(threadIdx.x);
       dst[u] = -1;
       if (e < total) {
         const int i = e / kChunks;
@@ -288,9 +289,15 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
       const bool match = i < len && (key & pmask) == prefix;
       const uint32_t bin = (key >> sh) & 255u;
       const uint32_t active = __ballot_sync(0xffffffffu, match);
-      if (match) {
-        const uint32_t peers = __match_any_sync(active, bin);
-        if (lane == __ffs(peers) - 1) atomicAdd(&h[bin], static_cast<uint32_t>(__popc(peers)));
+      if (active) {
+        // one add per warp when its keys share the bin, else one per key
+        const int leader = __ffs(active) - 1;
+        const uint32_t lb = __shfl_sync(0xffffffffu, bin, leader);
+        if (__all_sync(0xffffffffu, !match || bin == lb)) {
+          if (lane == leader) atomicAdd(&h[lb], static_cast<uint32_t>(__popc(active)));
+        } else if (match) {
+          atomicAdd(&h[bin], 1u);
+        }
       }
     }
     unit_barrier<kCluster>();
@@ -420,12 +427,498 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   }
 }
 
+
+// ---------------------------------------------------------------------------
+// Sampled cluster select (per-group selection of a fused layer call): the same
+// result as select_kernel -- the top-k prefix positions of every unit by
+// pooled score, ties to the lower position, ascending, the window appended,
+// the K/V rows copied -- with three cluster barriers instead of one per radix
+// pass.  One cluster of C <= 16 CTAs per unit; CTA r owns the contiguous
+// slice [r*S, (r+1)*S) of the unit's prefix positions.
+//   1. The slice's pooled scores go to shared memory; each CTA sends 64
+//      evenly spaced scores of its slice to every CTA of the cluster.
+//   2. Every CTA takes the same lower bound lo for the k-th largest score:
+//      the r-th largest sample, r a few standard deviations above the
+//      expected number k * (samples / n) of samples above the k-th score.
+//   3. Each CTA lists its keys >= lo in position order and sends the count.
+//      When between k and kScCandCap keys reach lo (the usual case), every
+//      CTA reads all lists (position order across the cluster), finds the
+//      k-th largest key tau and how many keys equal to it are kept, and
+//      writes its own selected positions at offsets counted in that list.
+//      Otherwise every CTA runs the same search over all of the unit's
+//      scores (read from global memory) and counts from there.
+//   4. The last CTA appends the window; every CTA copies its own K/V rows.
+// Pooled scores are >= 0, so their fp32 bit patterns order like the values.
+constexpr int kScThreads = 256;
+constexpr int kScWarps = kScThreads / 32;
+constexpr int kScSamples = 64;    // samples per CTA
+constexpr int kScMaxC = 16;       // CTAs per cluster
+constexpr int kScCandCap = 4096;  // candidates per unit
+static_assert(kScThreads == 256, "one thread per radix bin");
+
+struct ScShared {
+  uint32_t samp[kScMaxC * kScSamples];  // written by every CTA of the cluster
+  int samp_cnt[kScMaxC];
+  int cand_cnt[kScMaxC];
+  int ovf[kScMaxC];
+  uint32_t ckey[kScCandCap];  // own candidates, position order
+  int cpos[kScCandCap];
+  uint32_t all[kScCandCap];   // every CTA's candidates, position order
+  uint32_t hist[4][256];      // radix histograms, used in rotation
+  int wcnt[kScWarps];
+  int wbase[kScWarps];
+  uint32_t key_or[2], key_and[2];  // one pair per search
+  int red[2][2];                    // one pair of sums per use
+  int red0;
+};
+
+// Zero state the searches below expect (before the kernel's first barrier).
+__device__ __forceinline__ void sc_init_shared(ScShared& sh) {
+  const int tid = threadIdx.x;
+  for (int i = tid; i < 2 * 256; i += kScThreads) sh.hist[i >> 8][i & 255] = 0u;
+  if (tid < 2) {
+    sh.key_or[tid] = 0u;
+    sh.key_and[tid] = 0xFFFFFFFFu;
+    sh.red[tid][0] = 0;
+    sh.red[tid][1] = 0;
+  }
+}
+
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  __syncwarp();
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_arrive_release() {
+  __syncwarp();
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  __syncwarp();
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Whole warp: the bin of `h[0..255]` (counts; higher bin = larger keys)
+// holding the rem-th largest key, and the count of keys in the bins above it
+// (every lane receives both).
+__device__ __forceinline__ void warp_pick_bin256(const uint32_t* h, int rem, int lane, int* bin,
+                                                 int* above_out) {
+  uint32_t c[8];
+  uint32_t cnt = 0u;
+#pragma unroll
+  for (int b = 0; b < 8; ++b) {
+    c[b] = h[lane * 8 + b];
+    cnt += c[b];
+  }
+  uint32_t suf = cnt;  // inclusive suffix sum over lanes
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const uint32_t y = __shfl_down_sync(0xffffffffu, suf, off);
+    if (lane + off < 32) suf += y;
+  }
+  const uint32_t ok = __ballot_sync(0xffffffffu, suf >= static_cast<uint32_t>(rem));
+  const int top = ok ? 31 - __clz(ok) : 0;
+  uint32_t above = __shfl_sync(0xffffffffu, suf - cnt, top);  // keys above lane top's bins
+  int bsel = top * 8;
+  if (lane == top) {
+    for (int b = 7; b >= 0; --b) {
+      if (above + c[b] >= static_cast<uint32_t>(rem)) {
+        bsel = top * 8 + b;
+        break;
+      }
+      above += c[b];
+    }
+  }
+  *bin = __shfl_sync(0xffffffffu, bsel, top);
+  *above_out = static_cast<int>(__shfl_sync(0xffffffffu, above, top));
+}
+
+// CTA-wide: the r-th largest (1 <= r <= number of keys) of the keys that
+// `visit` presents (visit(f) calls f(key, valid) equally often on every lane
+// of a warp).  Returns the key tau; *rem = how many keys equal to tau are
+// among the r largest.  The radix passes (8 bits each) start at the highest
+// bit in which the keys differ; each pass has one barrier: pass number pc
+// counts into hist[pc % 4] (zero on entry, as is hist[(pc + 1) % 4]) while
+// hist[(pc + 2) % 4], last read two passes earlier, is cleared, and every warp
+// then picks the bin itself.  `slot` selects this search's key_or / key_and.
+template <class Visit>
+__device__ uint32_t cta_kth_largest(const Visit& visit, int r, ScShared& sh, int slot, int& pc,
+                                    int* rem) {
+  const int tid = threadIdx.x;
+  const int lane = tid & 31;
+  uint32_t ko = 0u, ka = 0xFFFFFFFFu;
+  visit([&](uint32_t key, bool valid) {
+    if (valid) {
+      ko |= key;
+      ka &= key;
+    }
+  });
+  ko = __reduce_or_sync(0xffffffffu, ko);
+  ka = __reduce_and_sync(0xffffffffu, ka);
+  if (lane == 0) {
+    atomicOr(&sh.key_or[slot], ko);
+    atomicAnd(&sh.key_and[slot], ka);
+  }
+  __syncthreads();
+  const uint32_t diff = sh.key_or[slot] ^ sh.key_and[slot];
+  const uint32_t kand = sh.key_and[slot];
+  int remaining = r;
+  if (diff == 0u) {  // all keys equal
+    *rem = remaining;
+    return kand;
+  }
+  int hb = 31 - __clz(diff);
+  uint32_t pmask = hb == 31 ? 0u : ~((2u << hb) - 1u);
+  uint32_t prefix = kand & pmask;
+#pragma unroll 1
+  while (hb >= 0) {
+    const int width = min(8, hb + 1);
+    const int shf = hb + 1 - width;
+    const uint32_t fm = (1u << width) - 1u;
+    uint32_t* h = sh.hist[pc & 3];
+    visit([&](uint32_t key, bool valid) {
+      const bool m = valid && (key & pmask) == prefix;
+      const uint32_t act = __ballot_sync(0xffffffffu, m);
+      if (!act) return;
+      const uint32_t bin = (key >> shf) & fm;
+      const int leader = __ffs(act) - 1;
+      const uint32_t lb = __shfl_sync(0xffffffffu, bin, leader);
+      // one add per warp when its keys share the bin (dense scores), else
+      // one per key
+      if (__all_sync(0xffffffffu, !m || bin == lb)) {
+        if (lane == leader) atomicAdd(&h[lb], static_cast<uint32_t>(__popc(act)));
+      } else if (m) {
+        atomicAdd(&h[bin], 1u);
+      }
+    });
+    sh.hist[(pc + 2) & 3][tid] = 0u;  // kScThreads == 256 bins
+    __syncthreads();
+    int bin, above;
+    warp_pick_bin256(h, remaining, lane, &bin, &above);
+    remaining -= above;
+    prefix |= static_cast<uint32_t>(bin) << shf;
+    pmask |= fm << shf;
+    hb = shf - 1;
+    ++pc;
+  }
+  *rem = remaining;
+  return prefix;
+}
+
+// CTA-wide sums of two ints into sh.red[slot] (zero on entry; every thread
+// receives both).
+__device__ __forceinline__ void cta_sum2(int a, int b, ScShared& sh, int slot, int* sa, int* sb) {
+  a = __reduce_add_sync(0xffffffffu, a);
+  b = __reduce_add_sync(0xffffffffu, b);
+  if ((threadIdx.x & 31) == 0) {
+    atomicAdd(&sh.red[slot][0], a);
+    atomicAdd(&sh.red[slot][1], b);
+  }
+  __syncthreads();
+  *sa = sh.red[slot][0];
+  *sb = sh.red[slot][1];
+}
+
+__global__ void __launch_bounds__(kScThreads)
+    select_sampled_kernel(const __grid_constant__ SelectParams p) {
+  extern __shared__ __align__(16) uint8_t sc_raw[];
+  ScShared& sh = *reinterpret_cast<ScShared*>(sc_raw);
+  float* s_keys = reinterpret_cast<float*>(sc_raw + ((sizeof(ScShared) + 15) & ~size_t(15)));
+  cg::cluster_group cluster = cg::this_cluster();
+  const int C = static_cast<int>(cluster.num_blocks());
+  const int cr = static_cast<int>(cluster.block_rank());
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5;
+  const int lane = tid & 31;
+  const int u = blockIdx.x / C;
+  const int s = u / p.num_kv_heads;
+  const int g = u - s * p.num_kv_heads;
+  const int seq0 = p.cu_seqlens[s];
+  const int L = p.cu_seqlens[s + 1] - seq0;
+  const int W = p.window;
+  const int n = max(L - W, 0);
+  const int out0 = p.head_budgets ? p.unit_out[u].x : p.cu_out[s];
+  const int kept = p.head_budgets ? p.unit_out[u].y : p.cu_out[s + 1] - out0;
+  int32_t* out = p.indices + (p.head_budgets ? 0 : static_cast<long long>(g) * p.o_total) + out0;
+  const float* pooled = p.pooled_in + static_cast<long long>(g) * p.p_total + p.cu_prefix[s];
+  const uint32_t* gkeys = reinterpret_cast<const uint32_t*>(pooled);
+  const int S = p.slice;
+  const int lo_c = min(n, cr * S);
+  const int len = min(n, lo_c + S) - lo_c;
+
+  pdl_launch_dependents();
+  cluster_arrive_relaxed();  // this CTA has started (remote shared memory may be written)
+  pdl_wait();                // pooled scores come from the previous kernel
+
+  if (kept >= L) {  // keep everything (uniform over the cluster)
+    const int per = (L + C - 1) / C;
+    const int a0 = min(L, cr * per);
+    const int a1 = min(L, a0 + per);
+    for (int i = a0 + tid; i < a1; i += kScThreads) out[i] = i;
+    if (p.gather && a1 > a0) {
+      __syncthreads();
+      copy_kv_rows<kScThreads>(p, seq0, g, out, out0, a0, a1 - a0);
+    }
+    cluster_wait();
+    return;
+  }
+  const int k = kept - W;  // 0 <= k < n
+  if (cr == C - 1)
+    for (int w = tid; w < W; w += kScThreads) out[k + w] = n + w;
+  if (k == 0) {
+    if (p.gather && cr == C - 1) {
+      __syncthreads();
+      copy_kv_rows<kScThreads>(p, seq0, g, out, out0, 0, W);
+    }
+    cluster_wait();
+    return;
+  }
+
+  // 1. slice -> shared memory; samples to every CTA
+  sc_init_shared(sh);
+  int pc = 0;  // radix passes run so far (histogram rotation)
+  for (int i = tid; i < len; i += kScThreads) cp_async4(smem_u32(s_keys + i), pooled + lo_c + i);
+  cp_async_wait_all();
+  __syncthreads();
+  auto key_at = [&](int i) { return __float_as_uint(s_keys[i]); };
+  const int ns_c = min(kScSamples, len);
+  cluster_wait();  // every CTA has started
+  if (tid < ns_c) {
+    const uint32_t v = key_at(static_cast<int>((static_cast<long long>(tid) * len) / ns_c));
+    for (int t = 0; t < C; ++t) *cluster.map_shared_rank(&sh.samp[cr * kScSamples + tid], t) = v;
+  }
+  if (tid < C) *cluster.map_shared_rank(&sh.samp_cnt[cr], tid) = ns_c;
+  cluster_arrive_release();
+  cluster_wait();
+
+  // 2. lower bound from the samples
+  int nsamp = 0;
+  for (int c = 0; c < C; ++c) nsamp += sh.samp_cnt[c];
+  const float mu = static_cast<float>(k) * static_cast<float>(nsamp) / static_cast<float>(n);
+  const int rs = min(nsamp, static_cast<int>(ceilf(mu + 3.f * sqrtf(mu))) + 2);
+  int rem_s;
+  const uint32_t lo = cta_kth_largest(
+      [&](const auto& f) {
+        for (int j0 = 0; j0 < C * kScSamples; j0 += kScThreads) {
+          const int j = j0 + tid;
+          const bool v = j < C * kScSamples && (j % kScSamples) < sh.samp_cnt[j / kScSamples];
+          f(v ? sh.samp[j] : 0u, v);
+        }
+      },
+      rs, sh, 0, pc, &rem_s);
+
+  // 3. own candidates (keys >= lo) in position order; counts to every CTA
+  const int seg = ((len + kScThreads - 1) / kScThreads) * 32;  // positions per warp
+  const int wlo = min(len, warp * seg);
+  const int whi = min(len, wlo + seg);
+  int wc = 0;
+  for (int b0 = wlo; b0 < whi; b0 += 32) {
+    const int i = b0 + lane;
+    wc += __popc(__ballot_sync(0xffffffffu, i < whi && key_at(i) >= lo));
+  }
+  if (lane == 0) sh.wcnt[warp] = wc;
+  __syncthreads();
+  if (warp == 0) {
+    const int v = lane < kScWarps ? sh.wcnt[lane] : 0;
+    const int ex = warp_exclusive_scan(v, lane);
+    if (lane < kScWarps) sh.wbase[lane] = ex;
+    if (lane == kScWarps - 1) sh.red0 = ex + v;  // own candidate count
+  }
+  __syncthreads();
+  const int own = sh.red0;
+  {
+    int o = sh.wbase[warp];
+    for (int b0 = wlo; b0 < whi; b0 += 32) {
+      const int i = b0 + lane;
+      const bool c = i < whi && key_at(i) >= lo;
+      const uint32_t mm = __ballot_sync(0xffffffffu, c);
+      const int slot = o + __popc(mm & lanemask_lt(lane));
+      if (c && slot < kScCandCap) {
+        sh.ckey[slot] = key_at(i);
+        sh.cpos[slot] = lo_c + i;
+      }
+      o += __popc(mm);
+    }
+  }
+  if (tid < C) {
+    *cluster.map_shared_rank(&sh.cand_cnt[cr], tid) = own;
+    *cluster.map_shared_rank(&sh.ovf[cr], tid) = own > kScCandCap ? 1 : 0;
+  }
+  __syncthreads();  // own list complete before the others may read it
+  cluster_arrive_release();
+  cluster_wait();
+  int total = 0, before = 0, any_ovf = 0;
+  for (int c = 0; c < C; ++c) {
+    if (c < cr) before += sh.cand_cnt[c];
+    total += sh.cand_cnt[c];
+    any_ovf |= sh.ovf[c];
+  }
+  const bool fast = !any_ovf && total >= k && total <= kScCandCap;
+
+  // k-th largest key tau, keys equal to it that are kept, and this CTA's
+  // counts of keys > tau / == tau at lower positions of the unit
+  uint32_t tau;
+  int need_eq, gt_before, eq_before;
+  if (fast) {
+    // every CTA's list, concatenated in cluster (= position) order
+    for (int j = tid; j < total; j += kScThreads) {
+      int c = 0, off = 0;
+      while (off + sh.cand_cnt[c] <= j) off += sh.cand_cnt[c++];
+      sh.all[j] = *cluster.map_shared_rank(&sh.ckey[j - off], c);
+    }
+    __syncthreads();
+    cluster_arrive_release();  // done reading the other CTAs' shared memory
+    tau = cta_kth_largest(
+        [&](const auto& f) {
+          for (int j0 = 0; j0 < total; j0 += kScThreads) {
+            const int j = j0 + tid;
+            f(j < total ? sh.all[j] : 0u, j < total);
+          }
+        },
+        k, sh, 1, pc, &need_eq);
+    int a = 0, b = 0;
+    for (int j = tid; j < before; j += kScThreads) {
+      a += sh.all[j] > tau ? 1 : 0;
+      b += sh.all[j] == tau ? 1 : 0;
+    }
+    cta_sum2(a, b, sh, 0, &gt_before, &eq_before);
+  } else {
+    cluster_arrive_release();
+    tau = cta_kth_largest(
+        [&](const auto& f) {
+          for (int j0 = 0; j0 < n; j0 += kScThreads) {
+            const int j = j0 + tid;
+            f(j < n ? __ldg(gkeys + j) : 0u, j < n);
+          }
+        },
+        k, sh, 1, pc, &need_eq);
+    int a = 0, b = 0;
+    for (int j = tid; j < lo_c; j += kScThreads) {
+      const uint32_t key = __ldg(gkeys + j);
+      a += key > tau ? 1 : 0;
+      b += key == tau ? 1 : 0;
+    }
+    cta_sum2(a, b, sh, 1, &gt_before, &eq_before);
+  }
+
+  // 4. this CTA's selected positions (keys > tau, and keys == tau while fewer
+  //    than need_eq equal keys precede them), in position order
+  const int take_before = min(eq_before, need_eq);
+  const int first = gt_before + take_before;  // first output slot of this CTA
+  int count = 0;
+  {
+    int o = first;
+    int eq_seen = eq_before;
+    // scan the own keys >= tau in position order: the candidate list when it
+    // is complete, else the slice
+    const bool use_list = fast;
+    const int m = use_list ? own : len;
+    for (int j0 = 0; j0 < m; j0 += 32 * kScWarps) {
+      // one warp-wide step per 32 entries, warps in order
+      const int j = j0 + warp * 32 + lane;
+      const bool in = j < m;
+      const uint32_t key = in ? (use_list ? sh.ckey[j] : key_at(j)) : 0u;
+      const int pos = in ? (use_list ? sh.cpos[j] : lo_c + j) : 0;
+      const bool gt = in && key > tau;
+      const bool eq = in && key == tau;
+      const uint32_t mgt = __ballot_sync(0xffffffffu, gt);
+      const uint32_t meq = __ballot_sync(0xffffffffu, eq);
+      if (lane == 0) {
+        sh.wcnt[warp] = __popc(mgt);
+        sh.wbase[warp] = __popc(meq);
+      }
+      __syncthreads();
+      int gtb = 0, eqb = 0;
+      for (int w = 0; w < warp; ++w) {
+        gtb += sh.wcnt[w];
+        eqb += sh.wbase[w];
+      }
+      int gtt = gtb, eqt = eqb;
+      for (int w = warp; w < kScWarps; ++w) {
+        gtt += sh.wcnt[w];
+        eqt += sh.wbase[w];
+      }
+      const int eq_rank = eq_seen + eqb + __popc(meq & lanemask_lt(lane));
+      const bool take_eq = eq && eq_rank < need_eq;
+      const uint32_t msel = mgt | __ballot_sync(0xffffffffu, take_eq);
+      // selected entries before this lane: earlier warps' (gt + taken eq) + this warp's
+      const int eq_taken_before = max(0, min(need_eq - eq_seen, eqb));
+      const int slot = o + gtb + eq_taken_before + __popc(msel & lanemask_lt(lane));
+      if ((msel >> lane) & 1u) {
+        if (slot < k) out[slot] = pos;
+      }
+      const int eq_taken = max(0, min(need_eq - eq_seen, eqt));
+      o += gtt + eq_taken;
+      eq_seen += eqt;
+      __syncthreads();  // wcnt / wbase are rewritten by the next step
+    }
+    count = o - first;
+  }
+  if (p.gather) {
+    __syncthreads();  // the indices written above are read back by the copy
+    const int cnt = min(count, k - first);
+    if (cnt > 0) copy_kv_rows<kScThreads>(p, seq0, g, out, out0, first, cnt);
+    if (cr == C - 1) copy_kv_rows<kScThreads>(p, seq0, g, out, out0, k, W);
+  }
+  cluster_wait();  // no CTA leaves while another may still read its candidates
+}
+
 }  // namespace
+
+size_t select_sampled_smem_bytes(int slice) {
+  return ((sizeof(ScShared) + 15) & ~size_t(15)) + static_cast<size_t>(slice) * sizeof(float);
+}
+
+int select_sampled_max_cluster(int slice) {
+  // clusters of 16 CTAs are a non-portable size: use them when the device
+  // can hold one (else 8)
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(kScMaxC);
+  cfg.blockDim = dim3(kScThreads);
+  cfg.dynamicSmemBytes = select_sampled_smem_bytes(slice);
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = kScMaxC;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&clusters, select_sampled_kernel, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 8;
+  }
+  return clusters > 0 ? kScMaxC : 8;
+}
+
+cudaError_t launch_select_sampled(const SelectParams& p, int n_units, size_t smem,
+                                  cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(n_units * p.cluster));
+  cfg.blockDim = dim3(kScThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = static_cast<unsigned>(p.cluster);
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, select_sampled_kernel, p);
+}
 
 int select_max_smem_floats() { return (227 * 1024 - kSelStaticSmem - 1024) / 4; }
 
 cudaError_t select_set_smem_limit(size_t bytes) {
-  cudaError_t e = cudaFuncSetAttribute(select_kernel<false>,
+  cudaError_t e = cudaFuncSetAttribute(select_sampled_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(select_sampled_smem_bytes(kScMaxSlice)));
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(select_sampled_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(select_kernel<false>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(bytes));
   if (e != cudaSuccess) return e;
