@@ -143,8 +143,10 @@ typedef struct ckv_problem {
  * Returns 0 if `p` is invalid. */
 size_t compresskv_workspace_size(const ckv_problem* p);
 
-/* Zero the workspace status word (enqueued on `stream`).  Call once after
- * allocating a workspace, and after reading a non-zero device status. */
+/* Zero the workspace header -- the status word and the per-unit counters the
+ * scoring kernel uses to merge softmax denominators (4.3 KB, enqueued on
+ * `stream`).  Call once after allocating a workspace, and after reading a
+ * non-zero device status (an aborted call can leave the counters set). */
 int compresskv_workspace_init(void* workspace, size_t workspace_bytes, void* stream);
 
 /* Host-only: per-sequence offsets of the prefix scores (cu_prefix, [batch+1])

@@ -19,7 +19,11 @@ using namespace ckv;
 
 namespace {
 
-constexpr size_t kStatusBytes = 256;
+// Workspace header, zeroed by compresskv_workspace_init: the device status
+// word (256 B) and one ticket per scoring item (the scoring kernel's
+// last-CTA-per-unit merge resets the tickets it uses).
+constexpr size_t kTicketOffset = 256;
+constexpr size_t kStatusBytes = kTicketOffset + static_cast<size_t>(kMaxItems) * sizeof(int);
 // Units are scored in sets whose exponent tables (bounded with every head of
 // a group counted as SRH) take at most this many bytes; one set's table is
 // written by the scoring kernel and read back by the combine kernel, ideally
@@ -29,6 +33,7 @@ constexpr size_t kStatusBytes = 256;
 #endif
 constexpr long long kExpoSetBytes = CKV_EXPO_SET_BYTES;
 constexpr size_t kPartialBytes = static_cast<size_t>(kMaxItems) * kMaxQRows * sizeof(float2);
+constexpr size_t kBiasBytes = static_cast<size_t>(kMaxItems) * kMaxQRows * sizeof(float);
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
@@ -192,7 +197,9 @@ void plan_sets(const Info& I, std::vector<UnitSet>& sets) {
 
 struct Workspace {
   int* status = nullptr;
+  int* tickets = nullptr;    // [kMaxItems], in the header
   float2* partials = nullptr;
+  float* bias = nullptr;     // [kMaxItems][kMaxQRows] log2 softmax denominators per unit
   float* pooled = nullptr;   // score layout
   uint16_t* expo = nullptr;  // one set's exponent table
   float* refs = nullptr;     // one set's reference table
@@ -213,7 +220,7 @@ WorkspaceLayout workspace_layout(const Info& I) {
     r = std::max(r, S.ref_floats);
   }
   WorkspaceLayout W;
-  W.pooled = kStatusBytes + kPartialBytes;
+  W.pooled = kStatusBytes + kPartialBytes + kBiasBytes;
   W.expo = W.pooled + align256(static_cast<size_t>(I.Hkv) * I.p_total * sizeof(float));
   W.refs = W.expo + align256(static_cast<size_t>(e) * sizeof(uint16_t));
   W.shared = W.refs + align256(static_cast<size_t>(r) * sizeof(float));
@@ -229,7 +236,9 @@ int carve(const Info& I, void* ws, size_t bytes, Workspace& out) {
   if (!ws || bytes < W.total || (reinterpret_cast<uintptr_t>(ws) & 255u)) return CKV_ERR_WORKSPACE;
   char* b = static_cast<char*>(ws);
   out.status = reinterpret_cast<int*>(b);
+  out.tickets = reinterpret_cast<int*>(b + kTicketOffset);
   out.partials = reinterpret_cast<float2*>(b + kStatusBytes);
+  out.bias = reinterpret_cast<float*>(b + kStatusBytes + kPartialBytes);
   out.pooled = reinterpret_cast<float*>(b + W.pooled);
   out.expo = reinterpret_cast<uint16_t*>(b + W.expo);
   out.refs = reinterpret_cast<float*>(b + W.refs);
@@ -363,6 +372,8 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
   if ((rc = make_k_map(I, p, k, &P.tmap_k)) != CKV_OK) return rc;
   P.q = static_cast<const uint16_t*>(q_win);
   P.partials = ws.partials;
+  P.bias = ws.bias;
+  P.tickets = ws.tickets;
   P.expo = ws.expo;
   P.refs = ws.refs;
   P.status = ws.status;
@@ -380,7 +391,7 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
   P.raw_out = raw;
   P.p_total = static_cast<int>(I.p_total);
   for (int s = 0; s <= I.B; ++s) P.cu_prefix[s] = I.cu_prefix[s];
-  C.partials = ws.partials;
+  C.bias = ws.bias;
   C.expo = ws.expo;
   C.refs = ws.refs;
   C.raw_out = raw;

@@ -43,6 +43,8 @@ struct ScoreParams {
   CUtensorMap tmap_k;          // 3-D map over K: (d, kv head, token)
   const uint16_t* q;           // window queries (f16/bf16 bits)
   float2* partials;            // [n_items][kMaxQRows]: (M, S) with sum 2^(z*c) = S * 2^M
+  float* bias;                 // [item of the unit's first item][kMaxQRows]: log2 D_q per unit
+  int* tickets;                // [kMaxItems]: items of the unit done (zero between calls)
   uint16_t* expo;              // fp16 2^(z*c - R) per prefix key and query row (Nr per key)
   float* refs;                 // per (tile, quarter, query row): the R used for expo
   const float* lse;            // given-LSE mode: natural-log LSE per (sequence, head, window row)
@@ -65,7 +67,7 @@ struct ScoreParams {
 
 // Combine: normalised scores from the stored exponents, then pooling.
 struct CombineParams {
-  const float2* partials;
+  const float* bias;           // per unit (row = its first scoring item): log2 D_q
   const uint16_t* expo;
   const float* refs;
   float* raw_out;              // optional, score layout

@@ -4,15 +4,12 @@
 //
 // For unit (s, g) the scoring kernel stored, per prefix key j and query row
 // q, e_qj = 2^(z_qj*c - R) in fp16, where R = refs[quarter(j), q] is the
-// reference its warp used for that 32-key quarter, and per work item i the
-// pair (M_i, S_i) with  sum over the item's keys of 2^(z*c) = S_i * 2^M_i.
-// This kernel
-//   1. merges the pairs of the unit's items into bias_q = log2 D_q, the log2
-//      of query q's softmax denominator (merged in a fixed order);
-//   2. raw_j = sum_q e_qj * 2^(R - bias_q)   (every weight is <= 1);
-//   3. pooled_j = (sum_{t=-h..h} raw_{j+t}) / P with zeros outside [0, n),
+// reference its warp used for that 32-key quarter, and per query row
+// bias_q = log2 D_q, the log2 of its softmax denominator.  This kernel
+//   1. raw_j = sum_q e_qj * 2^(R - bias_q)   (every weight is <= 1);
+//   2. pooled_j = (sum_{t=-h..h} raw_{j+t}) / P with zeros outside [0, n),
 //      summed in a fixed order.
-// One CTA per chunk of 32-key quarters of one unit.  The unit's pairs, the
+// One CTA per chunk of 32-key quarters of one unit.  The unit's bias row, the
 // references of every quarter the chunk touches (the chunk plus an h-key
 // halo on each side) and the first exponent rows are requested together;
 // the weights 2^(R - bias_q) are then tabulated in shared memory and the
@@ -36,7 +33,6 @@ namespace {
 
 constexpr int kCombThreads = 256;
 constexpr int kLoadBatch = 4;  // 16-byte loads per batch (two batches in flight per thread)
-constexpr int kPairSlots = 4096;  // softmax pairs staged per round
 static_assert(kMaxQRows <= kCombThreads, "one thread per query row");
 
 __device__ __forceinline__ float dot8(const uint4 v, const float* w) {
@@ -62,7 +58,6 @@ __global__ void __launch_bounds__(kCombThreads)
     combine_kernel(const __grid_constant__ CombineParams p) {
   extern __shared__ __align__(16) float s_dyn[];  // weights [nqt][Nr] | raw [span]
   __shared__ float s_bias[kMaxQRows];
-  __shared__ float2 s_pairs[kPairSlots];
 
   const int tid = threadIdx.x;
   const WorkItem it = p.items[blockIdx.x];
@@ -89,10 +84,10 @@ __global__ void __launch_bounds__(kCombThreads)
   float* s_raw = s_dyn + nqt * Nr;
 
   for (int i = tid; i < span; i += kCombThreads) s_raw[i] = 0.f;
-  pdl_wait();  // pairs and tables come from the scoring kernel
+  pdl_wait();  // denominators and tables come from the scoring kernel
 
   // Everything below depends on three independent reads -- the unit's
-  // softmax pairs, the references of the quarters touched and the exponent
+  // denominators, the references of the quarters touched and the exponent
   // rows -- so all three are issued before any of them is waited on.
   const uint4* E4 = reinterpret_cast<const uint4*>(p.expo + it.eoff);
   const int f_lo = ea * cpr;
@@ -107,77 +102,21 @@ __global__ void __launch_bounds__(kCombThreads)
   };
   load_batch(f_lo, ev);
   // references (16-byte chunks: nqt * Nr is a multiple of 8 and the rows are
-  // 32-byte aligned) and softmax pairs arrive by asynchronous copies, all in
-  // flight together
+  // 32-byte aligned) and denominators arrive by asynchronous copies
   const float* R = p.refs + it.roff + static_cast<long long>(q0) * Nr;
   for (int i = 4 * tid; i < nqt * Nr; i += 4 * kCombThreads) cp_async16(smem_u32(s_w + i), R + i);
-  const int per = kPairSlots / N;  // items staged per round
-  const int ni0 = min(per, static_cast<int>(it.count));
-  auto stage_pairs = [&](int i0, int ni) {
-    for (int e = tid; e < ni * N; e += kCombThreads) {
-      const int ii = e / N;
-      const int q = e - ii * N;
-      cp_async8(smem_u32(s_pairs + e),
-                p.partials + static_cast<long long>(it.first + i0 + ii) * kMaxQRows + q);
-    }
-    cp_async_wait_all();
-  };
-  stage_pairs(0, ni0);
+  if (tid < N) cp_async4(smem_u32(s_bias + tid), p.bias + static_cast<long long>(it.first) * kMaxQRows + tid);
+  cp_async_wait_all();
   __syncthreads();
 
-  // 1. per-query log2 softmax denominators.  The item pairs are merged by
-  //    nm = 256 / N threads per query (thread t: query t % N, items
-  //    i = t / N (mod nm)), then the nm partial pairs in that order; units
-  //    with many items take several staging rounds.
-  {
-    const int nm = kCombThreads / N;
-    const int q = tid % N;
-    const int sub = tid / N;
-    float m = -INFINITY, z = 0.f;
-    auto merge = [&](float pm, float pz) {
-      if (pm == -INFINITY) return;
-      if (pm > m) {
-        z = fmaf(z, ex2_approx(m - pm), pz);
-        m = pm;
-      } else {
-        z = fmaf(pz, ex2_approx(pm - m), z);
-      }
-    };
-    for (int i0 = 0; i0 < it.count; i0 += per) {
-      const int ni = min(per, it.count - i0);
-      if (i0 > 0) {
-        __syncthreads();
-        stage_pairs(i0, ni);
-        __syncthreads();
-      }
-      if (sub < nm) {
-        for (int ii = sub; ii < ni; ii += nm) {
-          const float2 pr = s_pairs[ii * N + q];
-          merge(pr.x, pr.y);
-        }
-      }
-    }
-    __syncthreads();  // every round's pairs have been read
-    float2* part = s_pairs;  // [nm][N] partial pairs
-    if (sub < nm) part[sub * N + q] = make_float2(m, z);
-    __syncthreads();
-    if (tid < N) {
-      m = -INFINITY;
-      z = 0.f;
-      for (int j = 0; j < nm; ++j) merge(part[j * N + tid].x, part[j * N + tid].y);
-      s_bias[tid] = m + __log2f(z);
-    }
-  }
-  __syncthreads();
-
-  // 2. weights 2^(R - bias_q) of the quarters touched, in place
+  // weights 2^(R - bias_q) of the quarters touched, in place
   for (int i = tid; i < nqt * Nr; i += kCombThreads) {
     const int cc = i & (Nr - 1);
     s_w[i] = cc < N ? ex2_approx(s_w[i] - s_bias[cc]) : 0.f;
   }
   __syncthreads();
 
-  // 3. raw scores of the keys [ea, eb): one contiguous run of exponent rows,
+  // 1. raw scores of the keys [ea, eb): one contiguous run of exponent rows,
   //    the next batch in flight while the current one is reduced
   for (int f0 = f_lo; f0 < f_hi; f0 += kLoadBatch * kCombThreads) {
     uint4 nx[kLoadBatch];
@@ -213,7 +152,7 @@ __global__ void __launch_bounds__(kCombThreads)
     }
   }
 
-  // 4. pooling (and the raw scores, when asked for)
+  // 2. pooling (and the raw scores, when asked for)
   const long long soff = static_cast<long long>(g) * p.p_total + p.cu_prefix[s];
   const float fP = static_cast<float>(p.pool_width);
   for (int j = a + tid; j < b; j += kCombThreads) {

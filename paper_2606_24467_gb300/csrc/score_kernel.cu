@@ -341,9 +341,11 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
       // wait cannot tell phase k from phase k+2, so warpgroups sharing a
       // buffer could read it early.
       const int nwg = kWG < nbuf ? kWG : nbuf;
-      // The exponent and reference tables are reused: an earlier kernel of the
-      // stream may still read them, so wait for it before the first store.
-      pdl_wait();
+      // The exponent and reference tables and the softmax pairs are reused
+      // across calls on one workspace.  Their only reader, the combine kernel,
+      // triggers its dependents after its last read of them, so this grid
+      // (launched no earlier than that trigger) may overwrite them without
+      // waiting for the kernels before it.
 
       for (int i = wg; wg < nwg && i < ntiles; i += nwg) {
         const int b = i % nbuf;
@@ -482,15 +484,78 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
       // merge the epilogue warps' (R, sum) pairs per query into the item's pair
       named_bar_sync(kBarEpi, 32 * kNumEpiWarps);
       const int te = static_cast<int>(threadIdx.x) - kFirstEpiWarp * 32;
-      if (te < N && !*abort_flag) {
-        float m = kNegInf;
-        for (int w = 0; w < kNumEpiWarps; ++w) m = fmaxf(m, sRef[w * kMaxQRows + te]);
-        float z = 0.f;
-        for (int w = 0; w < kNumEpiWarps; ++w) {
-          const float rw = sRef[w * kMaxQRows + te];
-          if (rw != kNegInf) z += sAcc[w * kMaxQRows + te] * ex2_approx(rw - m);
+      // the first epilogue warp writes the item's pairs, makes them visible
+      // device-wide and takes the unit's ticket: the last CTA of the unit to
+      // get here (no waiting) merges the pairs of all the unit's items,
+      // split over 32*E / N threads per query, into bias_q = log2 D_q for
+      // the combine kernel, and resets the ticket
+      volatile int* last = abort_flag + 1;
+      if (te < 32) {
+        for (int q = te; q < N && !*abort_flag; q += 32) {
+          float m = kNegInf;
+          for (int w = 0; w < kNumEpiWarps; ++w) m = fmaxf(m, sRef[w * kMaxQRows + q]);
+          float z = 0.f;
+          for (int w = 0; w < kNumEpiWarps; ++w) {
+            const float rw = sRef[w * kMaxQRows + q];
+            if (rw != kNegInf) z += sAcc[w * kMaxQRows + q] * ex2_approx(rw - m);
+          }
+          p.partials[static_cast<long long>(blockIdx.x) * kMaxQRows + q] = make_float2(m, z);
         }
-        p.partials[static_cast<long long>(blockIdx.x) * kMaxQRows + te] = make_float2(m, z);
+        __threadfence();
+        __syncwarp();
+        if (te == 0)
+          *last = (!*abort_flag && atomicAdd(p.tickets + it.first, 1) == it.count - 1) ? 1 : 0;
+      }
+      named_bar_sync(kBarEpi, 32 * kNumEpiWarps);
+      if (*last) {
+        __threadfence();
+        const int nm = (32 * kNumEpiWarps) / N;
+        const int q = te % N;
+        const int sub = te / N;
+        float m = kNegInf, z = 0.f;
+        if (sub < nm) {
+          // eight pairs in flight per batch (L2 reads of the other CTAs' rows)
+          for (int i0 = sub; i0 < it.count; i0 += 8 * nm) {
+            float2 pr[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+              const int i = i0 + u * nm;
+              pr[u] = i < it.count
+                          ? __ldcg(p.partials + static_cast<long long>(it.first + i) * kMaxQRows + q)
+                          : make_float2(kNegInf, 0.f);
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+              if (pr[u].x == kNegInf) continue;
+              if (pr[u].x > m) {
+                z = fmaf(z, ex2_approx(m - pr[u].x), pr[u].y);
+                m = pr[u].x;
+              } else {
+                z = fmaf(pr[u].y, ex2_approx(pr[u].x - m), z);
+              }
+            }
+          }
+          sRef[sub * N + q] = m;
+          sAcc[sub * N + q] = z;
+        }
+        named_bar_sync(kBarEpi, 32 * kNumEpiWarps);
+        if (te < N) {
+          m = kNegInf;
+          z = 0.f;
+          for (int j = 0; j < nm; ++j) {
+            const float pm = sRef[j * N + te];
+            const float pz = sAcc[j * N + te];
+            if (pm == kNegInf) continue;
+            if (pm > m) {
+              z = fmaf(z, ex2_approx(m - pm), pz);
+              m = pm;
+            } else {
+              z = fmaf(pz, ex2_approx(pm - m), z);
+            }
+          }
+          p.bias[static_cast<long long>(it.first) * kMaxQRows + te] = m + __log2f(z);
+        }
+        if (te == 0) p.tickets[it.first] = 0;
       }
     }
   }
@@ -498,14 +563,16 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
   // ------------------------------------------------------------ teardown
   // The next kernel is launched once every CTA has reached this point, so its
   // CTAs spread over all SMs instead of packing the ones that freed first.
+  // The tensor memory is released before the wait for the kernels before
+  // this one (completion of this grid then implies theirs).
   pdl_launch_dependents();
-  pdl_wait();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tbase, tcols);
   }
+  pdl_wait();
 }
 
 }  // namespace

@@ -435,31 +435,35 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
 // the K/V rows copied -- with three cluster barriers instead of one per radix
 // pass.  One cluster of C <= 16 CTAs per unit; CTA r owns the contiguous
 // slice [r*S, (r+1)*S) of the unit's prefix positions.
-//   1. The slice's pooled scores go to shared memory; each CTA sends 64
+//   1. The slice's pooled scores go to shared memory; each CTA sends 256 / C
 //      evenly spaced scores of its slice to every CTA of the cluster.
 //   2. Every CTA takes the same lower bound lo for the k-th largest score:
-//      the r-th largest sample, r a few standard deviations above the
-//      expected number k * (samples / n) of samples above the k-th score.
+//      the r-th largest sample (found by counting, for every sample, the
+//      samples above it), r a few standard deviations above the expected
+//      number k * (samples / n) of samples above the k-th score.
 //   3. Each CTA lists its keys >= lo in position order and sends the count.
 //      When between k and kScCandCap keys reach lo (the usual case), every
 //      CTA reads all lists (position order across the cluster), finds the
-//      k-th largest key tau and how many keys equal to it are kept, and
-//      writes its own selected positions at offsets counted in that list.
+//      k-th largest key tau and how many keys equal to it are kept (radix
+//      passes over min(key - lo, 2^16 - 1), which resolve tau whenever it is
+//      below lo + 2^16 - 1, else over the keys themselves), and writes its
+//      own selected positions at offsets counted in that list.
 //      Otherwise every CTA runs the same search over all of the unit's
 //      scores (read from global memory) and counts from there.
 //   4. The last CTA appends the window; every CTA copies its own K/V rows.
 // Pooled scores are >= 0, so their fp32 bit patterns order like the values.
 constexpr int kScThreads = 256;
 constexpr int kScWarps = kScThreads / 32;
-constexpr int kScSamples = 64;    // samples per CTA
+constexpr int kScSampleTotal = 256;  // samples per unit (kScSampleTotal / C per CTA)
 constexpr int kScMaxC = 16;       // CTAs per cluster
 constexpr int kScCandCap = 4096;  // candidates per unit
-static_assert(kScThreads == 256, "one thread per radix bin");
+static_assert(kScThreads == 256 && kScSampleTotal == kScThreads, "one thread per radix bin and per sample");
 
 struct ScShared {
-  uint32_t samp[kScMaxC * kScSamples];  // written by every CTA of the cluster
+  int samp[kScSampleTotal];  // keys as int (>= 0); -1 = no sample; written by every CTA
   int samp_cnt[kScMaxC];
   int cand_cnt[kScMaxC];
+  int cand_off[kScMaxC + 1];
   int ovf[kScMaxC];
   uint32_t ckey[kScCandCap];  // own candidates, position order
   int cpos[kScCandCap];
@@ -470,11 +474,13 @@ struct ScShared {
   uint32_t key_or[2], key_and[2];  // one pair per search
   int red[2][2];                    // one pair of sums per use
   int red0;
+  uint32_t lo;
 };
 
 // Zero state the searches below expect (before the kernel's first barrier).
-__device__ __forceinline__ void sc_init_shared(ScShared& sh) {
+__device__ __forceinline__ void sc_init_shared(ScShared& sh, int sampled_slots) {
   const int tid = threadIdx.x;
+  if (tid >= sampled_slots && tid < kScSampleTotal) sh.samp[tid] = -1;  // slots no CTA fills
   for (int i = tid; i < 2 * 256; i += kScThreads) sh.hist[i >> 8][i & 255] = 0u;
   if (tid < 2) {
     sh.key_or[tid] = 0u;
@@ -674,46 +680,61 @@ __global__ void __launch_bounds__(kScThreads)
   }
 
   // 1. slice -> shared memory; samples to every CTA
-  sc_init_shared(sh);
+  const int per_cta = kScSampleTotal / C;
+  sc_init_shared(sh, C * per_cta);
   int pc = 0;  // radix passes run so far (histogram rotation)
   for (int i = tid; i < len; i += kScThreads) cp_async4(smem_u32(s_keys + i), pooled + lo_c + i);
   cp_async_wait_all();
   __syncthreads();
   auto key_at = [&](int i) { return __float_as_uint(s_keys[i]); };
-  const int ns_c = min(kScSamples, len);
+  const int ns_c = min(per_cta, len);
   cluster_wait();  // every CTA has started
-  if (tid < ns_c) {
-    const uint32_t v = key_at(static_cast<int>((static_cast<long long>(tid) * len) / ns_c));
-    for (int t = 0; t < C; ++t) *cluster.map_shared_rank(&sh.samp[cr * kScSamples + tid], t) = v;
+  if (tid < per_cta) {
+    const int v = tid < ns_c
+                      ? static_cast<int>(key_at(static_cast<int>((static_cast<long long>(tid) * len) / ns_c)))
+                      : -1;
+    for (int t = 0; t < C; ++t) *cluster.map_shared_rank(&sh.samp[cr * per_cta + tid], t) = v;
   }
   if (tid < C) *cluster.map_shared_rank(&sh.samp_cnt[cr], tid) = ns_c;
   cluster_arrive_release();
   cluster_wait();
 
-  // 2. lower bound from the samples
+  // 2. lower bound from the samples: the rs-th largest, by counting for each
+  //    sample the samples above it and equal to it
   int nsamp = 0;
   for (int c = 0; c < C; ++c) nsamp += sh.samp_cnt[c];
   const float mu = static_cast<float>(k) * static_cast<float>(nsamp) / static_cast<float>(n);
   const int rs = min(nsamp, static_cast<int>(ceilf(mu + 3.f * sqrtf(mu))) + 2);
-  int rem_s;
-  const uint32_t lo = cta_kth_largest(
-      [&](const auto& f) {
-        for (int j0 = 0; j0 < C * kScSamples; j0 += kScThreads) {
-          const int j = j0 + tid;
-          const bool v = j < C * kScSamples && (j % kScSamples) < sh.samp_cnt[j / kScSamples];
-          f(v ? sh.samp[j] : 0u, v);
-        }
-      },
-      rs, sh, 0, pc, &rem_s);
+  {
+    const int v = sh.samp[tid];  // kScThreads == kScSampleTotal: one sample per thread
+    const int4* s4 = reinterpret_cast<const int4*>(sh.samp);
+    int gt = 0, eq = 0;
+#pragma unroll 8
+    for (int j = 0; j < kScSampleTotal / 4; ++j) {  // empty slots (-1) never count
+      const int4 x = s4[j];
+      gt += (x.x > v) + (x.y > v) + (x.z > v) + (x.w > v);
+      eq += (x.x == v) + (x.y == v) + (x.z == v) + (x.w == v);
+    }
+    if (v >= 0 && gt < rs && rs <= gt + eq) sh.lo = static_cast<uint32_t>(v);  // equal samples agree
+  }
+  __syncthreads();
+  const uint32_t lo = sh.lo;
 
   // 3. own candidates (keys >= lo) in position order; counts to every CTA
   const int seg = ((len + kScThreads - 1) / kScThreads) * 32;  // positions per warp
   const int wlo = min(len, warp * seg);
   const int whi = min(len, wlo + seg);
   int wc = 0;
-  for (int b0 = wlo; b0 < whi; b0 += 32) {
-    const int i = b0 + lane;
-    wc += __popc(__ballot_sync(0xffffffffu, i < whi && key_at(i) >= lo));
+  for (int b0 = wlo; b0 < whi; b0 += 8 * 32) {  // eight rows of 32 keys per step
+    uint32_t kk[8];
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+      const int i = b0 + 32 * r + lane;
+      kk[r] = i < whi ? key_at(i) : 0u;
+    }
+#pragma unroll
+    for (int r = 0; r < 8; ++r)
+      wc += __popc(__ballot_sync(0xffffffffu, b0 + 32 * r + lane < whi && kk[r] >= lo));
   }
   if (lane == 0) sh.wcnt[warp] = wc;
   __syncthreads();
@@ -727,16 +748,25 @@ __global__ void __launch_bounds__(kScThreads)
   const int own = sh.red0;
   {
     int o = sh.wbase[warp];
-    for (int b0 = wlo; b0 < whi; b0 += 32) {
-      const int i = b0 + lane;
-      const bool c = i < whi && key_at(i) >= lo;
-      const uint32_t mm = __ballot_sync(0xffffffffu, c);
-      const int slot = o + __popc(mm & lanemask_lt(lane));
-      if (c && slot < kScCandCap) {
-        sh.ckey[slot] = key_at(i);
-        sh.cpos[slot] = lo_c + i;
+    for (int b0 = wlo; b0 < whi; b0 += 8 * 32) {
+      uint32_t kk[8];
+#pragma unroll
+      for (int r = 0; r < 8; ++r) {
+        const int i = b0 + 32 * r + lane;
+        kk[r] = i < whi ? key_at(i) : 0u;
       }
-      o += __popc(mm);
+#pragma unroll
+      for (int r = 0; r < 8; ++r) {
+        const int i = b0 + 32 * r + lane;
+        const bool c = i < whi && kk[r] >= lo;
+        const uint32_t mm = __ballot_sync(0xffffffffu, c);
+        const int slot = o + __popc(mm & lanemask_lt(lane));
+        if (c && slot < kScCandCap) {
+          sh.ckey[slot] = kk[r];
+          sh.cpos[slot] = lo_c + i;
+        }
+        o += __popc(mm);
+      }
     }
   }
   if (tid < C) {
@@ -760,22 +790,51 @@ __global__ void __launch_bounds__(kScThreads)
   int need_eq, gt_before, eq_before;
   if (fast) {
     // every CTA's list, concatenated in cluster (= position) order
-    for (int j = tid; j < total; j += kScThreads) {
-      int c = 0, off = 0;
-      while (off + sh.cand_cnt[c] <= j) off += sh.cand_cnt[c++];
-      sh.all[j] = *cluster.map_shared_rank(&sh.ckey[j - off], c);
+    if (warp == 0) {
+      const int cc = lane < C ? sh.cand_cnt[lane] : 0;
+      const int ex = warp_exclusive_scan(cc, lane);
+      if (lane <= C) sh.cand_off[lane] = ex;
     }
     __syncthreads();
+    constexpr int kPer = kScCandCap / kScThreads;  // list entries per thread, at most
+    uint32_t kv[kPer];
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+      const int j = i * kScThreads + tid;
+      kv[i] = 0u;
+      if (j < total) {
+        int c = 0;
+#pragma unroll
+        for (int q = 1; q < kScMaxC; ++q) c += (q < C && j >= sh.cand_off[q]) ? 1 : 0;
+        kv[i] = *cluster.map_shared_rank(&sh.ckey[j - sh.cand_off[c]], c);
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < kPer; ++i)
+      if (i * kScThreads + tid < total) sh.all[i * kScThreads + tid] = kv[i];
+    __syncthreads();
     cluster_arrive_release();  // done reading the other CTAs' shared memory
-    tau = cta_kth_largest(
+    // offsets above lo, clamped to 16 bits: at most two passes
+    constexpr uint32_t kClamp = 0xFFFFu;
+    const uint32_t td = cta_kth_largest(
         [&](const auto& f) {
-          for (int j0 = 0; j0 < total; j0 += kScThreads) {
-            const int j = j0 + tid;
-            f(j < total ? sh.all[j] : 0u, j < total);
-          }
+#pragma unroll
+          for (int i = 0; i < kPer; ++i)
+            if (i * kScThreads < total) f(min(kv[i] - lo, kClamp), i * kScThreads + tid < total);
         },
-        k, sh, 1, pc, &need_eq);
+        k, sh, 0, pc, &need_eq);
+    tau = lo + td;
+    if (td == kClamp) {  // tau at or above the clamp: the keys themselves
+      tau = cta_kth_largest(
+          [&](const auto& f) {
+#pragma unroll
+            for (int i = 0; i < kPer; ++i)
+              if (i * kScThreads < total) f(kv[i], i * kScThreads + tid < total);
+          },
+          k, sh, 1, pc, &need_eq);
+    }
     int a = 0, b = 0;
+#pragma unroll 4
     for (int j = tid; j < before; j += kScThreads) {
       a += sh.all[j] > tau ? 1 : 0;
       b += sh.all[j] == tau ? 1 : 0;
