@@ -57,7 +57,7 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-lse", action="store_true",
                     help="skip the given-LSE (log-sum-exp supplied) measurement")
-    ap.add_argument("--streams", type=int, default=3,
+    ap.add_argument("--streams", type=int, default=4,
                     help="layers in flight: layer l runs on stream l %% S with its own workspace")
     return ap.parse_args()
 

@@ -25,6 +25,7 @@
 #include <cuda_runtime.h>
 
 #include "ckv_device.cuh"
+#include "select_common.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -36,18 +37,6 @@ constexpr int kSelThreads = 512;
 constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kBins = 256;
 constexpr int kSelStaticSmem = 2 * kBins * 4 + kBins * 4 + 8 * kSelWarps * 4 + 256;
-
-__device__ __forceinline__ uint32_t lanemask_lt(int lane) { return (1u << lane) - 1u; }
-
-__device__ __forceinline__ int warp_exclusive_scan(int v, int lane) {
-  int x = v;
-#pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, x, off);
-    if (lane >= off) x += y;
-  }
-  return x - v;
-}
 
 // Cluster-wide barrier.  The .aligned forms require every thread of a warp
 // to execute them together, so the warp is reconverged first.
@@ -73,47 +62,6 @@ template <bool kCluster, class T>
 __device__ __forceinline__ T* unit_rank_ptr(T* ptr, int rank) {
   if (kCluster) return cg::this_cluster().map_shared_rank(ptr, rank);
   return ptr;
-}
-
-// The whole CTA copies the K and V rows of `count` tokens to consecutive
-// output rows: token i is out[first + i] (a position in the sequence) and goes
-// to output row out0 + first + i.  Each thread moves 16-byte chunks, issuing
-// a batch of loads before the matching stores.
-template <int kThreads = kSelThreads>
-__device__ __forceinline__ void copy_kv_rows(const SelectParams& p, int seq0, int g,
-                                             const int32_t* out, int out0, int first, int count) {
-  constexpr int kChunks = 2 * kHeadDim * 2 / 16;  // 16 K + 16 V chunks per token
-  constexpr int kBatch = 4;
-  const int total = count * kChunks;
-  for (int base = 0; base < total; base += kBatch * kThreads) {
-    uint4 v[kBatch];
-    long long dst[kBatch];
-    bool is_v[kBatch];
-#pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
-      const int e = base + u * kThreads + static_cast<int>(threadIdx.x);
-      dst[u] = -1;
-      if (e < total) {
-        const int i = e / kChunks;
-        const int ch = e - i * kChunks;
-        const int tok = out[first + i];
-        is_v[u] = ch >= kChunks / 2;
-        const int part = ch & (kChunks / 2 - 1);
-        const long long src = static_cast<long long>(seq0 + tok) * p.tok_stride_v16 +
-                              static_cast<long long>(g) * p.head_stride_v16 + part;
-        v[u] = __ldg((is_v[u] ? p.v : p.k) + src);
-        // one row per (token, group), or per token of this group when the
-        // output is packed group-major (head-level budgets)
-        dst[u] = (p.head_budgets ? static_cast<long long>(out0 + first + i)
-                                 : static_cast<long long>(out0 + first + i) * p.num_kv_heads + g) *
-                     (kHeadDim * 2 / 16) + part;
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
-      if (dst[u] >= 0) (is_v[u] ? p.v_out : p.k_out)[dst[u]] = v[u];
-    }
-  }
 }
 
 template <bool kCluster>
@@ -255,7 +203,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
       for (int rr = 0; rr < nrows; ++rr) out[rr * ostride + i] = i;
     if (p.gather && a1 > a0) {
       __syncthreads();  // the indices written above are read back by the copy
-      for (int rr = 0; rr < nrows; ++rr) copy_kv_rows(p, seq0, g + rr, out, out0, a0, a1 - a0);
+      for (int rr = 0; rr < nrows; ++rr) copy_kv_rows<kSelThreads>(p, seq0, g + rr, out, out0, a0, a1 - a0);
     }
     return;  // uniform over the cluster: no cluster barrier is pending
   }
@@ -267,7 +215,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   if (k == 0) {  // window only (uniform over the cluster)
     if (p.gather && crank == C - 1) {
       __syncthreads();
-      for (int rr = 0; rr < nrows; ++rr) copy_kv_rows(p, seq0, g + rr, out, out0, k, W);
+      for (int rr = 0; rr < nrows; ++rr) copy_kv_rows<kSelThreads>(p, seq0, g + rr, out, out0, k, W);
     }
     return;
   }
@@ -421,8 +369,8 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
     const int cta_first = s_cta_first;
     const int cta_count = min(k - cta_first, s_cta_count);
     for (int rr = 0; rr < nrows; ++rr) {
-      if (cta_count > 0) copy_kv_rows(p, seq0, g + rr, out, out0, cta_first, cta_count);
-      if (crank == C - 1) copy_kv_rows(p, seq0, g + rr, out, out0, k, W);
+      if (cta_count > 0) copy_kv_rows<kSelThreads>(p, seq0, g + rr, out, out0, cta_first, cta_count);
+      if (crank == C - 1) copy_kv_rows<kSelThreads>(p, seq0, g + rr, out, out0, k, W);
     }
   }
 }
@@ -468,11 +416,10 @@ struct ScShared {
   uint32_t ckey[kScCandCap];  // own candidates, position order
   int cpos[kScCandCap];
   uint32_t all[kScCandCap];   // every CTA's candidates, position order
-  uint32_t hist[4][256];      // radix histograms, used in rotation
+  RadixShared rs;
   int wcnt[kScWarps];
   int wbase[kScWarps];
-  uint32_t key_or[2], key_and[2];  // one pair per search
-  int red[2][2];                    // one pair of sums per use
+  int red[2][2];              // one pair of sums per use
   int red0;
   uint32_t lo;
 };
@@ -481,10 +428,8 @@ struct ScShared {
 __device__ __forceinline__ void sc_init_shared(ScShared& sh, int sampled_slots) {
   const int tid = threadIdx.x;
   if (tid >= sampled_slots && tid < kScSampleTotal) sh.samp[tid] = -1;  // slots no CTA fills
-  for (int i = tid; i < 2 * 256; i += kScThreads) sh.hist[i >> 8][i & 255] = 0u;
+  radix_init(sh.rs);
   if (tid < 2) {
-    sh.key_or[tid] = 0u;
-    sh.key_and[tid] = 0xFFFFFFFFu;
     sh.red[tid][0] = 0;
     sh.red[tid][1] = 0;
   }
@@ -501,113 +446,6 @@ __device__ __forceinline__ void cluster_arrive_release() {
 __device__ __forceinline__ void cluster_wait() {
   __syncwarp();
   asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-
-// Whole warp: the bin of `h[0..255]` (counts; higher bin = larger keys)
-// holding the rem-th largest key, and the count of keys in the bins above it
-// (every lane receives both).
-__device__ __forceinline__ void warp_pick_bin256(const uint32_t* h, int rem, int lane, int* bin,
-                                                 int* above_out) {
-  uint32_t c[8];
-  uint32_t cnt = 0u;
-#pragma unroll
-  for (int b = 0; b < 8; ++b) {
-    c[b] = h[lane * 8 + b];
-    cnt += c[b];
-  }
-  uint32_t suf = cnt;  // inclusive suffix sum over lanes
-#pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    const uint32_t y = __shfl_down_sync(0xffffffffu, suf, off);
-    if (lane + off < 32) suf += y;
-  }
-  const uint32_t ok = __ballot_sync(0xffffffffu, suf >= static_cast<uint32_t>(rem));
-  const int top = ok ? 31 - __clz(ok) : 0;
-  uint32_t above = __shfl_sync(0xffffffffu, suf - cnt, top);  // keys above lane top's bins
-  int bsel = top * 8;
-  if (lane == top) {
-    for (int b = 7; b >= 0; --b) {
-      if (above + c[b] >= static_cast<uint32_t>(rem)) {
-        bsel = top * 8 + b;
-        break;
-      }
-      above += c[b];
-    }
-  }
-  *bin = __shfl_sync(0xffffffffu, bsel, top);
-  *above_out = static_cast<int>(__shfl_sync(0xffffffffu, above, top));
-}
-
-// CTA-wide: the r-th largest (1 <= r <= number of keys) of the keys that
-// `visit` presents (visit(f) calls f(key, valid) equally often on every lane
-// of a warp).  Returns the key tau; *rem = how many keys equal to tau are
-// among the r largest.  The radix passes (8 bits each) start at the highest
-// bit in which the keys differ; each pass has one barrier: pass number pc
-// counts into hist[pc % 4] (zero on entry, as is hist[(pc + 1) % 4]) while
-// hist[(pc + 2) % 4], last read two passes earlier, is cleared, and every warp
-// then picks the bin itself.  `slot` selects this search's key_or / key_and.
-template <class Visit>
-__device__ uint32_t cta_kth_largest(const Visit& visit, int r, ScShared& sh, int slot, int& pc,
-                                    int* rem) {
-  const int tid = threadIdx.x;
-  const int lane = tid & 31;
-  uint32_t ko = 0u, ka = 0xFFFFFFFFu;
-  visit([&](uint32_t key, bool valid) {
-    if (valid) {
-      ko |= key;
-      ka &= key;
-    }
-  });
-  ko = __reduce_or_sync(0xffffffffu, ko);
-  ka = __reduce_and_sync(0xffffffffu, ka);
-  if (lane == 0) {
-    atomicOr(&sh.key_or[slot], ko);
-    atomicAnd(&sh.key_and[slot], ka);
-  }
-  __syncthreads();
-  const uint32_t diff = sh.key_or[slot] ^ sh.key_and[slot];
-  const uint32_t kand = sh.key_and[slot];
-  int remaining = r;
-  if (diff == 0u) {  // all keys equal
-    *rem = remaining;
-    return kand;
-  }
-  int hb = 31 - __clz(diff);
-  uint32_t pmask = hb == 31 ? 0u : ~((2u << hb) - 1u);
-  uint32_t prefix = kand & pmask;
-#pragma unroll 1
-  while (hb >= 0) {
-    const int width = min(8, hb + 1);
-    const int shf = hb + 1 - width;
-    const uint32_t fm = (1u << width) - 1u;
-    uint32_t* h = sh.hist[pc & 3];
-    visit([&](uint32_t key, bool valid) {
-      const bool m = valid && (key & pmask) == prefix;
-      const uint32_t act = __ballot_sync(0xffffffffu, m);
-      if (!act) return;
-      const uint32_t bin = (key >> shf) & fm;
-      const int leader = __ffs(act) - 1;
-      const uint32_t lb = __shfl_sync(0xffffffffu, bin, leader);
-      // one add per warp when its keys share the bin (dense scores), else
-      // one per key
-      if (__all_sync(0xffffffffu, !m || bin == lb)) {
-        if (lane == leader) atomicAdd(&h[lb], static_cast<uint32_t>(__popc(act)));
-      } else if (m) {
-        atomicAdd(&h[bin], 1u);
-      }
-    });
-    sh.hist[(pc + 2) & 3][tid] = 0u;  // kScThreads == 256 bins
-    __syncthreads();
-    int bin, above;
-    warp_pick_bin256(h, remaining, lane, &bin, &above);
-    remaining -= above;
-    prefix |= static_cast<uint32_t>(bin) << shf;
-    pmask |= fm << shf;
-    hb = shf - 1;
-    ++pc;
-  }
-  *rem = remaining;
-  return prefix;
 }
 
 // CTA-wide sums of two ints into sh.red[slot] (zero on entry; every thread
@@ -822,7 +660,7 @@ __global__ void __launch_bounds__(kScThreads)
           for (int i = 0; i < kPer; ++i)
             if (i * kScThreads < total) f(min(kv[i] - lo, kClamp), i * kScThreads + tid < total);
         },
-        k, sh, 0, pc, &need_eq);
+        k, sh.rs, 0, pc, &need_eq);
     tau = lo + td;
     if (td == kClamp) {  // tau at or above the clamp: the keys themselves
       tau = cta_kth_largest(
@@ -831,7 +669,7 @@ __global__ void __launch_bounds__(kScThreads)
             for (int i = 0; i < kPer; ++i)
               if (i * kScThreads < total) f(kv[i], i * kScThreads + tid < total);
           },
-          k, sh, 1, pc, &need_eq);
+          k, sh.rs, 1, pc, &need_eq);
     }
     int a = 0, b = 0;
 #pragma unroll 4
@@ -849,7 +687,7 @@ __global__ void __launch_bounds__(kScThreads)
             f(j < n ? __ldg(gkeys + j) : 0u, j < n);
           }
         },
-        k, sh, 1, pc, &need_eq);
+        k, sh.rs, 1, pc, &need_eq);
     int a = 0, b = 0;
     for (int j = tid; j < lo_c; j += kScThreads) {
       const uint32_t key = __ldg(gkeys + j);
