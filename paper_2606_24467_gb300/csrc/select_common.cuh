@@ -27,9 +27,11 @@ __device__ __forceinline__ int warp_exclusive_scan(int v, int lane) {
 // output rows: token i is out[first + i] (a position in the sequence) and goes
 // to output row out0 + first + i.  Each thread moves 16-byte chunks, issuing
 // a batch of loads before the matching stores.
+// Kept out of line (one copy per instantiation): the selection kernels run
+// once per SM and are bound by instruction fetch.
 template <int kThreads, class Params>
-__device__ __forceinline__ void copy_kv_rows(const Params& p, int seq0, int g, const int32_t* out,
-                                             int out0, int first, int count) {
+__device__ __noinline__ void copy_kv_rows(const Params& p, int seq0, int g, const int32_t* out,
+                                          int out0, int first, int count) {
   constexpr int kChunks = 2 * kHeadDim * 2 / 16;  // 16 K + 16 V chunks per token
   constexpr int kBatch = 4;
   const int total = count * kChunks;
@@ -116,26 +118,33 @@ __device__ __forceinline__ void warp_pick_bin256(const uint32_t* h, int rem, int
   *above_out = static_cast<int>(__shfl_sync(0xffffffffu, above, top));
 }
 
-// CTA-wide: the r-th largest (1 <= r <= number of keys) of the keys that
-// `visit` presents (visit(f) calls f(key, valid) equally often on every lane
-// of a warp).  Returns the key tau; *rem = how many keys equal to tau are
-// among the r largest.  The radix passes (8 bits each) start at the highest
-// bit in which the keys differ; each pass has one barrier: pass number pc
-// counts into hist[pc % 4] (zero on entry, as is hist[(pc + 1) % 4]) while
+// CTA-wide (256 threads): the r-th largest (1 <= r <= count) of the keys
+// min(keys[j] - sub, clamp), j < count, where `keys` may point to shared or
+// global memory (keys[j] >= sub).  Returns that value tau; *rem = how many of
+// the count keys equal tau among the r largest (the caller takes those in
+// position order).  Radix passes of 8 bits start at the highest bit in which
+// the keys differ; each pass has one barrier: pass number pc counts into
+// hist[pc % 4] (zero on entry, as is hist[(pc + 1) % 4]) while
 // hist[(pc + 2) % 4], last read two passes earlier, is cleared, and every warp
-// then picks the bin itself.  `slot` selects this search's key_or / key_and.
-template <class Visit>
-__device__ uint32_t cta_kth_largest(const Visit& visit, int r, RadixShared& sh, int slot, int& pc,
-                                    int* rem) {
+// then picks the bin itself.  `slot` selects this search's key_or / key_and
+// (zero / all ones on entry).  Kept out of line: the kernels that call it run
+// once per SM, so code size (instruction fetch) matters more than inlining.
+__device__ __noinline__ uint32_t cta_kth_largest(const uint32_t* keys, int count, uint32_t sub,
+                                                 uint32_t clamp, int r, RadixShared& sh, int slot,
+                                                 int& pc, int* rem) {
   const int tid = threadIdx.x;
   const int lane = tid & 31;
+  const int iters = (count + 255) >> 8;  // warp-uniform trip count
   uint32_t ko = 0u, ka = 0xFFFFFFFFu;
-  visit([&](uint32_t key, bool valid) {
-    if (valid) {
+#pragma unroll 4
+  for (int i = 0; i < iters; ++i) {
+    const int j = (i << 8) + tid;
+    if (j < count) {
+      const uint32_t key = min(keys[j] - sub, clamp);
       ko |= key;
       ka &= key;
     }
-  });
+  }
   ko = __reduce_or_sync(0xffffffffu, ko);
   ka = __reduce_and_sync(0xffffffffu, ka);
   if (lane == 0) {
@@ -159,10 +168,13 @@ __device__ uint32_t cta_kth_largest(const Visit& visit, int r, RadixShared& sh, 
     const int shf = hb + 1 - width;
     const uint32_t fm = (1u << width) - 1u;
     uint32_t* h = sh.hist[pc & 3];
-    visit([&](uint32_t key, bool valid) {
-      const bool m = valid && (key & pmask) == prefix;
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i) {
+      const int j = (i << 8) + tid;
+      const uint32_t key = j < count ? min(keys[j] - sub, clamp) : 0u;
+      const bool m = j < count && (key & pmask) == prefix;
       const uint32_t act = __ballot_sync(0xffffffffu, m);
-      if (!act) return;
+      if (!act) continue;
       const uint32_t bin = (key >> shf) & fm;
       const int leader = __ffs(act) - 1;
       const uint32_t lb = __shfl_sync(0xffffffffu, bin, leader);
@@ -173,7 +185,7 @@ __device__ uint32_t cta_kth_largest(const Visit& visit, int r, RadixShared& sh, 
       } else if (m) {
         atomicAdd(&h[bin], 1u);
       }
-    });
+    }
     sh.hist[(pc + 2) & 3][tid] = 0u;  // one thread per bin (256 threads)
     __syncthreads();
     int bin, above;

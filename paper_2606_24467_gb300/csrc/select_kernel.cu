@@ -563,16 +563,10 @@ __global__ void __launch_bounds__(kScThreads)
   const int wlo = min(len, warp * seg);
   const int whi = min(len, wlo + seg);
   int wc = 0;
-  for (int b0 = wlo; b0 < whi; b0 += 8 * 32) {  // eight rows of 32 keys per step
-    uint32_t kk[8];
-#pragma unroll
-    for (int r = 0; r < 8; ++r) {
-      const int i = b0 + 32 * r + lane;
-      kk[r] = i < whi ? key_at(i) : 0u;
-    }
-#pragma unroll
-    for (int r = 0; r < 8; ++r)
-      wc += __popc(__ballot_sync(0xffffffffu, b0 + 32 * r + lane < whi && kk[r] >= lo));
+#pragma unroll 4
+  for (int b0 = wlo; b0 < whi; b0 += 32) {
+    const int i = b0 + lane;
+    wc += __popc(__ballot_sync(0xffffffffu, i < whi && key_at(i) >= lo));
   }
   if (lane == 0) sh.wcnt[warp] = wc;
   __syncthreads();
@@ -586,25 +580,18 @@ __global__ void __launch_bounds__(kScThreads)
   const int own = sh.red0;
   {
     int o = sh.wbase[warp];
-    for (int b0 = wlo; b0 < whi; b0 += 8 * 32) {
-      uint32_t kk[8];
-#pragma unroll
-      for (int r = 0; r < 8; ++r) {
-        const int i = b0 + 32 * r + lane;
-        kk[r] = i < whi ? key_at(i) : 0u;
+#pragma unroll 2
+    for (int b0 = wlo; b0 < whi; b0 += 32) {
+      const int i = b0 + lane;
+      const uint32_t key = i < whi ? key_at(i) : 0u;
+      const bool c = i < whi && key >= lo;
+      const uint32_t mm = __ballot_sync(0xffffffffu, c);
+      const int slot = o + __popc(mm & lanemask_lt(lane));
+      if (c && slot < kScCandCap) {
+        sh.ckey[slot] = key;
+        sh.cpos[slot] = lo_c + i;
       }
-#pragma unroll
-      for (int r = 0; r < 8; ++r) {
-        const int i = b0 + 32 * r + lane;
-        const bool c = i < whi && kk[r] >= lo;
-        const uint32_t mm = __ballot_sync(0xffffffffu, c);
-        const int slot = o + __popc(mm & lanemask_lt(lane));
-        if (c && slot < kScCandCap) {
-          sh.ckey[slot] = kk[r];
-          sh.cpos[slot] = lo_c + i;
-        }
-        o += __popc(mm);
-      }
+      o += __popc(mm);
     }
   }
   if (tid < C) {
@@ -634,43 +621,20 @@ __global__ void __launch_bounds__(kScThreads)
       if (lane <= C) sh.cand_off[lane] = ex;
     }
     __syncthreads();
-    constexpr int kPer = kScCandCap / kScThreads;  // list entries per thread, at most
-    uint32_t kv[kPer];
-#pragma unroll
-    for (int i = 0; i < kPer; ++i) {
-      const int j = i * kScThreads + tid;
-      kv[i] = 0u;
-      if (j < total) {
-        int c = 0;
-#pragma unroll
-        for (int q = 1; q < kScMaxC; ++q) c += (q < C && j >= sh.cand_off[q]) ? 1 : 0;
-        kv[i] = *cluster.map_shared_rank(&sh.ckey[j - sh.cand_off[c]], c);
-      }
+#pragma unroll 4
+    for (int j = tid; j < total; j += kScThreads) {
+      int c = 0;
+      for (int q = 1; q < C; ++q) c += j >= sh.cand_off[q] ? 1 : 0;
+      sh.all[j] = *cluster.map_shared_rank(&sh.ckey[j - sh.cand_off[c]], c);
     }
-#pragma unroll
-    for (int i = 0; i < kPer; ++i)
-      if (i * kScThreads + tid < total) sh.all[i * kScThreads + tid] = kv[i];
     __syncthreads();
     cluster_arrive_release();  // done reading the other CTAs' shared memory
     // offsets above lo, clamped to 16 bits: at most two passes
     constexpr uint32_t kClamp = 0xFFFFu;
-    const uint32_t td = cta_kth_largest(
-        [&](const auto& f) {
-#pragma unroll
-          for (int i = 0; i < kPer; ++i)
-            if (i * kScThreads < total) f(min(kv[i] - lo, kClamp), i * kScThreads + tid < total);
-        },
-        k, sh.rs, 0, pc, &need_eq);
+    const uint32_t td = cta_kth_largest(sh.all, total, lo, kClamp, k, sh.rs, 0, pc, &need_eq);
     tau = lo + td;
-    if (td == kClamp) {  // tau at or above the clamp: the keys themselves
-      tau = cta_kth_largest(
-          [&](const auto& f) {
-#pragma unroll
-            for (int i = 0; i < kPer; ++i)
-              if (i * kScThreads < total) f(kv[i], i * kScThreads + tid < total);
-          },
-          k, sh.rs, 1, pc, &need_eq);
-    }
+    if (td == kClamp)  // tau at or above the clamp: the keys themselves
+      tau = cta_kth_largest(sh.all, total, 0u, 0xFFFFFFFFu, k, sh.rs, 1, pc, &need_eq);
     int a = 0, b = 0;
 #pragma unroll 4
     for (int j = tid; j < before; j += kScThreads) {
@@ -680,14 +644,7 @@ __global__ void __launch_bounds__(kScThreads)
     cta_sum2(a, b, sh, 0, &gt_before, &eq_before);
   } else {
     cluster_arrive_release();
-    tau = cta_kth_largest(
-        [&](const auto& f) {
-          for (int j0 = 0; j0 < n; j0 += kScThreads) {
-            const int j = j0 + tid;
-            f(j < n ? __ldg(gkeys + j) : 0u, j < n);
-          }
-        },
-        k, sh.rs, 1, pc, &need_eq);
+    tau = cta_kth_largest(gkeys, n, 0u, 0xFFFFFFFFu, k, sh.rs, 1, pc, &need_eq);
     int a = 0, b = 0;
     for (int j = tid; j < lo_c; j += kScThreads) {
       const uint32_t key = __ldg(gkeys + j);
