@@ -120,13 +120,8 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
   const int Npad = (N + 15) & ~15;
   const int Nr = expo_stride(N);  // row length of the exponent table
   const int tstride = Npad <= 64 ? 64 : (Npad <= 128 ? 128 : 256);
-  // Units of at most 64 query rows keep, per epilogue warpgroup, each
-  // token's running exponent sums in 64 more TMEM columns (reduced across
-  // tokens once per item instead of once per tile), with one accumulator
-  // buffer per warpgroup; larger units reduce every tile.
-  const bool tacc = !kLse && Npad <= 64;
-  const int nbuf = tacc ? kWG : ((4 * tstride <= 512) ? 4 : 2);
-  const uint32_t tcols = static_cast<uint32_t>(nbuf * tstride + (tacc ? kWG * 64 : 0));
+  const int nbuf = (4 * tstride <= 512) ? 4 : 2;
+  const uint32_t tcols = static_cast<uint32_t>(nbuf * tstride);
   const int t0 = it.t0;
   const int ntiles = it.t1 - t0;  // >= 1 by construction
 
@@ -351,15 +346,6 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
       // triggers its dependents after its last read of them, so this grid
       // (launched no earlier than that trigger) may overwrite them without
       // waiting for the kernels before it.
-      // Per-token running sums (tacc): this warp's lanes of its warpgroup's
-      // 64 columns, zero at the start of the item.
-      const uint32_t tsum = tbase + (static_cast<uint32_t>(qd * 32) << 16) +
-                            static_cast<uint32_t>(nbuf * tstride + wg * 64);
-      if (tacc && wg < nwg) {
-        const uint32_t zz[32] = {};
-        for (int c0 = 0; c0 < N; c0 += 32) tmem_store32(tsum + c0, zz);
-        tmem_wait_st();
-      }
 
       for (int i = wg; wg < nwg && i < ntiles; i += nwg) {
         const int b = i % nbuf;
@@ -446,20 +432,7 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
             const float old = rf[lane];
             const float nw = fmaxf(old, m - kShift);
             // the sums kept against the old R shrink by 2^(old - new)
-            const float shrink =
-                (nw == old) ? 1.f : ((old == kNegInf) ? 0.f : ex2_approx(old - nw));
-            if (tacc) {
-              uint32_t a[32];
-              tmem_load32_async(tsum + c0, a);
-              tmem_wait_ld(a);
-#pragma unroll
-              for (int j = 0; j < 32; ++j)
-                a[j] = __float_as_uint(__uint_as_float(a[j]) * __shfl_sync(0xffffffffu, shrink, j));
-              tmem_store32(tsum + c0, a);
-              tmem_wait_st();
-            } else {
-              acc_s[c0 + lane] *= shrink;
-            }
+            acc_s[c0 + lane] *= (nw == old) ? 1.f : ((old == kNegInf) ? 0.f : ex2_approx(old - nw));
             __syncwarp();
             rf[lane] = nw;
             __syncwarp();
@@ -495,19 +468,9 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
               }
             }
           }
-          if (tacc) {
-            uint32_t a[32];
-            tmem_load32_async(tsum + c0, a);
-            tmem_wait_ld(a);
-#pragma unroll
-            for (int j = 0; j < 32; ++j) a[j] = __float_as_uint(__uint_as_float(a[j]) + e[j]);
-            tmem_store32(tsum + c0, a);
-            tmem_wait_st();
-          } else {
-            const float colsum = warp_transpose_sum32(e, lane);
-            acc_s[c0 + lane] += colsum;
-            __syncwarp();
-          }
+          const float colsum = warp_transpose_sum32(e, lane);
+          acc_s[c0 + lane] += colsum;
+          __syncwarp();
         }
         // the references this tile quarter's exponents are relative to
         {
@@ -517,19 +480,6 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(tempty0 + 8 * b);
-      }
-      if (tacc && wg < nwg && !*abort_flag) {
-        // per-token sums -> this warp's per-query sums (one reduction per item)
-        for (int c0 = 0; c0 < N; c0 += 32) {
-          uint32_t a[32];
-          tmem_load32_async(tsum + c0, a);
-          tmem_wait_ld(a);
-          float v[32];
-#pragma unroll
-          for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(a[j]);
-          acc_s[c0 + lane] = warp_transpose_sum32(v, lane);
-        }
-        __syncwarp();
       }
       // merge the epilogue warps' (R, sum) pairs per query into the item's pair
       named_bar_sync(kBarEpi, 32 * kNumEpiWarps);
