@@ -129,6 +129,28 @@ def test_exact_ties_break_to_lower_position(cuda_device):
         assert idx[g, :k].tolist() == list(range(r, r + k))
 
 
+def test_selection_full_search_paths(cuda_device):
+    """The fused call's selection lists the keys at or above a sampled lower
+    bound and falls back to a search over all of a unit's keys when that list
+    would exceed 4096 keys.  Equal keys at L = 10000 (about 10000 tied
+    candidates) and a budget of 9000 at L = 12000 take the fallback; both must
+    still equal the oracle (ties to the lowest interior positions)."""
+    cfg = wl.get("c1").scaled(seq_len=10000, dtype="bf16")
+    d = wl.make_layer(cfg, 0, sinks=False, needle_gain=0.0)
+    d["k"][:] = d["k"][0:1]
+    out, res, ties = check(d, cfg.window, cfg.pool_width, cuda_device)
+    assert ties == 0
+    r = (cfg.pool_width - 1) // 2
+    k = 128 - cfg.window
+    idx = out.indices.cpu().numpy()
+    for g in range(8):
+        assert idx[g, :k].tolist() == list(range(r, r + k))
+
+    cfg = wl.get("c1").scaled(seq_len=12000, dtype="bf16", srh_per_group=(1, 2))
+    d = wl.make_layer(cfg, 0, budgets=np.array([[9000]], np.int32))
+    check(d, cfg.window, cfg.pool_width, cuda_device)
+
+
 def test_strided_inputs(cuda_device):
     """K and V as views of one packed KV tensor; Q as a slice of a larger window."""
     cfg = wl.get("c1").scaled(seq_len=777, dtype="bf16", srh_per_group=(2, 2))
