@@ -352,9 +352,19 @@ struct LseInput {
   long long batch_stride = 0, head_stride = 0;
 };
 
+// Without a given LSE, units are scored in one of two ways:
+//  * one pass with the exponent table and the combine kernel (raw and pooled
+//    scores), when the layer's table -- with the actual SRH rows -- fits one
+//    set of kExpoSetBytes, i.e. stays in L2 between the two kernels;
+//  * otherwise two passes over K without a table (*two_pass set): the scoring
+//    kernel in stats-only mode leaves the per-unit log2 softmax denominators,
+//    and the given-LSE kernel reads them and writes raw scores (into `raw`,
+//    else the workspace's raw row); the caller then pools and selects from
+//    raw scores.  Reading K twice moves fewer bytes than writing and reading
+//    a table that does not stay in L2.
 int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void* k,
               const uint8_t* mask, float* raw, float* pooled, const Workspace& ws,
-              cudaStream_t stream, const LseInput& lse = LseInput{}) {
+              cudaStream_t stream, const LseInput& lse = LseInput{}, bool* two_pass = nullptr) {
   const bool given_lse = lse.lse != nullptr;
   if (!q_win || !k || (given_lse ? !raw : !pooled)) return CKV_ERR_INVALID_ARG;
   if (!aligned16(q_win) || !aligned16(k)) return CKV_ERR_INVALID_ARG;
@@ -415,7 +425,22 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
       for (int g = 0; g < I.Hkv; ++g)
         units.push_back({s, g, (I.len[s] + kTileTokens - 1) / kTileTokens, (I.n[s] + 31) / 32});
   std::vector<UnitSet> sets;
-  plan_sets(I, sets);
+  // the layer's exponent table with the actual SRH rows
+  long long table_bytes = 0;
+  for (const Unit& U : units) table_bytes += 2LL * I.n[U.s] * expo_stride(S.rows[U.g]);
+  const bool passes2 = !given_lse && table_bytes > kExpoSetBytes;
+  if (two_pass) *two_pass = passes2;
+  if (passes2) {
+    // no table: sets are bounded by the work-item tables only
+    sets.clear();
+    for (int u0 = 0; u0 < static_cast<int>(units.size()); u0 += kMaxItems / 2)
+      sets.push_back({u0, std::min<int>(static_cast<int>(units.size()), u0 + kMaxItems / 2), 0, 0});
+    if (!raw) raw = ws.raw;
+    P.stats_only = 1;
+    P.raw_out = raw;
+  } else {
+    plan_sets(I, sets);
+  }
   Tracer tr{p->trace, stream};
   // Per-layer selection sums the groups' scores: a group without an SRH head
   // contributes zeros.
@@ -537,6 +562,16 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
       if (rc != CKV_OK) return rc;
       continue;
     }
+    if (passes2) {
+      // pass 1: denominators only; pass 2: raw scores from them
+      rc = traced(tr, CKV_KERNEL_SCORE, [&] { return launch_score(P, n_items, smem, stream); });
+      if (rc != CKV_OK) return rc;
+      P.lse_bias = ws.bias;
+      rc = traced(tr, CKV_KERNEL_SCORE, [&] { return launch_score_lse(P, n_items, smem, stream); });
+      P.lse_bias = nullptr;
+      if (rc != CKV_OK) return rc;
+      continue;
+    }
     rc = traced(tr, CKV_KERNEL_SCORE, [&] { return launch_score(P, n_items, smem, stream); });
     if (rc != CKV_OK) return rc;
     rc = traced(tr, CKV_KERNEL_COMBINE,
@@ -604,9 +639,10 @@ int run_select(const ckv_problem* p, const Info& I, const float* raw, const floa
     P.cu_out[s] = cu_out[s];
     if (s < I.B) max_n = std::max(max_n, I.n[s]);
   }
-  if (pooled_in && !I.layer) {
+  if (pooled_in && !I.layer && max_n <= 32 * 1024) {
     // fused layer call, per-group selection: sampled select, a cluster of up
-    // to 16 CTAs per unit with about kScTargetSlice positions each
+    // to 16 CTAs per unit with about kScTargetSlice positions each (longer
+    // prefixes list too many keys above the sampled bound)
     const int C = std::min(F->sampled_cluster,
                            std::max(1, (max_n + kScTargetSlice - 1) / kScTargetSlice));
     const int S = std::max(32, ((max_n + C - 1) / C + 31) / 32 * 32);
@@ -769,7 +805,13 @@ int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const voi
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   float* pooled = pooled_scores ? pooled_scores : ws.pooled;
   std::copy(co.begin(), co.end(), cu_out);
-  if ((rc = run_score(p, I, q_win, k, srh_mask, raw_scores, pooled, ws, st)) != CKV_OK) return rc;
+  bool two_pass = false;
+  if ((rc = run_score(p, I, q_win, k, srh_mask, raw_scores, pooled, ws, st, LseInput{},
+                      &two_pass)) != CKV_OK)
+    return rc;
+  if (two_pass)  // raw scores only: pool and select from them
+    return run_select(p, I, raw_scores ? raw_scores : ws.raw, nullptr, co, indices,
+                      pooled_scores, ws, st, k, v, k_out, v_out);
   return run_select(p, I, nullptr, pooled, co, indices, nullptr, ws, st, k, v, k_out, v_out);
 }
 
@@ -846,7 +888,13 @@ int compresskv_compress_layer_head_budgets(const ckv_problem* p, const void* q_w
   co[I.B] = static_cast<int>(row);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   float* pooled = pooled_scores ? pooled_scores : ws.pooled;
-  if ((rc = run_score(p, I, q_win, k, srh_mask, raw_scores, pooled, ws, st)) != CKV_OK) return rc;
+  bool two_pass = false;
+  if ((rc = run_score(p, I, q_win, k, srh_mask, raw_scores, pooled, ws, st, LseInput{},
+                      &two_pass)) != CKV_OK)
+    return rc;
+  if (two_pass)  // raw scores only: pool and select from them
+    return run_select(p, I, raw_scores ? raw_scores : ws.raw, nullptr, co, indices,
+                      pooled_scores, ws, st, k, v, k_out, v_out, &unit_out);
   return run_select(p, I, nullptr, pooled, co, indices, nullptr, ws, st, k, v, k_out, v_out,
                     &unit_out);
 }

@@ -44,6 +44,8 @@ struct ScoreParams {
   const uint16_t* q;           // window queries (f16/bf16 bits)
   float2* partials;            // [n_items][kMaxQRows]: (M, S) with sum 2^(z*c) = S * 2^M
   float* bias;                 // [item of the unit's first item][kMaxQRows]: log2 D_q per unit
+  int stats_only;              // 1: no exponent / reference tables (first of two passes)
+  const float* lse_bias;       // given-LSE kernel: log2 D_q rows of a first pass instead of lse
   int* tickets;                // [kMaxItems]: items of the unit done (zero between calls)
   uint16_t* expo;              // fp16 2^(z*c - R) per prefix key and query row (Nr per key)
   float* refs;                 // per (tile, quarter, query row): the R used for expo

@@ -209,14 +209,21 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
     fence_proxy_async_smem();
     for (int q = st_tid; q < kMaxQRows; q += kStagedThreads) sWpos[q] = q < N ? q % W : 0;
     if constexpr (kLse) {
-      // log2 of every query row's softmax denominator (first rows of sRef)
+      // log2 of every query row's softmax denominator (first rows of sRef);
+      // a first pass's rows are read only once that kernel has completed
+      if (p.lse_bias) pdl_wait();
       for (int q = st_tid; q < kMaxQRows; q += kStagedThreads) {
         float l2 = 0.f;
         if (q < N) {
-          const int head = p.srh_heads[h0 + q / W];
-          const int w = q - (q / W) * W;
-          l2 = p.lse[static_cast<long long>(s) * p.lse_bs + static_cast<long long>(head) * p.lse_hs +
-                     w] * 1.4426950408889634f;
+          if (p.lse_bias) {  // second pass: the first pass's log2 denominators
+            l2 = p.lse_bias[static_cast<long long>(it.first) * kMaxQRows + q];
+          } else {
+            const int head = p.srh_heads[h0 + q / W];
+            const int w = q - (q / W) * W;
+            l2 = p.lse[static_cast<long long>(s) * p.lse_bs +
+                       static_cast<long long>(head) * p.lse_hs + w] *
+                 1.4426950408889634f;
+          }
         }
         sRef[q] = l2;
       }
@@ -361,7 +368,7 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
         const bool edge = (tile + 1) * kTileTokens > n;
         const int vis = n - tok;  // query row q sees this key iff tok < L and wpos(q) >= -vis
         const bool key = tok < L;    // a key of the sequence (the last tile may run past L)
-        const bool store = tok < n;  // the table holds prefix keys only
+        const bool store = tok < n && !p.stats_only;  // the table holds prefix keys only
         uint16_t* erow = p.expo + it.eoff + static_cast<long long>(tok) * Nr;
 
         for (int grp = 0; grp < ngrp; ++grp) {
@@ -473,7 +480,7 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
           __syncwarp();
         }
         // the references this tile quarter's exponents are relative to
-        {
+        if (!p.stats_only) {
           float* rt = p.refs + it.roff + (static_cast<long long>(tile) * kQuarters + qd) * Nr;
           for (int q = lane; q < N; q += 32) rt[q] = ref[q];
         }
