@@ -156,7 +156,8 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
     }
     for (int b = 0; b < 4; ++b) {
       mbar_init(tfull0 + 8 * b, 1);
-      mbar_init(tempty0 + 8 * b, 4);
+      // released by every warp of the warpgroups sharing the buffer
+      mbar_init(tempty0 + 8 * b, (!kLse && kWG > nbuf) ? 8 : 4);
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -348,13 +349,20 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
       // wait cannot tell phase k from phase k+2, so warpgroups sharing a
       // buffer could read it early.
       const int nwg = kWG < nbuf ? kWG : nbuf;
+      // With fewer TMEM buffers than warpgroups (query rows > 128: two
+      // buffers), two warpgroups share each buffer and split its 32-column
+      // groups (even / odd), so every epilogue warp has work.
+      const bool csplit = kWG > nbuf;
+      const int tg = wg % nwg;                  // tiles i % nwg == tg
+      const int gbeg = csplit ? wg / nwg : 0;   // first column group, step gstep
+      const int gstep = csplit ? 2 : 1;
       // The exponent and reference tables and the softmax pairs are reused
       // across calls on one workspace.  Their only reader, the combine kernel,
       // triggers its dependents after its last read of them, so this grid
       // (launched no earlier than that trigger) may overwrite them without
       // waiting for the kernels before it.
 
-      for (int i = wg; wg < nwg && i < ntiles; i += nwg) {
+      for (int i = tg; i < ntiles; i += nwg) {
         const int b = i % nbuf;
         const uint32_t use = static_cast<uint32_t>(i / nbuf) & 1u;
         const bool got = mbar_wait_bounded(tfull0 + 8 * b, use, abort_flag, p.status);
@@ -371,7 +379,7 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
         const bool store = tok < n && !p.stats_only;  // the table holds prefix keys only
         uint16_t* erow = p.expo + it.eoff + static_cast<long long>(tok) * Nr;
 
-        for (int grp = 0; grp < ngrp; ++grp) {
+        for (int grp = gbeg; grp < ngrp; grp += gstep) {
           const int c0 = 32 * grp;
           const int ncols = min(32, Nr - c0);  // 8, 16 or 32 (Nr is a power of two)
           if (c0 >= N) {
@@ -482,7 +490,7 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
         // the references this tile quarter's exponents are relative to
         if (!p.stats_only) {
           float* rt = p.refs + it.roff + (static_cast<long long>(tile) * kQuarters + qd) * Nr;
-          for (int q = lane; q < N; q += 32) rt[q] = ref[q];
+          for (int q = 32 * gbeg + lane; q < N; q += 32 * gstep) rt[q] = ref[q];
         }
         tc_fence_before();
         __syncwarp();
