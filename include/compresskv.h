@@ -34,7 +34,12 @@
  *   L_s = cu_seqlens[s+1] - cu_seqlens[s], n_s = max(L_s - W, 0).
  * - K, V: [T][num_kv_heads][head_dim] elements of `dtype`, head_dim contiguous,
  *   element strides kv_token_stride / kv_head_stride (multiples of 8, base
- *   16-byte aligned).  V shares K's strides.
+ *   16-byte aligned).  V shares K's strides.  V (read only by the gather)
+ *   may also live in page-locked host memory (cudaHostAlloc /
+ *   cudaHostRegister), which the device reads through unified addressing:
+ *   only the retained rows then cross the host link.  Pageable host memory
+ *   is refused with CKV_ERR_INVALID_ARG (checked with
+ *   cudaPointerGetAttributes before anything is enqueued).
  * - Window queries q_win: element (s, h, w, :) at
  *   q_win + s*q_batch_stride + h*q_head_stride + w*q_win_stride, head_dim
  *   contiguous; row w is the query of prompt position L_s - W + w.

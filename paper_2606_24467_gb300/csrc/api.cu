@@ -102,6 +102,26 @@ struct Info {
 
 bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
 
+// The address under which the device reads `ptr`: device or managed memory
+// as is, page-locked host memory through its mapped (unified) address.
+// Pageable or unknown memory is refused: a kernel must not touch it.
+int device_readable(const void* ptr, const void** dev) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, ptr) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return CKV_ERR_INVALID_ARG;
+  }
+  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) {
+    *dev = ptr;
+    return CKV_OK;
+  }
+  if (a.type == cudaMemoryTypeHost && a.devicePointer) {
+    *dev = a.devicePointer;
+    return CKV_OK;
+  }
+  return CKV_ERR_INVALID_ARG;
+}
+
 int validate(const ckv_problem* p, Info& I) {
   if (!p || !p->cu_seqlens) return CKV_ERR_INVALID_ARG;
   if (p->batch < 1 || p->batch > kMaxBatch) return CKV_ERR_UNSUPPORTED;
@@ -583,6 +603,20 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
 }
 
 // ------------------------------------------------------------------ select / gather
+// Arguments of the selection's outputs and, when `k` is given, of the fused
+// gather; `v` is replaced by the address the device reads it under.  The
+// fused layer calls run this before their first launch.
+int check_outputs(const Info& I, const std::vector<int>& cu_out, const int32_t* indices,
+                  const void* k, const void*& v, const void* k_out, const void* v_out) {
+  if (cu_out[I.B] == 0) return CKV_OK;
+  if (!indices) return CKV_ERR_INVALID_ARG;
+  if (!k) return CKV_OK;
+  if (!v || !k_out || !v_out) return CKV_ERR_INVALID_ARG;
+  if (!aligned16(k) || !aligned16(v) || !aligned16(k_out) || !aligned16(v_out))
+    return CKV_ERR_INVALID_ARG;
+  return device_readable(v, &v);
+}
+
 // Pooling (unless `pooled_in` holds the pooled scores already), top-k and
 // window append, optionally fused with the K/V gather.
 // With `unit_out` (head-level budgets) every unit (s, g) has its own output
@@ -594,13 +628,9 @@ int run_select(const ckv_problem* p, const Info& I, const float* raw, const floa
                const void* v = nullptr, void* k_out = nullptr, void* v_out = nullptr,
                const std::vector<int2>* unit_out = nullptr) {
   if (!raw && !pooled_in && I.p_total > 0) return CKV_ERR_INVALID_ARG;
-  if (!indices && cu_out[I.B] > 0) return CKV_ERR_INVALID_ARG;
   const bool gather = k != nullptr;
-  if (gather && cu_out[I.B] > 0) {
-    if (!v || !k_out || !v_out) return CKV_ERR_INVALID_ARG;
-    if (!aligned16(k) || !aligned16(v) || !aligned16(k_out) || !aligned16(v_out))
-      return CKV_ERR_INVALID_ARG;
-  }
+  const int rg = check_outputs(I, cu_out, indices, k, v, k_out, v_out);
+  if (rg != CKV_OK) return rg;
   DeviceFacts* F = nullptr;
   int rc = device_facts(&F);
   if (rc != CKV_OK) return rc;
@@ -681,6 +711,8 @@ int run_gather(const ckv_problem* p, const Info& I, const int32_t* indices,
   if (!indices || !k || !v || !k_out || !v_out) return CKV_ERR_INVALID_ARG;
   if (!aligned16(k) || !aligned16(v) || !aligned16(k_out) || !aligned16(v_out))
     return CKV_ERR_INVALID_ARG;
+  const int rv = device_readable(v, &v);
+  if (rv != CKV_OK) return rv;
   static thread_local GatherParams P;
   std::memset(&P, 0, sizeof(P));
   P.k = static_cast<const uint4*>(k);
@@ -805,6 +837,7 @@ int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const voi
   if ((rc = srh_lists(I, srh_mask, S)) != CKV_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   float* pooled = pooled_scores ? pooled_scores : ws.pooled;
+  if ((rc = check_outputs(I, co, indices, k, v, k_out, v_out)) != CKV_OK) return rc;
   std::copy(co.begin(), co.end(), cu_out);
   bool two_pass = false;
   if ((rc = run_score(p, I, q_win, k, srh_mask, raw_scores, pooled, ws, st, LseInput{},
@@ -838,6 +871,7 @@ int compresskv_compress_layer_lse(const ckv_problem* p, const void* q_win, const
   if ((rc = srh_lists(I, srh_mask, S)) != CKV_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   float* raw = raw_scores ? raw_scores : ws.raw;
+  if ((rc = check_outputs(I, co, indices, k, v, k_out, v_out)) != CKV_OK) return rc;
   std::copy(co.begin(), co.end(), cu_out);
   LseInput lse;
   lse.lse = lse_win;
@@ -887,6 +921,7 @@ int compresskv_compress_layer_head_budgets(const ckv_problem* p, const void* q_w
   }
   std::vector<int> co(I.B + 1, 0);
   co[I.B] = static_cast<int>(row);
+  if ((rc = check_outputs(I, co, indices, k, v, k_out, v_out)) != CKV_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   float* pooled = pooled_scores ? pooled_scores : ws.pooled;
   bool two_pass = false;

@@ -219,6 +219,42 @@ def test_gather_reports_bad_index(cuda_device):
     assert torch.equal(k_out[5, 3], k[5, 3])
 
 
+def test_v_in_page_locked_host_memory(cuda_device):
+    """V read in place from page-locked host memory (only the kept rows cross
+    the host link) gives the same outputs as V on the device, through the
+    fused call and the gather entry point; pageable host memory is refused
+    before anything is enqueued."""
+    cfg = wl.get("c1").scaled(seq_len=2500, dtype="bf16", batch=2, srh_per_group=(1, 2))
+    d = wl.make_layer(cfg, 0, lengths=[2500, 1300], budgets=np.array([[260, 130]], np.int32))
+    dev = cuda_device
+    ref, cu_ref = run_gpu(d, cfg.window, cfg.pool_width, dev)
+    v_host = d["v"].contiguous().pin_memory()
+    out, cu_out = run_gpu(d, cfg.window, cfg.pool_width, dev, v=v_host)
+    assert np.array_equal(cu_out, cu_ref)
+    assert torch.equal(out.indices, ref.indices)
+    assert torch.equal(out.k_out.view(torch.int16), ref.k_out.view(torch.int16))
+    assert torch.equal(out.v_out.view(torch.int16), ref.v_out.view(torch.int16))
+    q, k = d["q_win"].to(dev), d["k"].to(dev)
+    prob = ckv.Problem(q, k, d["cu_seqlens"], cfg.window, cfg.pool_width)
+    ws = ckv.workspace(prob, dev)
+    k2, v2 = torch.zeros_like(out.k_out), torch.zeros_like(out.v_out)
+    ckv.gather(prob, out.indices, cu_out, k, v_host, k2, v2, ws)
+    torch.cuda.synchronize()
+    assert ckv.read_device_status(ws) == 0
+    assert torch.equal(v2.view(torch.int16), ref.v_out.view(torch.int16))
+    pageable = d["v"].contiguous()
+    assert not pageable.is_pinned()
+    o3 = ckv.LayerOutputs(prob, d["budgets"], 128, k.dtype, dev)
+    with pytest.raises(ckv.CompressKVError) as e:
+        ckv.compress_layer(prob, q, k, pageable, d["srh_mask"], d["budgets"], o3.indices,
+                           o3.k_out, o3.v_out, ws)
+    assert e.value.code == ckv.compresskv.CKV_ERR_INVALID_ARG
+    with pytest.raises(ckv.CompressKVError):
+        ckv.gather(prob, out.indices, cu_out, k, pageable, k2, v2, ws)
+    torch.cuda.synchronize()
+    assert ckv.read_device_status(ws) == 0
+
+
 # ---------------------------------------------------------------------------
 # full-size layers of the benchmark workloads (every unit of a sampled layer)
 # ---------------------------------------------------------------------------
