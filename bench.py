@@ -25,6 +25,7 @@ import statistics
 import subprocess
 import sys
 import time
+import types
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
@@ -57,8 +58,10 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-lse", action="store_true",
                     help="skip the given-LSE (log-sum-exp supplied) measurement")
-    ap.add_argument("--streams", type=int, default=4,
-                    help="layers in flight: layer l runs on stream l %% S with its own workspace")
+    ap.add_argument("--streams", type=int, default=3,
+                    help="calls in flight: call c runs on stream c %% S with its own workspace")
+    ap.add_argument("--layers-per-call", type=int, default=2,
+                    help="layers compressed by one compress_layers call (one launch per kernel)")
     return ap.parse_args()
 
 
@@ -232,46 +235,77 @@ def run_ours(args):
     lengths, masks, budgets, layers = build_layers(cfg, dev)
     tokens = sum(lengths)
 
-    # library objects: one problem per layer, a shared workspace, per-layer outputs.
-    # Two graphs of the same step: `graph` (timed; consecutive kernels overlap
-    # through programmatic dependent launch) and `traced` (every launch
-    # bracketed by CUDA events, which serialises the kernels) for the
-    # per-kernel durations.
+    # The step's K, V and window queries live in one allocation each, like a
+    # model's cache [n_layers][T][H_kv][d]; each layer is a view into it.
+    B, T = cfg.batch, layers[0]["k"].shape[0]
+    k_all = torch.cat([lay["k"] for lay in layers])
+    v_all = torch.cat([lay["v"] for lay in layers])
+    q_all = torch.cat([lay["q_win"] for lay in layers])
+    for l, lay in enumerate(layers):
+        lay["k"], lay["v"] = k_all[l * T:(l + 1) * T], v_all[l * T:(l + 1) * T]
+        lay["q_win"] = q_all[l * B:(l + 1) * B]
+    torch.cuda.empty_cache()
+
+    # library objects: one compress_layers call per `layers_per_call` layers
+    # (the layers packed as one batch, one SRH mask per layer), a workspace
+    # per stream, per-call outputs.  Two graphs of the same step: `graph`
+    # (timed; consecutive kernels overlap through programmatic dependent
+    # launch) and `traced` (every launch bracketed by CUDA events, which
+    # serialises the kernels) for the per-kernel durations.
     trace = ckv.Trace(capacity=16 * cfg.n_layers)
     counter = ckv.Trace(capacity=0)
-    probs = [ckv.Problem(lay["q_win"], lay["k"], lay["cu_seqlens"], cfg.window, cfg.pool_width,
-                         trace=counter) for lay in layers]
-    tprobs = [ckv.Problem(lay["q_win"], lay["k"], lay["cu_seqlens"], cfg.window, cfg.pool_width,
-                          trace=trace) for lay in layers]
-    # Layers are independent: with S streams, layer l is compressed on stream
-    # l % S with that stream's workspace, so one layer's latency-bound select
-    # overlaps the next layer's K stream.  Each stream's kernels still chain
-    # through programmatic dependent launch.
+    lpc = max(1, args.layers_per_call)
+    calls = [(l0, min(l0 + lpc, cfg.n_layers)) for l0 in range(0, cfg.n_layers, lpc)]
+
+    def call_problem(l0, l1, tr):
+        m = l1 - l0
+        cu = np.concatenate([np.asarray(layers[0]["cu_seqlens"][:-1], np.int64) + j * T
+                             for j in range(m)] + [[m * T]]).astype(np.int32)
+        return ckv.Problem(q_all[l0 * B:l1 * B], k_all[l0 * T:l1 * T], cu, cfg.window,
+                           cfg.pool_width, trace=tr)
+
+    probs = [call_problem(l0, l1, counter) for l0, l1 in calls]
+    tprobs = [call_problem(l0, l1, trace) for l0, l1 in calls]
+    c_budgets = [np.concatenate([np.asarray(layers[l]["budgets"]).reshape(-1)
+                                 for l in range(l0, l1)]) for l0, l1 in calls]
+    c_masks = [np.stack([np.asarray(layers[l]["srh_mask"]) for l in range(l0, l1)])
+               for l0, l1 in calls]
+    # Calls are independent: with S streams, call c runs on stream c % S with
+    # that stream's workspace, so one call's latency-bound select overlaps
+    # the next call's K stream.  Each stream's kernels still chain through
+    # programmatic dependent launch.
     n_streams = max(1, args.streams)
     wss = [ckv.workspace(probs[0], dev) for _ in range(n_streams)]
     ws = wss[0]
     lanes = [torch.cuda.Stream() for _ in range(n_streams)]
-    outs = [ckv.LayerOutputs(probs[l], budgets[l], cfg.head_dim, layers[l]["k"].dtype, dev,
-                             scores=False) for l in range(cfg.n_layers)]
+    outs = [ckv.LayerOutputs(probs[c], c_budgets[c], cfg.head_dim, k_all.dtype, dev,
+                             scores=False) for c in range(len(calls))]
+    # per-layer problems and outputs for the single-layer measurements (e2e,
+    # given LSE)
+    lprobs = [ckv.Problem(lay["q_win"], lay["k"], lay["cu_seqlens"], cfg.window, cfg.pool_width)
+              for lay in layers]
+    louts = [ckv.LayerOutputs(lprobs[l], budgets[l], cfg.head_dim, layers[l]["k"].dtype, dev,
+                              scores=False) for l in range(cfg.n_layers)]
+
+    def run_call(pr, c, wsp, stream=None):
+        l0, l1 = calls[c]
+        o = outs[c]
+        ckv.compress_layers(pr[c], l1 - l0, q_all[l0 * B:l1 * B], k_all[l0 * T:l1 * T],
+                            v_all[l0 * T:l1 * T], c_masks[c], c_budgets[c], o.indices, o.k_out,
+                            o.v_out, wsp, stream=stream)
 
     def step(pr, streams=n_streams):
         if streams == 1:
-            for l, lay in enumerate(layers):
-                o = outs[l]
-                ckv.compress_layer(pr[l], lay["q_win"], lay["k"], lay["v"], lay["srh_mask"],
-                                   lay["budgets"], o.indices, o.k_out, o.v_out, ws)
+            for c in range(len(calls)):
+                run_call(pr, c, ws)
             return
         cur = torch.cuda.current_stream()
         fork = torch.cuda.Event()
         fork.record(cur)
         for st in lanes[:streams]:
             st.wait_event(fork)
-        for l, lay in enumerate(layers):
-            o = outs[l]
-            st = lanes[l % streams]
-            ckv.compress_layer(pr[l], lay["q_win"], lay["k"], lay["v"], lay["srh_mask"],
-                               lay["budgets"], o.indices, o.k_out, o.v_out, wss[l % streams],
-                               stream=st)
+        for c in range(len(calls)):
+            run_call(pr, c, wss[c % streams], stream=lanes[c % streams])
         for st in lanes[:streams]:
             done = torch.cuda.Event()
             done.record(st)
@@ -369,7 +403,7 @@ def run_ours(args):
                    "l2": f"inputs larger than L2: {sum(l['k'].numel() * 2 * 2 for l in layers) / 1e9:.2f} GB "
                          "of K/V per step, each layer's K read cold; no flush",
                    "cuda_graph": True, "parallelism": f"replicas x{world}",
-                   "layer_streams": n_streams,
+                   "layers_per_call": lpc, "call_streams": n_streams,
                    "l2_bytes": torch.cuda.get_device_properties(dev).L2_cache_size,
                    "sms": torch.cuda.get_device_properties(dev).multi_processor_count},
         "roofline": roofline,
@@ -383,11 +417,13 @@ def run_ours(args):
     }
 
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        result["cpu_baseline"], result["parity_layer0"] = cpu_baseline(cfg, layers[0], outs[0])
+        # layer 0's block of the first call's outputs
+        first = types.SimpleNamespace(indices=outs[0].indices[:, :int(outs[0].cu_out[B])])
+        result["cpu_baseline"], result["parity_layer0"] = cpu_baseline(cfg, layers[0], first)
     if not args.no_e2e:
-        result["e2e"] = run_e2e(args, cfg, layers, probs, ws, dev, dist, world)
+        result["e2e"] = run_e2e(args, cfg, layers, lprobs, ws, dev, dist, world)
     if not args.no_lse:
-        result["lse_fed"] = run_lse_fed(args, cfg, layers, outs, dev, dist, world, tokens)
+        result["lse_fed"] = run_lse_fed(args, cfg, layers, louts, dev, dist, world, tokens)
     if rank == 0:
         print(json.dumps(result), flush=True)
     if dist is not None:

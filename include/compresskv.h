@@ -208,6 +208,28 @@ int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const voi
                               float* raw_scores, float* pooled_scores,
                               void* workspace, size_t workspace_bytes, void* stream);
 
+/* compresskv_compress_layer for several layers in one call (prefill-end
+ * compression of a model: every layer's cache exists, Sec. 3; each layer
+ * selects with its own SRH heads, Sec. 3.3).  The batch of `p` packs n_masks blocks of
+ * batch / n_masks sequences and sequence s uses SRH mask s / (batch /
+ * n_masks): with a KV cache laid out [n_layers][T][H_kv][d], viewed as
+ * [n_layers*T][H_kv][d] with cu_seqlens repeated per layer (offset by l*T),
+ * and window queries [n_layers][B][H_q][W][d] viewed as
+ * [n_layers*B][H_q][W][d], block l is layer l.  One launch of each kernel
+ * then covers all the layers' units, so the scoring kernel's start-up and
+ * tail are paid once.
+ * n_masks: 1 <= n_masks <= 4, dividing batch (else CKV_ERR_INVALID_ARG /
+ *   CKV_ERR_UNSUPPORTED).
+ * srh_masks: host uint8 [n_masks][num_q_heads].
+ * budgets, cu_out and every output follow the packed batch (sequence
+ * l*B + s is sequence s of block l); the workspace is sized for `p`.
+ * With n_masks = 1 this is compresskv_compress_layer. */
+int compresskv_compress_layers(const ckv_problem* p, int n_masks, const void* q_win,
+                               const void* k, const void* v, const uint8_t* srh_masks,
+                               const int32_t* budgets, int32_t* indices, int32_t* cu_out,
+                               void* k_out, void* v_out, float* raw_scores, float* pooled_scores,
+                               void* workspace, size_t workspace_bytes, void* stream);
+
 /* compresskv_compress_layer when the softmax denominators of the window
  * queries are already known -- a prefill attention kernel has them as its
  * log-sum-exp (CompressKV's latency study, Sec. 4.4, runs on a

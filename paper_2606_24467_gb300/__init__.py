@@ -16,6 +16,7 @@ from .compresskv import (  # noqa: F401
     compress_layer_head_budgets,
     compress_layer_lse,
     compress_layer_noalloc,
+    compress_layers,
     gather,
     head_budget_layout,
     load,

@@ -42,6 +42,7 @@ EXPORTED = (
     "compresskv_select",
     "compresskv_gather",
     "compresskv_compress_layer",
+    "compresskv_compress_layers",
     "compresskv_compress_layer_noalloc",
     "compresskv_compress_layer_lse",
     "compresskv_compress_layer_head_budgets",
@@ -101,6 +102,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         "compresskv_gather": (c_int32, [pp, vp, i32p, vp, vp, vp, vp, vp, vp]),
         "compresskv_compress_layer": (c_int32, [pp, vp, vp, vp, vp, i32p, vp, i32p, vp, vp,
                                                  vp, vp, vp, c_size_t, vp]),
+        "compresskv_compress_layers": (c_int32, [pp, c_int32, vp, vp, vp, vp, i32p, vp, i32p, vp,
+                                                  vp, vp, vp, vp, c_size_t, vp]),
         "compresskv_compress_layer_noalloc": (c_int32, [pp, vp, vp, vp, vp, i32p, vp, i32p, vp,
                                                          vp, vp, vp, vp, vp]),
         "compresskv_compress_layer_lse": (c_int32, [pp, vp, vp, vp, vp, c_int64, c_int64, vp, i32p,
@@ -286,6 +289,26 @@ def compress_layer(problem: Problem, q_win, k, v, srh_mask, budgets, indices, k_
         problem.ref, _ptr(q_win), _ptr(k), _ptr(v), mp, bp, _ptr(indices),
         cu_out.ctypes.data_as(POINTER(c_int32)), _ptr(k_out), _ptr(v_out), _ptr(raw),
         _ptr(pooled), _ptr(ws), ws.numel(), _stream(stream)), "compresskv_compress_layer")
+    return cu_out
+
+
+def compress_layers(problem: Problem, n_masks: int, q_win, k, v, srh_masks, budgets, indices,
+                    k_out, v_out, ws, raw=None, pooled=None, stream=None) -> np.ndarray:
+    """Several layers in one call: ``problem``'s batch packs ``n_masks`` blocks
+    of sequences (block l = layer l: K ``[n_layers*T, H_kv, d]``, Q window
+    ``[n_layers*B, H_q, W, d]``, cu_seqlens repeated per layer with offset
+    l*T) and block l selects with ``srh_masks[l]`` (``[n_masks, H_q]``);
+    budgets ``[n_layers*B]``; outputs as for compress_layer on that batch."""
+    m = np.ascontiguousarray(np.asarray(srh_masks).astype(np.uint8).reshape(-1))
+    if n_masks >= 1 and m.size != int(n_masks) * int(problem.struct.num_q_heads):
+        raise CompressKVError(CKV_ERR_INVALID_ARG, "srh_masks must be [n_masks, num_q_heads]")
+    b, bp = _i32(budgets)
+    cu_out = np.zeros(problem.batch + 1, np.int32)
+    _check(load().compresskv_compress_layers(
+        problem.ref, int(n_masks), _ptr(q_win), _ptr(k), _ptr(v), c_void_p(m.ctypes.data), bp,
+        _ptr(indices), cu_out.ctypes.data_as(POINTER(c_int32)), _ptr(k_out), _ptr(v_out),
+        _ptr(raw), _ptr(pooled), _ptr(ws), ws.numel(), _stream(stream)),
+        "compresskv_compress_layers")
     return cu_out
 
 

@@ -98,6 +98,9 @@ struct Info {
   float scale = 0.f;
   std::vector<int> cu, len, n, cu_prefix;
   long long T = 0, p_total = 0;
+  // SRH masks: sequence s uses mask s / spm (n_masks masks, spm = B / n_masks)
+  int n_masks = 1, spm = 1;
+  int vgroup(int s, int g) const { return srh_group(s, g, spm, Hkv); }
 };
 
 bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
@@ -166,6 +169,8 @@ int validate(const ckv_problem* p, Info& I) {
   }
   I.T = I.cu[I.B];
   I.p_total = I.cu_prefix[I.B];
+  I.n_masks = 1;
+  I.spm = I.B;
   if (static_cast<long long>(I.Hkv) * I.p_total > (1LL << 31) - 1) return CKV_ERR_UNSUPPORTED;
   return CKV_OK;
 }
@@ -320,31 +325,40 @@ int traced(Tracer& tr, int kind, F&& fn) {
 }
 
 // ------------------------------------------------------------------ scoring
+// SRH heads per (mask, group), flattened: list v = m * H_kv + g holds
+// heads[off[v] .. off[v+1]) and rows[v] = |S| * W query rows.
 struct SrhLists {
   std::vector<uint16_t> off;
   std::vector<uint8_t> heads;
-  std::vector<int> rows;  // |S_g| * W per group
+  std::vector<int> rows;
 };
 
-int srh_lists(const Info& I, const uint8_t* mask, SrhLists& S) {
-  if (!mask) return CKV_ERR_INVALID_ARG;
-  S.off.assign(I.Hkv + 1, 0);
+// masks: I.n_masks masks of I.Hq bytes each.
+int srh_lists(const Info& I, const uint8_t* masks, SrhLists& S) {
+  if (!masks) return CKV_ERR_INVALID_ARG;
+  const int nv = I.n_masks * I.Hkv;
+  S.off.assign(nv + 1, 0);
   S.heads.clear();
-  S.rows.assign(I.Hkv, 0);
-  bool any_scored = false;
-  for (int s = 0; s < I.B; ++s) any_scored |= I.n[s] > 0;
-  for (int g = 0; g < I.Hkv; ++g) {
-    for (int h = g * I.G; h < (g + 1) * I.G; ++h)
-      if (mask[h]) S.heads.push_back(static_cast<uint8_t>(h));
-    S.off[g + 1] = static_cast<uint16_t>(S.heads.size());
-    const int cnt = S.off[g + 1] - S.off[g];
-    // per-group selection needs an SRH head in every group; per-layer
-    // selection only somewhere in the layer
-    if (cnt == 0 && any_scored && !I.layer) return CKV_ERR_EMPTY_SRH_GROUP;
-    S.rows[g] = cnt * I.W;
-    if (S.rows[g] > kMaxQRows) return CKV_ERR_UNSUPPORTED;
+  S.rows.assign(nv, 0);
+  for (int m = 0; m < I.n_masks; ++m) {
+    const uint8_t* mask = masks + static_cast<size_t>(m) * I.Hq;
+    bool any_scored = false;  // a sequence of this mask's block has a prefix
+    for (int s = m * I.spm; s < (m + 1) * I.spm; ++s) any_scored |= I.n[s] > 0;
+    const size_t first_head = S.heads.size();
+    for (int g = 0; g < I.Hkv; ++g) {
+      const int v = m * I.Hkv + g;
+      for (int h = g * I.G; h < (g + 1) * I.G; ++h)
+        if (mask[h]) S.heads.push_back(static_cast<uint8_t>(h));
+      S.off[v + 1] = static_cast<uint16_t>(S.heads.size());
+      const int cnt = S.off[v + 1] - S.off[v];
+      // per-group selection needs an SRH head in every group; per-layer
+      // selection only somewhere in the layer
+      if (cnt == 0 && any_scored && !I.layer) return CKV_ERR_EMPTY_SRH_GROUP;
+      S.rows[v] = cnt * I.W;
+      if (S.rows[v] > kMaxQRows) return CKV_ERR_UNSUPPORTED;
+    }
+    if (I.layer && S.heads.size() == first_head && any_scored) return CKV_ERR_EMPTY_SRH_GROUP;
   }
-  if (I.layer && S.heads.empty() && any_scored) return CKV_ERR_EMPTY_SRH_GROUP;
   return CKV_OK;
 }
 
@@ -435,19 +449,22 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
     C.cu_seqlens[s] = I.cu[s];
     C.cu_prefix[s] = I.cu_prefix[s];
   }
-  for (int g = 0; g <= I.Hkv; ++g) P.srh_off[g] = C.srh_off[g] = S.off[g];
+  P.seqs_per_mask = C.seqs_per_mask = I.spm;
+  for (size_t v = 0; v < S.off.size(); ++v) P.srh_off[v] = C.srh_off[v] = S.off[v];
   for (size_t h = 0; h < S.heads.size(); ++h) P.srh_heads[h] = S.heads[h];
 
-  struct Unit { int s, g, tiles, quarters; };
+  // units (s, g) with v = their SRH list
+  struct Unit { int s, g, v, tiles, quarters; };
   std::vector<Unit> units;
   for (int s = 0; s < I.B; ++s)
     if (I.n[s] > 0)
       for (int g = 0; g < I.Hkv; ++g)
-        units.push_back({s, g, (I.len[s] + kTileTokens - 1) / kTileTokens, (I.n[s] + 31) / 32});
+        units.push_back({s, g, I.vgroup(s, g), (I.len[s] + kTileTokens - 1) / kTileTokens,
+                         (I.n[s] + 31) / 32});
   std::vector<UnitSet> sets;
   // the layer's exponent table with the actual SRH rows
   long long table_bytes = 0;
-  for (const Unit& U : units) table_bytes += 2LL * I.n[U.s] * expo_stride(S.rows[U.g]);
+  for (const Unit& U : units) table_bytes += 2LL * I.n[U.s] * expo_stride(S.rows[U.v]);
   const bool passes2 = !given_lse && table_bytes > kExpoSetBytes;
   if (two_pass) *two_pass = passes2;
   if (passes2) {
@@ -459,20 +476,44 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
     P.stats_only = 1;
     P.raw_out = raw;
   } else {
-    plan_sets(I, sets);
+    // sets cut with the actual SRH rows, within the workspace's table space
+    const WorkspaceLayout WL = workspace_layout(I);
+    const long long cap_e = static_cast<long long>((WL.refs - WL.expo) / sizeof(uint16_t));
+    const long long cap_r = static_cast<long long>((WL.shared - WL.refs) / sizeof(float));
+    long long e = 0, r = 0;
+    int u0 = 0;
+    for (int u = 0; u < static_cast<int>(units.size()); ++u) {
+      const Unit& U = units[u];
+      const long long nr = expo_stride(S.rows[U.v]);
+      const long long ue = static_cast<long long>(I.n[U.s]) * nr;
+      const long long ur = static_cast<long long>(U.tiles) * kQuarters * nr;
+      if (u > u0 && (e + ue > cap_e || r + ur > cap_r || 2 * (e + ue) > kExpoSetBytes ||
+                     u - u0 >= kMaxItems / 2)) {
+        sets.push_back({u0, u, e, r});
+        u0 = u;
+        e = r = 0;
+      }
+      if (ue > cap_e || ur > cap_r) return CKV_ERR_WORKSPACE;  // cannot happen: the bound covers a unit
+      e += ue;
+      r += ur;
+    }
+    if (static_cast<int>(units.size()) > u0) sets.push_back({u0, static_cast<int>(units.size()), e, r});
   }
   Tracer tr{p->trace, stream};
   // Per-layer selection sums the groups' scores: a group without an SRH head
   // contributes zeros.
-  for (int g = 0; g < I.Hkv; ++g) {
-    if (S.rows[g] > 0) continue;
-    const size_t row = static_cast<size_t>(I.p_total) * sizeof(float);
-    if (pooled &&
-        cudaMemsetAsync(pooled + static_cast<size_t>(g) * I.p_total, 0, row, stream) != cudaSuccess)
-      return CKV_ERR_CUDA;
-    if (raw && cudaMemsetAsync(raw + static_cast<size_t>(g) * I.p_total, 0, row, stream) !=
-                   cudaSuccess)
-      return CKV_ERR_CUDA;
+  for (int m = 0; m < I.n_masks; ++m) {
+    for (int g = 0; g < I.Hkv; ++g) {
+      if (S.rows[m * I.Hkv + g] > 0) continue;
+      // the scores of this group for the mask's block of sequences
+      const size_t off = static_cast<size_t>(g) * I.p_total + I.cu_prefix[m * I.spm];
+      const size_t bytes =
+          static_cast<size_t>(I.cu_prefix[(m + 1) * I.spm] - I.cu_prefix[m * I.spm]) * sizeof(float);
+      if (bytes == 0) continue;
+      if (pooled && cudaMemsetAsync(pooled + off, 0, bytes, stream) != cudaSuccess)
+        return CKV_ERR_CUDA;
+      if (raw && cudaMemsetAsync(raw + off, 0, bytes, stream) != cudaSuccess) return CKV_ERR_CUDA;
+    }
   }
   for (const UnitSet& set : sets) {
     const int u0 = set.u0;
@@ -484,13 +525,13 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
     // split into balanced ranges.
     // (Units of a group without an SRH head -- per-layer selection only --
     // get no items.)
-    auto cost = [&](const Unit& U) { return 64LL + ((S.rows[U.g] + 15) & ~15); };
+    auto cost = [&](const Unit& U) { return 64LL + ((S.rows[U.v] + 15) & ~15); };
     std::vector<int> cnt(nu, 1);
     std::vector<long long> uw(nu);
     int active = 0;
     for (int u = 0; u < nu; ++u) {
       uw[u] = static_cast<long long>(units[u0 + u].tiles) * cost(units[u0 + u]);
-      cnt[u] = S.rows[units[u0 + u].g] > 0 ? 1 : 0;
+      cnt[u] = S.rows[units[u0 + u].v] > 0 ? 1 : 0;
       active += cnt[u];
     }
     if (active == 0) continue;
@@ -498,7 +539,7 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
     // their shared memory fits; else one CTA per SM with 16 epilogue warps.
     int max_rows = 16;
     for (int u = 0; u < nu; ++u)
-      if (cnt[u] > 0) max_rows = std::max(max_rows, (S.rows[units[u0 + u].g] + 15) & ~15);
+      if (cnt[u] > 0) max_rows = std::max(max_rows, (S.rows[units[u0 + u].v] + 15) & ~15);
     const int q_half = ((max_rows * 128) + 1023) & ~1023;
     const int per_sm =
         score_smem_bytes(q_half, 2, 8) <= static_cast<size_t>(F->smem_optin) / 2 - 1024 ? 2 : 1;
@@ -521,7 +562,7 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
     for (int u = 0; u < nu; ++u)
       if (cnt[u] > 0)
         weight += static_cast<long long>(units[u0 + u].quarters) *
-                  (expo_stride(S.rows[units[u0 + u].g]) + kQuarterFixed);
+                  (expo_stride(S.rows[units[u0 + u].v]) + kQuarterFixed);
     const long long ctarget = std::max(1, std::min(kMaxItems - nu, 2 * F->sms));
     const long long per_chunk = std::max<long long>(8 * (8 + kQuarterFixed),
                                                     (weight + ctarget - 1) / ctarget);
@@ -529,7 +570,7 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
     size_t csmem = 0;
     for (int u = 0; u < nu; ++u) {
       if (cnt[u] == 0) continue;
-      const int nr = expo_stride(S.rows[units[u0 + u].g]);
+      const int nr = expo_stride(S.rows[units[u0 + u].v]);
       int cq = static_cast<int>(std::max(1LL, per_chunk / (nr + kQuarterFixed)));
       // a chunk's weight table and raw scores must fit the shared memory
       while (cq > 1 && combine_smem_bytes(cq, nr, I.P) > F->combine_smem_max) cq = (cq + 1) / 2;
@@ -544,7 +585,7 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
       const Unit& U = units[u0 + u];
       const int c_u = cnt[u];
       if (c_u == 0) continue;
-      const int nr = expo_stride(S.rows[U.g]);
+      const int nr = expo_stride(S.rows[U.v]);
       if (n_items + c_u > kMaxItems) return CKV_ERR_UNSUPPORTED;
       for (int c = 0; c < c_u; ++c) {
         WorkItem& it = P.items[n_items + c];
@@ -825,9 +866,24 @@ int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const voi
                               int32_t* indices, int32_t* cu_out, void* k_out, void* v_out,
                               float* raw_scores, float* pooled_scores, void* workspace,
                               size_t workspace_bytes, void* stream) {
+  return compresskv_compress_layers(p, 1, q_win, k, v, srh_mask, budgets, indices, cu_out, k_out,
+                                    v_out, raw_scores, pooled_scores, workspace, workspace_bytes,
+                                    stream);
+}
+
+int compresskv_compress_layers(const ckv_problem* p, int n_masks, const void* q_win,
+                               const void* k, const void* v, const uint8_t* srh_masks,
+                               const int32_t* budgets, int32_t* indices, int32_t* cu_out,
+                               void* k_out, void* v_out, float* raw_scores, float* pooled_scores,
+                               void* workspace, size_t workspace_bytes, void* stream) {
   Info I;
   int rc = validate(p, I);
   if (rc != CKV_OK) return rc;
+  if (n_masks < 1 || I.B % n_masks != 0) return CKV_ERR_INVALID_ARG;
+  if (n_masks > kMaxMasks) return CKV_ERR_UNSUPPORTED;
+  I.n_masks = n_masks;
+  I.spm = I.B / n_masks;
+  const uint8_t* srh_mask = srh_masks;
   std::vector<int> co;
   if ((rc = output_layout(I, budgets, co)) != CKV_OK) return rc;
   if (!cu_out) return CKV_ERR_INVALID_ARG;

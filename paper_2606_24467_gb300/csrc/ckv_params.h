@@ -18,6 +18,8 @@ constexpr int kMaxQHeads = 256;
 constexpr int kMaxKvHeads = 64;
 constexpr int kMaxItems = 1024;     // score work items per launch
 constexpr int kMaxBudgetUnits = 2048;  // (sequence, group) pairs with their own budget
+constexpr int kMaxMasks = 4;        // SRH masks per call (the layers of one multi-layer call)
+constexpr int kMaxSrhGroups = kMaxMasks * kMaxKvHeads;
 constexpr uint64_t kWaitTimeoutNs = 2000000000ull;  // 2 s: far above any legitimate wait
 
 // Device status codes (mirrors of the public CKV_ERR_* values).
@@ -62,8 +64,11 @@ struct ScoreParams {
   int stages;                  // K tiles in the shared-memory ring (2..kStages)
   int epi_warps;               // 8 (two CTAs per SM) or 16 (one CTA per SM)
   int cu_seqlens[kMaxBatch + 1];
-  uint16_t srh_off[kMaxKvHeads + 1];   // SRH heads of group g: srh_heads[srh_off[g] .. srh_off[g+1])
-  uint8_t srh_heads[kMaxQHeads];
+  // SRH lists: sequence s uses mask m = s / seqs_per_mask; the SRH heads of
+  // its group g are srh_heads[srh_off[v] .. srh_off[v+1]), v = m*H_kv + g
+  int seqs_per_mask;
+  uint16_t srh_off[kMaxSrhGroups + 1];
+  uint8_t srh_heads[kMaxMasks * kMaxQHeads];
   WorkItem items[kMaxItems];
 };
 
@@ -77,9 +82,15 @@ struct CombineParams {
   int window, pool_width, num_kv_heads, p_total, n_items;
   int cu_seqlens[kMaxBatch + 1];
   int cu_prefix[kMaxBatch + 1];
-  uint16_t srh_off[kMaxKvHeads + 1];
+  int seqs_per_mask;           // as in ScoreParams
+  uint16_t srh_off[kMaxSrhGroups + 1];
   WorkItem items[kMaxItems];
 };
+
+// SRH list index of (sequence s, group g).
+__host__ __device__ inline int srh_group(int s, int g, int seqs_per_mask, int num_kv_heads) {
+  return (s / seqs_per_mask) * num_kv_heads + g;
+}
 
 // Row length (fp16 elements) of the exponent table for `rows` query rows:
 // the next power of two >= max(rows, 8), so that a row is a whole number of
@@ -128,6 +139,11 @@ struct GatherParams {
   int cu_seqlens[kMaxBatch + 1];
   int cu_out[kMaxBatch + 1];
 };
+
+// Kernel parameters travel by value; CUDA takes at most 32764 bytes of them.
+static_assert(sizeof(ScoreParams) <= 32764, "scoring kernel parameters");
+static_assert(sizeof(CombineParams) <= 32764, "combine kernel parameters");
+static_assert(sizeof(SelectParams) <= 32764, "selection kernel parameters");
 
 // Host-side launchers (defined next to each kernel).
 cudaError_t launch_score(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s);

@@ -66,7 +66,8 @@ __global__ void __launch_bounds__(kCombThreads)
   const int L = p.cu_seqlens[s + 1] - p.cu_seqlens[s];
   const int W = p.window;
   const int n = L - W;
-  const int N = (p.srh_off[g + 1] - p.srh_off[g]) * W;
+  const int vg = srh_group(s, g, p.seqs_per_mask, p.num_kv_heads);
+  const int N = (p.srh_off[vg + 1] - p.srh_off[vg]) * W;
   const int Nr = expo_stride(N);
   const int cpr = Nr >> 3;  // 16-byte chunks per key row (a power of two <= 32)
   const int lg_cpr = __ffs(cpr) - 1;

@@ -115,8 +115,9 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
   const int L = p.cu_seqlens[s + 1] - seq0;
   const int W = p.window;
   const int n = L - W;
-  const int h0 = p.srh_off[g];
-  const int N = (p.srh_off[g + 1] - h0) * W;
+  const int vg = srh_group(s, g, p.seqs_per_mask, p.num_kv_heads);
+  const int h0 = p.srh_off[vg];
+  const int N = (p.srh_off[vg + 1] - h0) * W;
   const int Npad = (N + 15) & ~15;
   const int Nr = expo_stride(N);  // row length of the exponent table
   const int tstride = Npad <= 64 ? 64 : (Npad <= 128 ? 128 : 256);
@@ -529,18 +530,18 @@ __global__ void __launch_bounds__(Shape<kEpi>::kThreads, Shape<kEpi>::kCtasPerSm
         const int sub = te / N;
         float m = kNegInf, z = 0.f;
         if (sub < nm) {
-          // eight pairs in flight per batch (L2 reads of the other CTAs' rows)
-          for (int i0 = sub; i0 < it.count; i0 += 8 * nm) {
-            float2 pr[8];
+          // sixteen pairs in flight per batch (L2 reads of the other CTAs' rows)
+          for (int i0 = sub; i0 < it.count; i0 += 16 * nm) {
+            float2 pr[16];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) {
+            for (int u = 0; u < 16; ++u) {
               const int i = i0 + u * nm;
               pr[u] = i < it.count
                           ? __ldcg(p.partials + static_cast<long long>(it.first + i) * kMaxQRows + q)
                           : make_float2(kNegInf, 0.f);
             }
 #pragma unroll
-            for (int u = 0; u < 8; ++u) {
+            for (int u = 0; u < 16; ++u) {
               if (pr[u].x == kNegInf) continue;
               if (pr[u].x > m) {
                 z = fmaf(z, ex2_approx(m - pr[u].x), pr[u].y);

@@ -380,8 +380,8 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
 // Sampled cluster select (per-group selection of a fused layer call): the same
 // result as select_kernel -- the top-k prefix positions of every unit by
 // pooled score, ties to the lower position, ascending, the window appended,
-// the K/V rows copied -- with three cluster barriers instead of one per radix
-// pass.  One cluster of C <= 16 CTAs per unit; CTA r owns the contiguous
+// the K/V rows copied -- with three cluster barriers (five on a retry)
+// instead of one per radix pass.  One cluster of C <= 16 CTAs per unit; CTA r owns the contiguous
 // slice [r*S, (r+1)*S) of the unit's prefix positions.
 //   1. The slice's pooled scores go to shared memory; each CTA sends 256 / C
 //      evenly spaced scores of its slice to every CTA of the cluster.
@@ -390,6 +390,9 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
 //      samples above it), r a few standard deviations above the expected
 //      number k * (samples / n) of samples above the k-th score.
 //   3. Each CTA lists its keys >= lo in position order and sends the count.
+//      If fewer than k keys reach lo (a unit whose few top keys hold several
+//      samples), steps 2-3 run once more with the r whose expected count of
+//      keys above it is halfway between k and kScCandCap.
 //      When between k and kScCandCap keys reach lo (the usual case), every
 //      CTA reads all lists (position order across the cluster), finds the
 //      k-th largest key tau and how many keys equal to it are kept (radix
@@ -537,75 +540,93 @@ __global__ void __launch_bounds__(kScThreads)
   cluster_arrive_release();
   cluster_wait();
 
-  // 2. lower bound from the samples: the rs-th largest, by counting for each
-  //    sample the samples above it and equal to it
+  // 2.-3. A lower bound lo from the samples, then every CTA's candidates
+  //    (keys >= lo); a second, looser bound when the first leaves fewer than
+  //    k candidates (a unit whose top keys are few and happen to hold
+  //    several samples), before the full search.
   int nsamp = 0;
   for (int c = 0; c < C; ++c) nsamp += sh.samp_cnt[c];
   const float mu = static_cast<float>(k) * static_cast<float>(nsamp) / static_cast<float>(n);
-  const int rs = min(nsamp, static_cast<int>(ceilf(mu + 3.f * sqrtf(mu))) + 2);
-  {
-    const int v = sh.samp[tid];  // kScThreads == kScSampleTotal: one sample per thread
-    const int4* s4 = reinterpret_cast<const int4*>(sh.samp);
-    int gt = 0, eq = 0;
+  int rs = min(nsamp, static_cast<int>(ceilf(mu + 3.f * sqrtf(mu))) + 2);
+  uint32_t lo = 0;
+  int own = 0, total = 0, before = 0, any_ovf = 0;
+  for (int attempt = 0; attempt < 2; ++attempt) {
+    // the rs-th largest sample, by counting for each sample the samples
+    // above it and equal to it
+    {
+      const int v = sh.samp[tid];  // kScThreads == kScSampleTotal: one sample per thread
+      const int4* s4 = reinterpret_cast<const int4*>(sh.samp);
+      int gt = 0, eq = 0;
 #pragma unroll 8
-    for (int j = 0; j < kScSampleTotal / 4; ++j) {  // empty slots (-1) never count
-      const int4 x = s4[j];
-      gt += (x.x > v) + (x.y > v) + (x.z > v) + (x.w > v);
-      eq += (x.x == v) + (x.y == v) + (x.z == v) + (x.w == v);
+      for (int j = 0; j < kScSampleTotal / 4; ++j) {  // empty slots (-1) never count
+        const int4 x = s4[j];
+        gt += (x.x > v) + (x.y > v) + (x.z > v) + (x.w > v);
+        eq += (x.x == v) + (x.y == v) + (x.z == v) + (x.w == v);
+      }
+      if (v >= 0 && gt < rs && rs <= gt + eq) sh.lo = static_cast<uint32_t>(v);  // equal samples agree
     }
-    if (v >= 0 && gt < rs && rs <= gt + eq) sh.lo = static_cast<uint32_t>(v);  // equal samples agree
-  }
-  __syncthreads();
-  const uint32_t lo = sh.lo;
+    __syncthreads();
+    lo = sh.lo;
 
-  // 3. own candidates (keys >= lo) in position order; counts to every CTA
-  const int seg = ((len + kScThreads - 1) / kScThreads) * 32;  // positions per warp
-  const int wlo = min(len, warp * seg);
-  const int whi = min(len, wlo + seg);
-  int wc = 0;
+    // own candidates (keys >= lo) in position order; counts to every CTA
+    const int seg = ((len + kScThreads - 1) / kScThreads) * 32;  // positions per warp
+    const int wlo = min(len, warp * seg);
+    const int whi = min(len, wlo + seg);
+    int wc = 0;
 #pragma unroll 4
-  for (int b0 = wlo; b0 < whi; b0 += 32) {
-    const int i = b0 + lane;
-    wc += __popc(__ballot_sync(0xffffffffu, i < whi && key_at(i) >= lo));
-  }
-  if (lane == 0) sh.wcnt[warp] = wc;
-  __syncthreads();
-  if (warp == 0) {
-    const int v = lane < kScWarps ? sh.wcnt[lane] : 0;
-    const int ex = warp_exclusive_scan(v, lane);
-    if (lane < kScWarps) sh.wbase[lane] = ex;
-    if (lane == kScWarps - 1) sh.red0 = ex + v;  // own candidate count
-  }
-  __syncthreads();
-  const int own = sh.red0;
-  {
-    int o = sh.wbase[warp];
-#pragma unroll 2
     for (int b0 = wlo; b0 < whi; b0 += 32) {
       const int i = b0 + lane;
-      const uint32_t key = i < whi ? key_at(i) : 0u;
-      const bool c = i < whi && key >= lo;
-      const uint32_t mm = __ballot_sync(0xffffffffu, c);
-      const int slot = o + __popc(mm & lanemask_lt(lane));
-      if (c && slot < kScCandCap) {
-        sh.ckey[slot] = key;
-        sh.cpos[slot] = lo_c + i;
-      }
-      o += __popc(mm);
+      wc += __popc(__ballot_sync(0xffffffffu, i < whi && key_at(i) >= lo));
     }
-  }
-  if (tid < C) {
-    *cluster.map_shared_rank(&sh.cand_cnt[cr], tid) = own;
-    *cluster.map_shared_rank(&sh.ovf[cr], tid) = own > kScCandCap ? 1 : 0;
-  }
-  __syncthreads();  // own list complete before the others may read it
-  cluster_arrive_release();
-  cluster_wait();
-  int total = 0, before = 0, any_ovf = 0;
-  for (int c = 0; c < C; ++c) {
-    if (c < cr) before += sh.cand_cnt[c];
-    total += sh.cand_cnt[c];
-    any_ovf |= sh.ovf[c];
+    if (lane == 0) sh.wcnt[warp] = wc;
+    __syncthreads();
+    if (warp == 0) {
+      const int v = lane < kScWarps ? sh.wcnt[lane] : 0;
+      const int ex = warp_exclusive_scan(v, lane);
+      if (lane < kScWarps) sh.wbase[lane] = ex;
+      if (lane == kScWarps - 1) sh.red0 = ex + v;  // own candidate count
+    }
+    __syncthreads();
+    own = sh.red0;
+    {
+      int o = sh.wbase[warp];
+#pragma unroll 2
+      for (int b0 = wlo; b0 < whi; b0 += 32) {
+        const int i = b0 + lane;
+        const uint32_t key = i < whi ? key_at(i) : 0u;
+        const bool c = i < whi && key >= lo;
+        const uint32_t mm = __ballot_sync(0xffffffffu, c);
+        const int slot = o + __popc(mm & lanemask_lt(lane));
+        if (c && slot < kScCandCap) {
+          sh.ckey[slot] = key;
+          sh.cpos[slot] = lo_c + i;
+        }
+        o += __popc(mm);
+      }
+    }
+    if (tid < C) {
+      *cluster.map_shared_rank(&sh.cand_cnt[cr], tid) = own;
+      *cluster.map_shared_rank(&sh.ovf[cr], tid) = own > kScCandCap ? 1 : 0;
+    }
+    __syncthreads();  // own list complete before the others may read it
+    cluster_arrive_release();
+    cluster_wait();
+    total = before = any_ovf = 0;
+    for (int c = 0; c < C; ++c) {
+      if (c < cr) before += sh.cand_cnt[c];
+      total += sh.cand_cnt[c];
+      any_ovf |= sh.ovf[c];
+    }
+    // the same decision in every CTA of the cluster
+    if (attempt == 1 || any_ovf || total >= k || rs >= nsamp) break;
+    // the rank whose expected count of keys above it lies halfway between k
+    // and the candidate capacity
+    rs = min(nsamp, max(rs + 1, static_cast<int>(ceilf(0.5f * static_cast<float>(k + kScCandCap) *
+                                                       static_cast<float>(nsamp) /
+                                                       static_cast<float>(n)))));
+    // every CTA has read this round's counts before they are overwritten
+    cluster_arrive_release();
+    cluster_wait();
   }
   const bool fast = !any_ovf && total >= k && total <= kScCandCap;
 

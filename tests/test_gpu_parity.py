@@ -151,6 +151,44 @@ def test_selection_full_search_paths(cuda_device):
     check(d, cfg.window, cfg.pool_width, cuda_device)
 
 
+def test_selection_second_sampled_bound(cuda_device):
+    """A unit whose few top keys sit where the selection samples: strong
+    needles at eleven of the sample positions of the first slice (L = 10000:
+    a cluster of 5 CTAs, 2016 positions and 51 evenly spaced samples each)
+    make the first sampled bound the 10th needle, so fewer than k = 96 keys
+    reach it and a second, looser bound is taken.  The result must equal the
+    oracle."""
+    cfg = wl.get("c1").scaled(seq_len=10000, dtype="bf16")
+    d = wl.make_layer(cfg, 0, sinks=False, needle_gain=0.0)
+    G = cfg.num_q_heads // cfg.num_kv_heads
+    slice_len, per_cta = 2016, 51
+    pos = [(t * slice_len) // per_cta for t in range(1, 12)]
+    for g in range(cfg.num_kv_heads):
+        qm = d["q_win"][0, g * G:(g + 1) * G].float().mean(dim=(0, 1))
+        key = (qm / qm.norm() * 6.0).to(d["k"].dtype)
+        for i, p in enumerate(pos):
+            d["k"][p, g] = key * (1.0 + 0.01 * i)  # distinct needle strengths
+    out, res, ties = check(d, cfg.window, cfg.pool_width, cuda_device)
+    # the construction: on the oracle's pooled scores the first bound (the
+    # r-th largest sample, r = ceil(mu + 3 sqrt(mu)) + 2) leaves fewer than k
+    # keys at or above it
+    n = 10000 - cfg.window
+    k = 128 - cfg.window
+    C = 5
+    samples = []
+    for c in range(C):
+        lo_c = min(n, c * slice_len)
+        ln = min(n, lo_c + slice_len) - lo_c
+        ns = min(256 // C, ln)
+        samples += [lo_c + (t * ln) // ns for t in range(ns)]
+    mu = k * len(samples) / n
+    r = min(len(samples), math.ceil(mu + 3 * math.sqrt(mu)) + 2)
+    for g in range(cfg.num_kv_heads):
+        pooled = res.pooled[g]
+        bound = np.sort(pooled[samples])[::-1][r - 1]
+        assert (pooled >= bound).sum() < k
+
+
 def test_strided_inputs(cuda_device):
     """K and V as views of one packed KV tensor; Q as a slice of a larger window."""
     cfg = wl.get("c1").scaled(seq_len=777, dtype="bf16", srh_per_group=(2, 2))
@@ -263,6 +301,71 @@ def test_full_size_layer(cuda_device, name, layer):
     cfg = wl.get(name)
     d = wl.make_layer(cfg, layer)
     check(d, cfg.window, cfg.pool_width, cuda_device)
+
+
+@pytest.mark.parametrize("n_layers,batch", [(2, 1), (3, 2), (4, 1)])
+def test_multi_layer_call(cuda_device, n_layers, batch):
+    """Several layers in one call (compress_layers): the layers' K/V and
+    window queries packed as one batch, one SRH mask per layer.  Every
+    layer's block of the outputs equals the oracle on that layer alone."""
+    dev = cuda_device
+    cfg = wl.get("c2").scaled(seq_len=3000, n_layers=n_layers, batch=batch)
+    lengths = wl.sequence_lengths(cfg)
+    masks = wl.srh_masks(cfg)
+    budgets = wl.layer_budgets(cfg, lengths)
+    layers = [wl.make_layer(cfg, l, lengths=lengths, masks=masks, budgets=budgets)
+              for l in range(n_layers)]
+    T = layers[0]["k"].shape[0]
+    k_all = torch.cat([lay["k"] for lay in layers]).to(dev)
+    v_all = torch.cat([lay["v"] for lay in layers]).to(dev)
+    q_all = torch.cat([lay["q_win"] for lay in layers]).to(dev)
+    cu = np.concatenate([np.asarray(lay["cu_seqlens"][:-1], np.int64) + l * T
+                         for l, lay in enumerate(layers)] + [[n_layers * T]]).astype(np.int32)
+    b_all = np.concatenate([np.asarray(lay["budgets"]).reshape(-1) for lay in layers])
+    m_all = np.stack([np.asarray(lay["srh_mask"]) for lay in layers])
+    prob = ckv.Problem(q_all, k_all, cu, cfg.window, cfg.pool_width)
+    out = ckv.LayerOutputs(prob, b_all, 128, k_all.dtype, dev)
+    ws = ckv.workspace(prob, dev)
+    cu_out = ckv.compress_layers(prob, n_layers, q_all, k_all, v_all, m_all, b_all, out.indices,
+                                 out.k_out, out.v_out, ws, raw=out.raw, pooled=out.pooled)
+    torch.cuda.synchronize()
+    assert ckv.read_device_status(ws) == 0
+    n = np.maximum(np.diff(cu) - cfg.window, 0)
+    cu_prefix = np.concatenate([[0], np.cumsum(n)])
+    raw, pooled = out.raw.cpu().numpy(), out.pooled.cpu().numpy()
+    idx = out.indices.cpu().numpy()
+    k_bits, v_bits = _bits(out.k_out), _bits(out.v_out)
+    for l, lay in enumerate(layers):
+        s0, s1 = l * batch, (l + 1) * batch
+        p0, p1 = cu_prefix[s0], cu_prefix[s1]
+        o0, o1 = cu_out[s0], cu_out[s1]
+        res = run_oracle(lay, cfg.window, cfg.pool_width)
+        assert np.array_equal(cu_out[s0:s1 + 1] - o0, res.cu_out)
+        compare.check_layer(res, raw[:, p0:p1], pooled[:, p0:p1], idx[:, o0:o1],
+                            lay["cu_seqlens"], cfg.window)
+        compare.check_scores("raw (fp16 table bound)", raw[:, p0:p1], res.raw, rtol=EXPO_RTOL,
+                             atol=1e-8)
+        compare.check_gather_bits(_bits(lay["k"]), _bits(lay["v"]), k_bits[o0:o1], v_bits[o0:o1],
+                                  idx[:, o0:o1], lay["cu_seqlens"], cu_out[s0:s1 + 1] - o0)
+
+
+def test_multi_layer_call_rejects_bad_mask_counts(cuda_device):
+    cfg = wl.get("c1").scaled(seq_len=500, batch=2)
+    d = wl.make_layer(cfg, 0, lengths=[500, 400])
+    dev = cuda_device
+    q, k, v = d["q_win"].to(dev), d["k"].to(dev), d["v"].to(dev)
+    prob = ckv.Problem(q, k, d["cu_seqlens"], cfg.window, cfg.pool_width)
+    out = ckv.LayerOutputs(prob, d["budgets"], 128, k.dtype, dev)
+    ws = ckv.workspace(prob, dev)
+    masks = np.stack([d["srh_mask"]] * 3)
+    for n_masks, code in ((3, ckv.compresskv.CKV_ERR_INVALID_ARG),   # does not divide the batch
+                          (0, ckv.compresskv.CKV_ERR_INVALID_ARG)):
+        with pytest.raises(ckv.CompressKVError) as e:
+            ckv.compress_layers(prob, n_masks, q, k, v, masks[:max(n_masks, 1)], d["budgets"],
+                                out.indices, out.k_out, out.v_out, ws)
+        assert e.value.code == code
+    torch.cuda.synchronize()
+    assert ckv.read_device_status(ws) == 0
 
 
 def test_graph_captured_multilayer_step_matches(cuda_device):
