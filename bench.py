@@ -58,10 +58,11 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-lse", action="store_true",
                     help="skip the given-LSE (log-sum-exp supplied) measurement")
-    ap.add_argument("--streams", type=int, default=3,
+    ap.add_argument("--streams", type=int, default=4,
                     help="calls in flight: call c runs on stream c %% S with its own workspace")
-    ap.add_argument("--layers-per-call", type=int, default=2,
-                    help="layers compressed by one compress_layers call (one launch per kernel)")
+    ap.add_argument("--layers-per-call", type=int, default=0,
+                    help="layers compressed by one compress_layers call (one launch per kernel); "
+                         "0 = as many (up to 4) as keep the call's exponent table in one set")
     return ap.parse_args()
 
 
@@ -173,9 +174,10 @@ def kernel_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(workload: str):
+def profiled_traffic(workload: str, layers_per_call: int):
     """DRAM bytes per launch of the scoring kernel from the committed
-    ncu summary, if it was taken on the current kernel sources."""
+    ncu summary, if it was taken on the current kernel sources with the same
+    workload and layers per call."""
     try:
         text = open(PROFILE_TRAFFIC).read()
     except OSError:
@@ -183,7 +185,9 @@ def profiled_traffic(workload: str):
     m = re.search(r"traffic_bytes_per_launch:\s*(\d+)", text)
     h = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", text)
     w = re.search(r"workload:\s*(\S+)", text)
-    if not (m and h and w) or h.group(1) != kernel_source_hash() or w.group(1) != workload:
+    c = re.search(r"layers_per_call:\s*(\d+)", text)
+    if not (m and h and w and c) or h.group(1) != kernel_source_hash() or \
+            w.group(1) != workload or int(c.group(1)) != layers_per_call:
         return None
     return int(m.group(1))
 
@@ -202,6 +206,36 @@ def build_layers(cfg, device):
     layers = [wl.make_layer(cfg, l, device=device, lengths=lengths, masks=masks, budgets=budgets)
               for l in range(cfg.n_layers)]
     return lengths, masks, budgets, layers
+
+
+# The library's exponent-table set (CKV_EXPO_SET_BYTES) and its row length
+# (query rows rounded up to a power of two >= 8): the automatic layers-per-
+# call choice packs layers while their tables fit one set.
+EXPO_SET_BYTES = 128 << 20
+MAX_LAYERS_PER_CALL = 4
+
+
+def expo_stride(rows: int) -> int:
+    r = 8
+    while r < rows:
+        r <<= 1
+    return r
+
+
+def layers_per_call(cfg, layers, lengths) -> int:
+    """Most layers (<= 4) whose exponent tables, with the actual SRH rows,
+    fit one set; 2 when a single layer's does not (it is scored in two
+    passes without a table, where pairs measured best)."""
+    G = cfg.num_q_heads // cfg.num_kv_heads
+    per_layer = []
+    for lay in layers:
+        m = np.asarray(lay["srh_mask"]).reshape(cfg.num_kv_heads, G).sum(axis=1)
+        nr = sum(expo_stride(int(c) * cfg.window) for c in m)
+        per_layer.append(2 * nr * sum(max(L - cfg.window, 0) for L in lengths))
+    worst = max(per_layer)
+    if worst > EXPO_SET_BYTES:
+        return 2
+    return max(1, min(MAX_LAYERS_PER_CALL, EXPO_SET_BYTES // worst))
 
 
 def algorithmic_bytes(cfg, layers, lengths):
@@ -254,7 +288,8 @@ def run_ours(args):
     # serialises the kernels) for the per-kernel durations.
     trace = ckv.Trace(capacity=16 * cfg.n_layers)
     counter = ckv.Trace(capacity=0)
-    lpc = max(1, args.layers_per_call)
+    lpc = args.layers_per_call if args.layers_per_call > 0 else layers_per_call(cfg, layers,
+                                                                                  lengths)
     calls = [(l0, min(l0 + lpc, cfg.n_layers)) for l0 in range(0, cfg.n_layers, lpc)]
 
     def call_problem(l0, l1, tr):
@@ -385,7 +420,7 @@ def run_ours(args):
                 "timing": f"CUDA events around each launch in a traced replay of the step "
                           f"({n_traced} steps, {traced_ms_per_step:.3f} ms/step serialised); the "
                           "timed step overlaps consecutive kernels",
-                "traffic": profiled_traffic(cfg.name)}
+                "traffic": profiled_traffic(cfg.name, lpc)}
     path_gbs = step_bytes / (ms_per_step / 1e3) / 1e9
     kernels = {k: {"launches_per_step": len(v), "avg_us": round(1e3 * sum(v) / len(v), 2),
                    "total_us_per_step": round(1e3 * sum(v), 1)} for k, v in per_kind.items()}

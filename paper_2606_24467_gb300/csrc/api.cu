@@ -24,12 +24,15 @@ namespace {
 // last-CTA-per-unit merge resets the tickets it uses).
 constexpr size_t kTicketOffset = 256;
 constexpr size_t kStatusBytes = kTicketOffset + static_cast<size_t>(kMaxItems) * sizeof(int);
-// Units are scored in sets whose exponent tables (bounded with every head of
-// a group counted as SRH) take at most this many bytes; one set's table is
-// written by the scoring kernel and read back by the combine kernel, ideally
-// while still in L2.
+// Units are scored in sets whose exponent tables take at most this many
+// bytes; one set's table is written by the scoring kernel and read back by
+// the combine kernel while (mostly) still in the 126 MB L2.  The workspace
+// reserves a set bounded with every head of a group counted as SRH; a call
+// packs its sets with the actual SRH rows.  Measured on GB300: 128 MiB sets
+// (four bench layers per call, ~100 MB of table) beat 64 MiB sets, and one
+// L=128K layer (~100 MB) runs as fast with its table as in two passes.
 #ifndef CKV_EXPO_SET_BYTES
-#define CKV_EXPO_SET_BYTES (64ll << 20)
+#define CKV_EXPO_SET_BYTES (128ll << 20)
 #endif
 constexpr long long kExpoSetBytes = CKV_EXPO_SET_BYTES;
 constexpr size_t kPartialBytes = static_cast<size_t>(kMaxItems) * kMaxQRows * sizeof(float2);
