@@ -556,17 +556,18 @@ int run_score(const ckv_problem* p, const Info& I, const void* q_win, const void
       if (best < 0) break;
       ++cnt[best];
     }
-    // Combine items: chunks of 32-token quarters, about two CTAs per SM (measured
-    // best of 2, 3 and 4 per SM),
-    // balanced by bytes: a quarter of a unit with exponent rows of nr
-    // columns weighs nr + 16 (table bytes plus a fixed share per key).
+    // Combine items: chunks of 32-token quarters, about three CTAs per SM
+    // (measured: 3 and 4 per SM best for four-layer calls, 2, 3 and 4 within
+    // 0.5% of each other for one-layer calls), balanced by bytes: a quarter
+    // of a unit with exponent rows of nr columns weighs nr + 16 (table bytes
+    // plus a fixed share per key).
     constexpr int kQuarterFixed = 16;
     long long weight = 0;
     for (int u = 0; u < nu; ++u)
       if (cnt[u] > 0)
         weight += static_cast<long long>(units[u0 + u].quarters) *
                   (expo_stride(S.rows[units[u0 + u].v]) + kQuarterFixed);
-    const long long ctarget = std::max(1, std::min(kMaxItems - nu, 2 * F->sms));
+    const long long ctarget = std::max(1, std::min(kMaxItems - nu, 3 * F->sms));
     const long long per_chunk = std::max<long long>(8 * (8 + kQuarterFixed),
                                                     (weight + ctarget - 1) / ctarget);
     std::vector<int> chunk_q(nu, 1);
