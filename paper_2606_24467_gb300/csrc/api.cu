@@ -716,11 +716,17 @@ int run_select(const ckv_problem* p, const Info& I, const float* raw, const floa
     if (s < I.B) max_n = std::max(max_n, I.n[s]);
   }
   if (pooled_in && !I.layer && max_n <= 32 * 1024) {
-    // fused layer call, per-group selection: sampled select, a cluster of up
-    // to 16 CTAs per unit with about kScTargetSlice positions each (longer
-    // prefixes list too many keys above the sampled bound)
-    const int C = std::min(F->sampled_cluster,
-                           std::max(1, (max_n + kScTargetSlice - 1) / kScTargetSlice));
+    // fused layer call, per-group selection: sampled select, one cluster of
+    // C CTAs per unit (longer prefixes list too many keys above the sampled
+    // bound).  C gives about kScTargetCtas CTAs per launch -- few, busy CTAs
+    // leave the SMs to the other calls' kernels (measured on the 32-layer
+    // bench: 8 units per launch best with C = 8 of 4/8/16, 32 units with
+    // C = 2-4 of 2-16) -- but at least slices of kScMaxSlice positions and
+    // at most the device's cluster limit.
+    const int units = I.B * I.Hkv;
+    const int c_min = (max_n + kScMaxSlice - 1) / kScMaxSlice;
+    const int C = std::max(std::max(1, c_min),
+                           std::min(F->sampled_cluster, (kScTargetCtas + units - 1) / units));
     const int S = std::max(32, ((max_n + C - 1) / C + 31) / 32 * 32);
     if (S <= kScMaxSlice) {
       P.cluster = C;

@@ -153,7 +153,8 @@ cudaError_t launch_select(const SelectParams& p, int n_units, size_t smem, cudaS
 // Per-group selection from pooled scores by sampling (clusters of up to 16
 // CTAs, `p.slice` <= kScMaxSlice positions per CTA).
 constexpr int kScMaxSlice = 16384;
-constexpr int kScTargetSlice = 2048;  // positions per CTA when the cluster allows
+constexpr int kScTargetSlice = 2048;  // slice of the cluster-size occupancy query
+constexpr int kScTargetCtas = 80;     // CTAs per sampled-select launch to aim for
 cudaError_t launch_select_sampled(const SelectParams& p, int n_units, size_t smem, cudaStream_t s);
 size_t select_sampled_smem_bytes(int slice);
 int select_sampled_max_cluster(int slice);  // 16 when the device takes such clusters, else 8

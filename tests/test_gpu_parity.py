@@ -153,15 +153,15 @@ def test_selection_full_search_paths(cuda_device):
 
 def test_selection_second_sampled_bound(cuda_device):
     """A unit whose few top keys sit where the selection samples: strong
-    needles at eleven of the sample positions of the first slice (L = 10000:
-    a cluster of 5 CTAs, 2016 positions and 51 evenly spaced samples each)
-    make the first sampled bound the 10th needle, so fewer than k = 96 keys
-    reach it and a second, looser bound is taken.  The result must equal the
-    oracle."""
+    needles at eleven of the sample positions of the first slice (L = 10000,
+    8 units: a cluster of 10 CTAs -- about 80 CTAs per launch --, 1024
+    positions and 25 evenly spaced samples each) make the first sampled
+    bound the 10th needle, so fewer than k = 96 keys reach it and a second,
+    looser bound is taken.  The result must equal the oracle."""
     cfg = wl.get("c1").scaled(seq_len=10000, dtype="bf16")
     d = wl.make_layer(cfg, 0, sinks=False, needle_gain=0.0)
     G = cfg.num_q_heads // cfg.num_kv_heads
-    slice_len, per_cta = 2016, 51
+    C, slice_len, per_cta = 10, 1024, 25
     pos = [(t * slice_len) // per_cta for t in range(1, 12)]
     for g in range(cfg.num_kv_heads):
         qm = d["q_win"][0, g * G:(g + 1) * G].float().mean(dim=(0, 1))
@@ -174,7 +174,6 @@ def test_selection_second_sampled_bound(cuda_device):
     # keys at or above it
     n = 10000 - cfg.window
     k = 128 - cfg.window
-    C = 5
     samples = []
     for c in range(C):
         lo_c = min(n, c * slice_len)
