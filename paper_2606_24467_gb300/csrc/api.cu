@@ -737,11 +737,17 @@ int run_select(const ckv_problem* p, const Info& I, const float* raw, const floa
                     [&] { return launch_select_sampled(P, I.B * I.Hkv, smem, stream); });
     }
   }
-  // A cluster of up to 8 CTAs per unit, about 4096 prefix tokens per CTA
-  // (one CTA per unit is several times slower: the four radix passes over a
-  // whole unit's keys serialise in one block).
+  // A cluster of up to 8 CTAs per unit (one CTA per unit is several times
+  // slower: the four radix passes over a whole unit's keys serialise in one
+  // block), at least 4096 prefix tokens and at most 16384 per CTA, and about
+  // 80 CTAs per launch where the units allow: few, busy clusters leave the
+  // SMs to the other calls' kernels (the ragged and 80-layer workloads ran
+  // 12-13% faster with C = 4 and 2 than with 8).
   const int r = (I.P - 1) / 2;
-  const int C = std::min(8, std::max(1, (max_n + 4095) / 4096));
+  const int n_units = I.layer ? I.B : I.B * I.Hkv;
+  const int C = std::min(8, std::max(std::max(1, (max_n + 16383) / 16384),
+                                     std::min((max_n + 4095) / 4096,
+                                              (kScTargetCtas + n_units - 1) / n_units)));
   const int S = std::max(32, ((max_n + C - 1) / C + 31) / 32 * 32);
   const int need = pooled_in ? S : 2 * S + 2 * r;  // floats of shared memory
   const bool fits = need <= select_max_smem_floats();
@@ -750,7 +756,6 @@ int run_select(const ckv_problem* p, const Info& I, const float* raw, const floa
   P.smem_slice = fits ? 1 : 0;
   const size_t smem = fits ? static_cast<size_t>(need) * 4 : 0;
   Tracer tr{p->trace, stream};
-  const int n_units = I.layer ? I.B : I.B * I.Hkv;
   return traced(tr, CKV_KERNEL_SELECT, [&] { return launch_select(P, n_units, smem, stream); });
 }
 
