@@ -112,6 +112,49 @@ def test_compress_layer_host_errors():
     assert call(big, budgets_ptr=bp3, wsn=ckv.workspace_size(prob)) == B.CKV_ERR_UNSUPPORTED
 
 
+def test_compress_layers_host_errors():
+    """The multi-layer call checks its mask count against the packed batch
+    and each mask's groups against its own block of sequences."""
+    lib = ckv.load()
+    prob, q, k = _problem()  # batch 2: two one-sequence blocks
+    vp = ctypes.c_void_p
+    ws = vp(_fake_dev_ptr())
+    n = ckv.workspace_size(prob)
+    mask_ok = np.zeros(8, np.uint8)
+    mask_ok[[1, 6]] = 1
+    mask_empty = np.zeros(8, np.uint8)
+    mask_empty[1] = 1  # group 1 (heads 4-7) has no SRH head
+    bud, bp = B._i32([64, 64])
+    cu_out = (ctypes.c_int32 * 3)()
+
+    def call(n_masks, masks, p=prob, budgets_ptr=bp, wsn=n):
+        m = np.ascontiguousarray(np.stack(masks))
+        return lib.compresskv_compress_layers(
+            p.ref, n_masks, vp(1 << 30), vp(1 << 30), vp(1 << 30), vp(m.ctypes.data),
+            budgets_ptr, vp(1 << 30), cu_out, vp(1 << 30), vp(1 << 30), None, None, ws, wsn,
+            None)
+
+    assert call(0, [mask_ok]) == B.CKV_ERR_INVALID_ARG
+    assert call(3, [mask_ok] * 3) == B.CKV_ERR_INVALID_ARG   # 3 does not divide batch 2
+    assert call(2, [mask_ok, mask_empty]) == B.CKV_ERR_EMPTY_SRH_GROUP  # second block
+    assert call(2, [mask_empty, mask_ok]) == B.CKV_ERR_EMPTY_SRH_GROUP  # first block
+    # one mask for both sequences is the single-layer call: the empty group fails too
+    assert call(1, [mask_empty]) == B.CKV_ERR_EMPTY_SRH_GROUP
+    p5, _, _ = _problem(L=(100,) * 5)
+    b5, bp5 = B._i32([64] * 5)
+    cu_out = (ctypes.c_int32 * 6)()
+    assert call(5, [mask_ok] * 5, p=p5, budgets_ptr=bp5,
+                wsn=ckv.workspace_size(p5)) == B.CKV_ERR_UNSUPPORTED  # more than 4 masks
+
+
+def test_compress_layers_binding_checks_mask_shape():
+    prob, q, k = _problem()
+    with pytest.raises(ckv.CompressKVError) as e:
+        ckv.compress_layers(prob, 2, q, k, k, np.ones((3, 8), np.uint8), [64, 64], k, k, k,
+                            torch.zeros(16, dtype=torch.uint8))
+    assert e.value.code == B.CKV_ERR_INVALID_ARG
+
+
 def test_selection_scope_validation():
     lib = ckv.load()
     prob, q, k = _problem()
