@@ -730,7 +730,10 @@ def run_reference(args):
         "ms_per_step": round(step_ms, 1), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic (same seeded generator)",
         "config": {"workload": cfg.name, "layers": cfg.n_layers, "batch": cfg.batch,
-                   "window": cfg.window, "pool_width": cfg.pool_width},
+                   "seq_len": cfg.seq_len if cfg.length_range is None else "ragged",
+                   "q_heads": cfg.num_q_heads, "kv_heads": cfg.num_kv_heads,
+                   "head_dim": cfg.head_dim, "window": cfg.window,
+                   "pool_width": cfg.pool_width},
         "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": cpu_cores(),
                          "kind": "oracle",
                          "sample": f"each step = 1 unit (1 sequence x 1 KV group, L={lengths[0]}) "
