@@ -249,6 +249,19 @@ int compresskv_compress_layer_lse(const ckv_problem* p, const void* q_win, const
                                   float* pooled_scores, void* workspace, size_t workspace_bytes,
                                   void* stream);
 
+/* compresskv_compress_layer_lse for several layers in one call: the packed
+ * batch, the per-block SRH masks and the outputs as for
+ * compresskv_compress_layers, and the window queries' LSE packed the same
+ * way (element (s, h, w) of the packed batch at
+ * lse_win + s*lse_batch_stride + h*lse_head_stride + w). */
+int compresskv_compress_layers_lse(const ckv_problem* p, int n_masks, const void* q_win,
+                                   const void* k, const void* v, const float* lse_win,
+                                   int64_t lse_batch_stride, int64_t lse_head_stride,
+                                   const uint8_t* srh_masks, const int32_t* budgets,
+                                   int32_t* indices, int32_t* cu_out, void* k_out, void* v_out,
+                                   float* raw_scores, float* pooled_scores, void* workspace,
+                                   size_t workspace_bytes, void* stream);
+
 /* compresskv_compress_layer with a budget per (sequence, KV group) -- the
  * head-level allocation CompressKV's token selection combines with (Sec.
  * 4.6, HeadKV / AdaKV style budgets, computed elsewhere).  Per-group

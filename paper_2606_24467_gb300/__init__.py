@@ -17,6 +17,7 @@ from .compresskv import (  # noqa: F401
     compress_layer_lse,
     compress_layer_noalloc,
     compress_layers,
+    compress_layers_lse,
     gather,
     head_budget_layout,
     load,

@@ -45,6 +45,7 @@ EXPORTED = (
     "compresskv_compress_layers",
     "compresskv_compress_layer_noalloc",
     "compresskv_compress_layer_lse",
+    "compresskv_compress_layers_lse",
     "compresskv_compress_layer_head_budgets",
     "compresskv_read_device_status",
     "compresskv_allocate_layer_budgets",
@@ -108,6 +109,9 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
                                                          vp, vp, vp, vp, vp]),
         "compresskv_compress_layer_lse": (c_int32, [pp, vp, vp, vp, vp, c_int64, c_int64, vp, i32p,
                                                      vp, i32p, vp, vp, vp, vp, vp, c_size_t, vp]),
+        "compresskv_compress_layers_lse": (c_int32, [pp, c_int32, vp, vp, vp, vp, c_int64,
+                                                      c_int64, vp, i32p, vp, i32p, vp, vp, vp,
+                                                      vp, vp, c_size_t, vp]),
         "compresskv_compress_layer_head_budgets": (c_int32, [pp, vp, vp, vp, vp, i32p, vp, i32p,
                                                               vp, vp, vp, vp, vp, c_size_t, vp]),
         "compresskv_read_device_status": (c_int32, [vp, vp, i32p]),
@@ -354,6 +358,26 @@ def compress_layer_lse(problem: Problem, q_win, k, v, lse_win, srh_mask, budgets
         lse_win.stride(1), mp, bp, _ptr(indices), cu_out.ctypes.data_as(POINTER(c_int32)),
         _ptr(k_out), _ptr(v_out), _ptr(raw), _ptr(pooled), _ptr(ws), ws.numel(), _stream(stream)),
         "compresskv_compress_layer_lse")
+    return cu_out
+
+
+def compress_layers_lse(problem: Problem, n_masks: int, q_win, k, v, lse_win, srh_masks, budgets,
+                        indices, k_out, v_out, ws, raw=None, pooled=None,
+                        stream=None) -> np.ndarray:
+    """compress_layers with the window queries' log-sum-exp given, packed like
+    the batch: ``lse_win`` is float32 ``[n_layers*B, H_q, W]``."""
+    if lse_win.dtype != torch.float32 or lse_win.stride(2) != 1:
+        raise CompressKVError(CKV_ERR_INVALID_ARG, "lse_win must be float32 with contiguous rows")
+    m = np.ascontiguousarray(np.asarray(srh_masks).astype(np.uint8).reshape(-1))
+    if n_masks >= 1 and m.size != int(n_masks) * int(problem.struct.num_q_heads):
+        raise CompressKVError(CKV_ERR_INVALID_ARG, "srh_masks must be [n_masks, num_q_heads]")
+    b, bp = _i32(budgets)
+    cu_out = np.zeros(problem.batch + 1, np.int32)
+    _check(load().compresskv_compress_layers_lse(
+        problem.ref, int(n_masks), _ptr(q_win), _ptr(k), _ptr(v), _ptr(lse_win),
+        lse_win.stride(0), lse_win.stride(1), c_void_p(m.ctypes.data), bp, _ptr(indices),
+        cu_out.ctypes.data_as(POINTER(c_int32)), _ptr(k_out), _ptr(v_out), _ptr(raw),
+        _ptr(pooled), _ptr(ws), ws.numel(), _stream(stream)), "compresskv_compress_layers_lse")
     return cu_out
 
 

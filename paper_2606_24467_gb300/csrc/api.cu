@@ -927,9 +927,27 @@ int compresskv_compress_layer_lse(const ckv_problem* p, const void* q_win, const
                                   void* k_out, void* v_out, float* raw_scores,
                                   float* pooled_scores, void* workspace, size_t workspace_bytes,
                                   void* stream) {
+  return compresskv_compress_layers_lse(p, 1, q_win, k, v, lse_win, lse_batch_stride,
+                                        lse_head_stride, srh_mask, budgets, indices, cu_out,
+                                        k_out, v_out, raw_scores, pooled_scores, workspace,
+                                        workspace_bytes, stream);
+}
+
+int compresskv_compress_layers_lse(const ckv_problem* p, int n_masks, const void* q_win,
+                                   const void* k, const void* v, const float* lse_win,
+                                   int64_t lse_batch_stride, int64_t lse_head_stride,
+                                   const uint8_t* srh_masks, const int32_t* budgets,
+                                   int32_t* indices, int32_t* cu_out, void* k_out, void* v_out,
+                                   float* raw_scores, float* pooled_scores, void* workspace,
+                                   size_t workspace_bytes, void* stream) {
   Info I;
   int rc = validate(p, I);
   if (rc != CKV_OK) return rc;
+  if (n_masks < 1 || I.B % n_masks != 0) return CKV_ERR_INVALID_ARG;
+  if (n_masks > kMaxMasks) return CKV_ERR_UNSUPPORTED;
+  I.n_masks = n_masks;
+  I.spm = I.B / n_masks;
+  const uint8_t* srh_mask = srh_masks;
   if (!lse_win || lse_batch_stride < 0 || lse_head_stride < 0) return CKV_ERR_INVALID_ARG;
   if (reinterpret_cast<uintptr_t>(lse_win) & 3u) return CKV_ERR_INVALID_ARG;
   std::vector<int> co;

@@ -87,3 +87,56 @@ def test_lse_path_layer_scope(cuda_device):
         unit = oracle.compresskv_oracle.UnitResult([], np.zeros(0), sh.pooled, sh.k, sh.tau,
                                                    sh.indices)
         compare.check_unit_indices(idx[0, o0:o1], unit, L, cfg.window)
+
+
+@pytest.mark.parametrize("n_layers,batch", [(2, 1), (3, 2)])
+def test_lse_path_multi_layer(cuda_device, n_layers, batch):
+    """Several layers in one given-LSE call (compress_layers_lse): each
+    layer's block of the outputs against the oracle on that layer."""
+    dev = cuda_device
+    cfg = wl.get("c2").scaled(seq_len=2000, n_layers=n_layers, batch=batch)
+    lengths = wl.sequence_lengths(cfg)
+    masks = wl.srh_masks(cfg)
+    budgets = wl.layer_budgets(cfg, lengths)
+    layers = [wl.make_layer(cfg, l, lengths=lengths, masks=masks, budgets=budgets)
+              for l in range(n_layers)]
+    T = layers[0]["k"].shape[0]
+    lse = torch.cat([torch.tensor(oracle.window_lse(lay["q_win"].float().numpy(),
+                                                    lay["k"].float().numpy(),
+                                                    lay["cu_seqlens"], cfg.window),
+                                  dtype=torch.float32) for lay in layers]).to(dev)
+    k_all = torch.cat([lay["k"] for lay in layers]).to(dev)
+    v_all = torch.cat([lay["v"] for lay in layers]).to(dev)
+    q_all = torch.cat([lay["q_win"] for lay in layers]).to(dev)
+    cu = np.concatenate([np.asarray(lay["cu_seqlens"][:-1], np.int64) + l * T
+                         for l, lay in enumerate(layers)] + [[n_layers * T]]).astype(np.int32)
+    b_all = np.concatenate([np.asarray(lay["budgets"]).reshape(-1) for lay in layers])
+    m_all = np.stack([np.asarray(lay["srh_mask"]) for lay in layers])
+    prob = ckv.Problem(q_all, k_all, cu, cfg.window, cfg.pool_width)
+    out = ckv.LayerOutputs(prob, b_all, 128, k_all.dtype, dev)
+    ws = ckv.workspace(prob, dev)
+    cu_out = ckv.compress_layers_lse(prob, n_layers, q_all, k_all, v_all, lse, m_all, b_all,
+                                     out.indices, out.k_out, out.v_out, ws, raw=out.raw,
+                                     pooled=out.pooled)
+    torch.cuda.synchronize()
+    assert ckv.read_device_status(ws) == 0
+    n = np.maximum(np.diff(cu) - cfg.window, 0)
+    cu_prefix = np.concatenate([[0], np.cumsum(n)])
+    raw, pooled = out.raw.cpu().numpy(), out.pooled.cpu().numpy()
+    idx = out.indices.cpu().numpy()
+    k_bits, v_bits = _bits(out.k_out), _bits(out.v_out)
+    for l, lay in enumerate(layers):
+        s0, s1 = l * batch, (l + 1) * batch
+        p0, p1 = cu_prefix[s0], cu_prefix[s1]
+        o0, o1 = cu_out[s0], cu_out[s1]
+        res = oracle.compress_layer(lay["q_win"].float().numpy(), lay["k"].float().numpy(),
+                                    lay["v"].float().numpy(), lay["cu_seqlens"],
+                                    lay["srh_mask"], lay["budgets"], cfg.window,
+                                    cfg.pool_width)
+        assert np.array_equal(cu_out[s0:s1 + 1] - o0, res.cu_out)
+        compare.check_scores("raw", raw[:, p0:p1], res.raw, rtol=RTOL, atol=1e-8)
+        compare.check_layer(res, raw[:, p0:p1], pooled[:, p0:p1], idx[:, o0:o1],
+                            lay["cu_seqlens"], cfg.window)
+        compare.check_gather_bits(_bits(lay["k"]), _bits(lay["v"]), k_bits[o0:o1],
+                                  v_bits[o0:o1], idx[:, o0:o1], lay["cu_seqlens"],
+                                  cu_out[s0:s1 + 1] - o0)
