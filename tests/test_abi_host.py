@@ -147,6 +147,32 @@ def test_compress_layers_host_errors():
                 wsn=ckv.workspace_size(p5)) == B.CKV_ERR_UNSUPPORTED  # more than 4 masks
 
 
+def test_compress_layers_lse_host_errors():
+    lib = ckv.load()
+    prob, q, k = _problem()
+    vp = ctypes.c_void_p
+    ws = vp(_fake_dev_ptr())
+    n = ckv.workspace_size(prob)
+    mask_ok = np.zeros(8, np.uint8)
+    mask_ok[[1, 6]] = 1
+    mask_empty = np.zeros(8, np.uint8)
+    mask_empty[1] = 1
+    bud, bp = B._i32([64, 64])
+    cu_out = (ctypes.c_int32 * 3)()
+
+    def call(n_masks, masks, lse=vp(1 << 30)):
+        m = np.ascontiguousarray(np.stack(masks))
+        return lib.compresskv_compress_layers_lse(
+            prob.ref, n_masks, vp(1 << 30), vp(1 << 30), vp(1 << 30), lse, 8 * 32, 32,
+            vp(m.ctypes.data), bp, vp(1 << 30), cu_out, vp(1 << 30), vp(1 << 30), None, None,
+            ws, n, None)
+
+    assert call(0, [mask_ok]) == B.CKV_ERR_INVALID_ARG
+    assert call(3, [mask_ok] * 3) == B.CKV_ERR_INVALID_ARG
+    assert call(2, [mask_ok, mask_ok], lse=vp(None)) == B.CKV_ERR_INVALID_ARG
+    assert call(2, [mask_ok, mask_empty]) == B.CKV_ERR_EMPTY_SRH_GROUP
+
+
 def test_compress_layers_binding_checks_mask_shape():
     prob, q, k = _problem()
     with pytest.raises(ckv.CompressKVError) as e:
