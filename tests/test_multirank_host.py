@@ -1,0 +1,64 @@
+"""The bench's N > 1 path on CPU: two ranks over gloo (replicas only -- the
+path has no collective, the bench only takes the max time over ranks and
+barriers around the timed region), and the reference arm under torchrun,
+where rank 0 alone prints its line."""
+import json
+import os
+import socket
+import subprocess
+import sys
+
+import torch
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port() -> int:
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, out):
+    os.environ.update(RANK=str(rank), WORLD_SIZE=str(world), LOCAL_RANK=str(rank),
+                      MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    sys.path.insert(0, ROOT)
+    import bench
+
+    r, w, lr = bench.dist_env()
+    assert (r, w, lr) == (rank, world, rank)
+    dist = bench.init_dist(w, "gloo")
+    bench.barrier(dist)
+    m = bench.reduce_max(dist, 1.5 + rank, torch.device("cpu"))
+    bench.barrier(dist)
+    out[rank] = m
+    dist.destroy_process_group()
+
+
+def test_two_ranks_reduce_max_and_barrier():
+    world = 2
+    out = mp.Manager().dict()
+    mp.spawn(_rank_main, args=(world, _free_port(), out), nprocs=world, join=True)
+    assert dict(out) == {0: 2.5, 1: 2.5}
+
+
+def test_single_rank_needs_no_process_group():
+    sys.path.insert(0, ROOT)
+    import bench
+
+    assert bench.init_dist(1, "gloo") is None
+    assert bench.reduce_max(None, 3.25, torch.device("cpu")) == 3.25
+
+
+def test_reference_arm_under_torchrun_prints_once():
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
+           "--master-addr", "127.0.0.1", "--master-port", str(_free_port()),
+           os.path.join(ROOT, "bench.py"), "--impl", "reference", "--gpus", "2",
+           "--workload", "c1", "--steps", "1", "--warmup", "1"]
+    res = subprocess.run(cmd, capture_output=True, text=True, timeout=300, cwd=ROOT)
+    assert res.returncode == 0, res.stderr[-2000:]
+    lines = [l for l in res.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["value"] > 0 and d["n_gpus"] == 2
