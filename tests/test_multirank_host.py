@@ -38,7 +38,7 @@ def _rank_main(rank, world, port, out):
 
 def test_two_ranks_reduce_max_and_barrier():
     world = 2
-    out = mp.Manager().dict()
+    out = mp.get_context("spawn").Manager().dict()
     mp.spawn(_rank_main, args=(world, _free_port(), out), nprocs=world, join=True)
     assert dict(out) == {0: 2.5, 1: 2.5}
 
