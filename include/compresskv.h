@@ -237,7 +237,9 @@ int compresskv_compress_layers(const ckv_problem* p, int n_masks, const void* q_
  * lse_win: device float, natural-log LSE of each window query's causal
  *   softmax over keys j <= L_s - W + w with the problem's scale: element
  *   (s, h, w) at lse_win + s*lse_batch_stride + h*lse_head_stride + w (4-byte
- *   aligned; only SRH heads are read).  Scores are then exp(z - LSE) summed
+ *   aligned; only SRH heads are read).  It must be device (or managed) memory
+ *   of the current device covering every (s, h, w) of the batch: host memory
+ *   is refused with CKV_ERR_INVALID_ARG.  Scores are then exp(z - LSE) summed
  *   in fp32 straight from the logits (no fp16 table), so their accuracy is
  *   the given LSE's.  Other arguments as for compresskv_compress_layer
  *   (pooled_scores must be NULL under CKV_SELECT_PER_LAYER). */
@@ -296,7 +298,10 @@ int compresskv_compress_layer_head_budgets(const ckv_problem* p, const void* q_w
  * - A problem whose compresskv_workspace_size exceeds CKV_STATIC_SCRATCH_BYTES
  *   is rejected with CKV_ERR_STATIC_SCRATCH before anything is enqueued.
  * - The first call on a device looks up the array's device address (with that
- *   device current); make that first call before any stream capture.
+ *   device current); make that first call before any stream capture.  The
+ *   address is looked up again when the device's context has changed (after
+ *   cudaDeviceReset): the first call after a reset, too, belongs before any
+ *   capture.
  * - Every call on a device shares the one array, which keeps the last call's
  *   contents: calls whose work may overlap on the GPU (different streams,
  *   different host threads) race and must be serialised by the caller.
@@ -313,7 +318,6 @@ int compresskv_compress_layer_noalloc(const ckv_problem* p, const void* q_win, c
  * CKV_OK (or CKV_ERR_CUDA if the copy fails). */
 int compresskv_read_device_status(const void* workspace, void* stream, int32_t* status);
 
-/* Static text for a status code. */
 /* Error-aware layer budgets (Sec. 3.4: the offline per-layer eviction
  * errors, normalised as in Eq. 4, share the total budget after every layer
  * gets a minimum m, no layer above a maximum M; Sec. 4 uses m = 32 and
@@ -333,6 +337,7 @@ int compresskv_allocate_layer_budgets(const double* layer_errors, int32_t n_laye
                                       int64_t total_budget, int32_t min_budget,
                                       int32_t max_budget, int32_t* budgets);
 
+/* Static text for a status code. */
 const char* compresskv_status_string(int status);
 
 #ifdef __cplusplus

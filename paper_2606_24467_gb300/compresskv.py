@@ -257,13 +257,31 @@ def output_layout(problem: Problem, budgets):
     return cu_prefix, cu_out
 
 
-def _mask(srh_mask):
-    m = np.ascontiguousarray(np.asarray(srh_mask).astype(np.uint8))
+def _mask(srh_mask, problem: "Problem"):
+    """One layer's SRH mask as host bytes; the library reads num_q_heads of them."""
+    m = np.ascontiguousarray(np.asarray(srh_mask).astype(np.uint8).reshape(-1))
+    if m.size != int(problem.struct.num_q_heads):
+        raise CompressKVError(CKV_ERR_INVALID_ARG, "srh_mask must have num_q_heads entries")
     return m, c_void_p(m.ctypes.data)
 
 
+def _check_lse(problem: "Problem", lse_win, k, rows: int):
+    """lse_win must be a float32 device tensor on K's device, [rows, H_q, W]
+    with contiguous window rows: the scoring kernel reads every (sequence,
+    SRH head, window row) element through the given strides."""
+    W = int(problem.struct.window)
+    shape = (int(rows), int(problem.struct.num_q_heads), W)
+    if (not isinstance(lse_win, torch.Tensor) or lse_win.dtype != torch.float32
+            or not lse_win.is_cuda or lse_win.device != k.device or tuple(lse_win.shape) != shape
+            or lse_win.stride(2) != 1 or (shape[1] > 1 and lse_win.stride(1) < W)
+            or (shape[0] > 1 and lse_win.stride(0) < 1)):
+        raise CompressKVError(CKV_ERR_INVALID_ARG,
+                              f"lse_win must be a float32 CUDA tensor on K's device of shape "
+                              f"{shape} with contiguous window rows")
+
+
 def score(problem: Problem, q_win, k, srh_mask, raw, ws, stream=None):
-    m, mp = _mask(srh_mask)
+    m, mp = _mask(srh_mask, problem)
     _check(load().compresskv_score(problem.ref, _ptr(q_win), _ptr(k), mp, _ptr(raw), _ptr(ws),
                                    ws.numel(), _stream(stream)), "compresskv_score")
 
@@ -286,7 +304,7 @@ def gather(problem: Problem, indices, cu_out, k, v, k_out, v_out, ws=None, strea
 
 def compress_layer(problem: Problem, q_win, k, v, srh_mask, budgets, indices, k_out, v_out, ws,
                    raw=None, pooled=None, stream=None) -> np.ndarray:
-    m, mp = _mask(srh_mask)
+    m, mp = _mask(srh_mask, problem)
     b, bp = _i32(budgets)
     cu_out = np.zeros(problem.batch + 1, np.int32)
     _check(load().compresskv_compress_layer(
@@ -321,7 +339,7 @@ def compress_layer_noalloc(problem: Problem, q_win, k, v, srh_mask, budgets, ind
                            stream=None) -> np.ndarray:
     """compress_layer without a workspace: the library's static scratch is
     used (for callers that cannot allocate device memory)."""
-    m, mp = _mask(srh_mask)
+    m, mp = _mask(srh_mask, problem)
     b, bp = _i32(budgets)
     cu_out = np.zeros(problem.batch + 1, np.int32)
     _check(load().compresskv_compress_layer_noalloc(
@@ -348,9 +366,8 @@ def compress_layer_lse(problem: Problem, q_win, k, v, lse_win, srh_mask, budgets
                        v_out, ws, raw=None, pooled=None, stream=None) -> np.ndarray:
     """compress_layer with the window queries' log-sum-exp given:
     ``lse_win`` is a float32 ``[B, H_q, W]`` tensor (window rows contiguous)."""
-    if lse_win.dtype != torch.float32 or lse_win.stride(2) != 1:
-        raise CompressKVError(CKV_ERR_INVALID_ARG, "lse_win must be float32 with contiguous rows")
-    m, mp = _mask(srh_mask)
+    _check_lse(problem, lse_win, k, problem.batch)
+    m, mp = _mask(srh_mask, problem)
     b, bp = _i32(budgets)
     cu_out = np.zeros(problem.batch + 1, np.int32)
     _check(load().compresskv_compress_layer_lse(
@@ -366,8 +383,7 @@ def compress_layers_lse(problem: Problem, n_masks: int, q_win, k, v, lse_win, sr
                         stream=None) -> np.ndarray:
     """compress_layers with the window queries' log-sum-exp given, packed like
     the batch: ``lse_win`` is float32 ``[n_layers*B, H_q, W]``."""
-    if lse_win.dtype != torch.float32 or lse_win.stride(2) != 1:
-        raise CompressKVError(CKV_ERR_INVALID_ARG, "lse_win must be float32 with contiguous rows")
+    _check_lse(problem, lse_win, k, problem.batch)
     m = np.ascontiguousarray(np.asarray(srh_masks).astype(np.uint8).reshape(-1))
     if n_masks >= 1 and m.size != int(n_masks) * int(problem.struct.num_q_heads):
         raise CompressKVError(CKV_ERR_INVALID_ARG, "srh_masks must be [n_masks, num_q_heads]")
@@ -403,7 +419,7 @@ def compress_layer_head_budgets(problem: Problem, q_win, k, v, srh_mask, group_b
     """compress_layer with a budget per (sequence, KV group): ``group_budgets``
     is ``[B, H_kv]``; outputs are packed group-major (see head_budget_layout);
     returns cu_out ``[H_kv, B+1]``."""
-    m, mp = _mask(srh_mask)
+    m, mp = _mask(srh_mask, problem)
     b, bp = _i32(np.asarray(group_budgets).reshape(-1))
     cu_out = np.zeros((problem.num_kv_heads, problem.batch + 1), np.int32)
     _check(load().compresskv_compress_layer_head_budgets(

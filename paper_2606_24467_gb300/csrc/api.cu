@@ -128,6 +128,21 @@ int device_readable(const void* ptr, const void** dev) {
   return CKV_ERR_INVALID_ARG;
 }
 
+// Device (or managed) memory of the current device: what a kernel may read
+// through a plain pointer.  Host memory of any kind is refused.
+int device_memory(const void* ptr) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, ptr) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return CKV_ERR_INVALID_ARG;
+  }
+  if (a.type == cudaMemoryTypeManaged) return CKV_OK;
+  int dev = -1;
+  if (a.type != cudaMemoryTypeDevice || cudaGetDevice(&dev) != cudaSuccess || a.device != dev)
+    return CKV_ERR_INVALID_ARG;
+  return CKV_OK;
+}
+
 int validate(const ckv_problem* p, Info& I) {
   if (!p || !p->cu_seqlens) return CKV_ERR_INVALID_ARG;
   if (p->batch < 1 || p->batch > kMaxBatch) return CKV_ERR_UNSUPPORTED;
@@ -961,6 +976,8 @@ int compresskv_compress_layers_lse(const ckv_problem* p, int n_masks, const void
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   float* raw = raw_scores ? raw_scores : ws.raw;
   if ((rc = check_outputs(I, co, indices, k, v, k_out, v_out)) != CKV_OK) return rc;
+  // the scoring kernel reads lse_win for every (sequence, SRH head, window row)
+  if (I.p_total > 0 && (rc = device_memory(lse_win)) != CKV_OK) return rc;
   std::copy(co.begin(), co.end(), cu_out);
   LseInput lse;
   lse.lse = lse_win;
@@ -1064,18 +1081,54 @@ namespace {
 
 std::mutex g_scratch_mutex;
 void* g_scratch_addr[64] = {};
+unsigned long long g_scratch_ctx[64] = {};  // context the address belongs to
+PFN_cuCtxGetCurrent_v4000 g_ctx_current = nullptr;
+PFN_cuCtxGetId_v12000 g_ctx_id = nullptr;
 
+// Unique id of the calling thread's current context (0 if it cannot be
+// read).  A device reset destroys the context the array's address was looked
+// up in; the next context gets a new id.
+unsigned long long current_context_id() {
+  if (!g_ctx_current || !g_ctx_id) {
+    void* f1 = nullptr;
+    void* f2 = nullptr;
+    cudaDriverEntryPointQueryResult q1, q2;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f1, 4000, cudaEnableDefault, &q1) !=
+            cudaSuccess ||
+        q1 != cudaDriverEntryPointSuccess ||
+        cudaGetDriverEntryPointByVersion("cuCtxGetId", &f2, 12000, cudaEnableDefault, &q2) !=
+            cudaSuccess ||
+        q2 != cudaDriverEntryPointSuccess || !f1 || !f2) {
+      cudaGetLastError();
+      return 0;
+    }
+    g_ctx_current = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(f1);
+    g_ctx_id = reinterpret_cast<PFN_cuCtxGetId_v12000>(f2);
+  }
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (g_ctx_current(&ctx) != CUDA_SUCCESS || !ctx || g_ctx_id(ctx, &id) != CUDA_SUCCESS) return 0;
+  return id;
+}
+
+// Device address of the static scratch on the current device, looked up once
+// per device and context (again after a device reset, whose new context has
+// the array at a possibly different address).
 int static_scratch_address(void** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return CKV_ERR_CUDA;
   std::lock_guard<std::mutex> lock(g_scratch_mutex);
-  if (!g_scratch_addr[dev]) {
+  const unsigned long long ctx = current_context_id();
+  if (!g_scratch_addr[dev] || ctx == 0 || ctx != g_scratch_ctx[dev]) {
     void* ptr = nullptr;
     if (cudaGetSymbolAddress(&ptr, g_static_scratch) != cudaSuccess || !ptr) {
       cudaGetLastError();
+      g_scratch_addr[dev] = nullptr;
       return CKV_ERR_CUDA;
     }
     g_scratch_addr[dev] = ptr;
+    // the lookup makes the device's primary context current if none was
+    g_scratch_ctx[dev] = ctx != 0 ? ctx : current_context_id();
   }
   *out = g_scratch_addr[dev];
   return CKV_OK;

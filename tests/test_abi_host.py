@@ -232,3 +232,37 @@ def test_head_budget_host_errors_and_layout():
     assert call([[100, 31], [100, 100]]) == B.CKV_ERR_BUDGET
     lay, _, _ = _problem(selection="layer")
     assert call([[100, 100], [100, 100]], lay) == B.CKV_ERR_INVALID_ARG
+
+
+def test_binding_checks_single_mask_length():
+    prob, q, k = _problem()
+    ws = torch.zeros(16, dtype=torch.uint8)
+    for call in (lambda m: ckv.compress_layer(prob, q, k, k, m, [64, 64], k, k, k, ws),
+                 lambda m: ckv.score(prob, q, k, m, k, ws),
+                 lambda m: ckv.compress_layer_noalloc(prob, q, k, k, m, [64, 64], k, k, k),
+                 lambda m: ckv.compress_layer_head_budgets(prob, q, k, k, m,
+                                                           np.full((2, 2), 64), k, k, k, ws)):
+        with pytest.raises(ckv.CompressKVError) as e:
+            call(np.ones(7, np.uint8))  # num_q_heads is 8
+        assert e.value.code == B.CKV_ERR_INVALID_ARG
+
+
+def test_binding_checks_lse_tensor():
+    prob, q, k = _problem()
+    ws = torch.zeros(16, dtype=torch.uint8)
+    mask = np.zeros(8, np.uint8)
+    mask[[1, 6]] = 1
+    good_shape = (2, 8, 32)
+    bad = [torch.zeros(good_shape, dtype=torch.float32),            # host memory
+           torch.zeros((2, 2, 32), dtype=torch.float32),            # [B, H_kv, W]
+           torch.zeros(good_shape, dtype=torch.float64),            # dtype
+           torch.zeros((2, 8, 64), dtype=torch.float32)[:, :, ::2]]  # strided rows
+    for lse in bad:
+        with pytest.raises(ckv.CompressKVError) as e:
+            ckv.compress_layer_lse(prob, q, k, k, lse, mask, [64, 64], k, k, k, ws)
+        assert e.value.code == B.CKV_ERR_INVALID_ARG
+        with pytest.raises(ckv.CompressKVError) as e:
+            ckv.compress_layers_lse(prob, 2, q, k, k, lse, np.stack([mask, mask]), [64, 64], k,
+                                    k, k, ws)
+        assert e.value.code == B.CKV_ERR_INVALID_ARG
+

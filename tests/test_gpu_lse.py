@@ -140,3 +140,29 @@ def test_lse_path_multi_layer(cuda_device, n_layers, batch):
         compare.check_gather_bits(_bits(lay["k"]), _bits(lay["v"]), k_bits[o0:o1],
                                   v_bits[o0:o1], idx[:, o0:o1], lay["cu_seqlens"],
                                   cu_out[s0:s1 + 1] - o0)
+
+
+def test_lse_in_host_memory_refused(cuda_device):
+    # every other argument is a valid device buffer; the library checks the
+    # LSE pointer with cudaPointerGetAttributes and refuses host memory before
+    # anything is enqueued (the binding's own check is bypassed here)
+    from ctypes import POINTER, c_int32, c_void_p
+
+    from paper_2606_24467_gb300 import compresskv as B
+    cfg = wl.get("c1").scaled(seq_len=600)
+    d = wl.make_layer(cfg, 0)
+    dev = cuda_device
+    q, k, v = d["q_win"].to(dev), d["k"].to(dev), d["v"].to(dev)
+    prob = ckv.Problem(q, k, d["cu_seqlens"], cfg.window, cfg.pool_width)
+    out = ckv.LayerOutputs(prob, d["budgets"], 128, k.dtype, dev)
+    ws = ckv.workspace(prob, dev)
+    lse = torch.zeros((prob.batch, q.shape[1], cfg.window), dtype=torch.float32)  # host
+    m = np.ascontiguousarray(np.asarray(d["srh_mask"], np.uint8))
+    b, bp = B._i32(d["budgets"])
+    cu_out = np.zeros(prob.batch + 1, np.int32)
+    rc = ckv.load().compresskv_compress_layer_lse(
+        prob.ref, B._ptr(q), B._ptr(k), B._ptr(v), c_void_p(lse.data_ptr()), lse.stride(0),
+        lse.stride(1), c_void_p(m.ctypes.data), bp, B._ptr(out.indices),
+        cu_out.ctypes.data_as(POINTER(c_int32)), B._ptr(out.k_out), B._ptr(out.v_out), None,
+        None, B._ptr(ws), ws.numel(), B._stream(None))
+    assert rc == B.CKV_ERR_INVALID_ARG
