@@ -38,10 +38,10 @@ import workloads as wl  # noqa: E402
 METRIC = ("prompt tokens compressed/sec per GB300 and achieved HBM GB/s vs peak at "
           "L=32K–128K")
 UNIT = "tokens/s"
-PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "score_llama8b_L32k.md")
-# the scoring kernel's own source: a committed traffic figure is shown only
+PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "fused_llama8b_L32k.md")
+# the timed kernel's own source: a committed traffic figure is shown only
 # while it matches
-KERNEL_SOURCES = ["paper_2606_24467_gb300/csrc/score_kernel.cu"]
+KERNEL_SOURCES = ["paper_2606_24467_gb300/csrc/fused_kernel.cu"]
 
 
 def parse_args():
@@ -58,11 +58,11 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-lse", action="store_true",
                     help="skip the given-LSE (log-sum-exp supplied) measurement")
-    ap.add_argument("--streams", type=int, default=4,
+    ap.add_argument("--streams", type=int, default=1,
                     help="calls in flight: call c runs on stream c %% S with its own workspace")
     ap.add_argument("--layers-per-call", type=int, default=0,
-                    help="layers compressed by one compress_layers call (one launch per kernel); "
-                         "0 = as many (up to 4) as keep the call's exponent table in one set")
+                    help="layers compressed by one compress_layers call; 0 = every layer of the "
+                         "workload in one call (one launch of the persistent kernel per step)")
     return ap.parse_args()
 
 
@@ -208,34 +208,16 @@ def build_layers(cfg, device):
     return lengths, masks, budgets, layers
 
 
-# The library's exponent-table set (CKV_EXPO_SET_BYTES) and its row length
-# (query rows rounded up to a power of two >= 8): the automatic layers-per-
-# call choice packs layers while their tables fit one set.
-EXPO_SET_BYTES = 128 << 20
-MAX_LAYERS_PER_CALL = 4
-
-
-def expo_stride(rows: int) -> int:
-    r = 8
-    while r < rows:
-        r <<= 1
-    return r
+# Most layers one per-group compress_layers call takes (one SRH mask each).
+MAX_LAYERS_PER_CALL = 256
+# ... and one given-LSE call (the separate scoring and selection kernels)
+MAX_LSE_LAYERS_PER_CALL = 4
 
 
 def layers_per_call(cfg, layers, lengths) -> int:
-    """Most layers (<= 4) whose exponent tables, with the actual SRH rows,
-    fit one set; 2 when a single layer's does not (it is scored in two
-    passes without a table, where pairs measured best)."""
-    G = cfg.num_q_heads // cfg.num_kv_heads
-    per_layer = []
-    for lay in layers:
-        m = np.asarray(lay["srh_mask"]).reshape(cfg.num_kv_heads, G).sum(axis=1)
-        nr = sum(expo_stride(int(c) * cfg.window) for c in m)
-        per_layer.append(2 * nr * sum(max(L - cfg.window, 0) for L in lengths))
-    worst = max(per_layer)
-    if worst > EXPO_SET_BYTES:
-        return 2
-    return max(1, min(MAX_LAYERS_PER_CALL, EXPO_SET_BYTES // worst))
+    """Every layer of the step in one call: the persistent kernel then
+    streams K from the first layer to the last without a break."""
+    return max(1, min(MAX_LAYERS_PER_CALL, cfg.n_layers))
 
 
 def algorithmic_bytes(cfg, layers, lengths):
@@ -315,12 +297,9 @@ def run_ours(args):
     lanes = [torch.cuda.Stream() for _ in range(n_streams)]
     outs = [ckv.LayerOutputs(probs[c], c_budgets[c], cfg.head_dim, k_all.dtype, dev,
                              scores=False) for c in range(len(calls))]
-    # per-layer problems and outputs for the single-layer measurements (e2e,
-    # given LSE)
+    # per-layer problems for the single-layer calls of the e2e measurement
     lprobs = [ckv.Problem(lay["q_win"], lay["k"], lay["cu_seqlens"], cfg.window, cfg.pool_width)
               for lay in layers]
-    louts = [ckv.LayerOutputs(lprobs[l], budgets[l], cfg.head_dim, layers[l]["k"].dtype, dev,
-                              scores=False) for l in range(cfg.n_layers)]
 
     def run_call(pr, c, wsp, stream=None):
         l0, l1 = calls[c]
@@ -364,24 +343,37 @@ def run_ours(args):
         step(tprobs, streams=1)
     torch.cuda.synchronize()
 
+    w0 = torch.cuda.Event(enable_timing=True)
+    w1 = torch.cuda.Event(enable_timing=True)
+    w0.record()
     for _ in range(max(args.warmup, 3)):
         graph.replay()
+    w1.record()
     torch.cuda.synchronize()
+    warm_ms = w0.elapsed_time(w1) / max(args.warmup, 3)
+    # Exactly `steps` steps per timed block, bracketed by a barrier and a
+    # synchronize; the block is repeated until about two seconds of timed
+    # work have run (so the clock sampler sees the GPU under load) and the
+    # median block is reported.
+    blocks = int(min(50, max(1, math.ceil(2000.0 / max(warm_ms * args.steps, 1e-3)))))
     barrier(dist)
     sampler = ClockSampler(dev)
     sampler.start()
-    t0 = torch.cuda.Event(enable_timing=True)
-    t1 = torch.cuda.Event(enable_timing=True)
-    torch.cuda.synchronize()
-    barrier(dist)
-    t0.record()
-    for _ in range(args.steps):
-        graph.replay()
-    t1.record()
-    torch.cuda.synchronize()
+    block_ms = []
+    for _ in range(blocks):
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        barrier(dist)
+        t0.record()
+        for _ in range(args.steps):
+            graph.replay()
+        t1.record()
+        torch.cuda.synchronize()
+        barrier(dist)
+        block_ms.append(reduce_max(dist, t0.elapsed_time(t1), dev))
     clocks = sampler.stop()
-    barrier(dist)
-    elapsed_ms = reduce_max(dist, t0.elapsed_time(t1), dev)
+    elapsed_ms = statistics.median(block_ms)
     ms_per_step = elapsed_ms / args.steps
     value = world * tokens * args.steps / (elapsed_ms / 1e3)
     for w in wss:
@@ -406,12 +398,19 @@ def run_ours(args):
         per_kind.setdefault(kind, []).append(ms)
     step_bytes, score_bytes = algorithmic_bytes(cfg, layers, lengths)
     peak, peak_src = measured_peaks()
-    stats_ms = per_kind.get("score", [float("nan")])
+    if "fused" in per_kind:
+        # the persistent kernel does the whole path: its algorithmic bytes are
+        # the path's (K once, the SRH query rows, retained K/V read + written)
+        kname, stats_ms, path_bytes = ("fused (scoring, pooling, top-k and gather of every "
+                                       "unit of the call; persistent)"), per_kind["fused"], step_bytes
+    else:
+        kname, stats_ms, path_bytes = ("score (one pass over K)", per_kind.get("score", [float("nan")]),
+                                       score_bytes)
     n_stats = len(stats_ms)
     avg_stats_ms = sum(stats_ms) / max(n_stats, 1)
-    bytes_per_launch = score_bytes / max(n_stats, 1)
+    bytes_per_launch = path_bytes / max(n_stats, 1)
     achieved = bytes_per_launch / (avg_stats_ms / 1e3) / 1e9
-    roofline = {"bound": "hbm", "kernel": "score (one pass over K)", "achieved": round(achieved, 1),
+    roofline = {"bound": "hbm", "kernel": kname, "achieved": round(achieved, 1),
                 "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4),
                 "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured"
                 else "fallback 6.8 TB/s",
@@ -449,6 +448,9 @@ def run_ours(args):
         "kernels": kernels,
         "gpu_launches": int(launches_per_step * args.steps),
         "clocks": clocks,
+        "timed_blocks": {"blocks": blocks, "steps_per_block": args.steps,
+                         "ms_per_block": [round(x, 3) for x in block_ms],
+                         "reported": "median block"},
     }
 
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -458,7 +460,8 @@ def run_ours(args):
     if not args.no_e2e:
         result["e2e"] = run_e2e(args, cfg, layers, lprobs, ws, dev, dist, world)
     if not args.no_lse:
-        result["lse_fed"] = run_lse_fed(args, cfg, layers, louts, dev, dist, world, tokens)
+        result["lse_fed"] = run_lse_fed(args, cfg, layers, (q_all, k_all, v_all, T, B), dev, dist,
+                                        world, tokens)
     if rank == 0:
         print(json.dumps(result), flush=True)
     if dist is not None:
@@ -527,20 +530,37 @@ def window_lse_torch(lay, cfg, dev):
     return lse
 
 
-def run_lse_fed(args, cfg, layers, outs, dev, dist, world, tokens):
-    """The same 32-layer step through compresskv_compress_layer_lse: the
-    window queries' log-sum-exp is an input (a prefill attention kernel
-    produces it), so scoring needs no normaliser pass and no exponent table.
-    Reported beside the headline, which computes everything itself."""
+def run_lse_fed(args, cfg, layers, packed, dev, dist, world, tokens):
+    """The same step through compresskv_compress_layers_lse: the window
+    queries' log-sum-exp is an input (a prefill attention kernel produces it),
+    so scoring needs no normaliser and no exponent table.  Up to four layers
+    per call (the given-LSE calls run the separate scoring and selection
+    kernels), calls on four streams.  Reported beside the headline, which
+    computes everything itself."""
     import paper_2606_24467_gb300 as ckv
 
-    lses = [window_lse_torch(lay, cfg, dev) for lay in layers]
-    n_streams = max(1, args.streams)
+    q_all, k_all, v_all, T, B = packed
+    lse_all = torch.cat([window_lse_torch(lay, cfg, dev) for lay in layers])
+    lpc = MAX_LSE_LAYERS_PER_CALL
+    calls = [(l0, min(l0 + lpc, cfg.n_layers)) for l0 in range(0, cfg.n_layers, lpc)]
+    n_streams = 4
     trace = ckv.Trace(capacity=8 * cfg.n_layers)
-    probs = [ckv.Problem(lay["q_win"], lay["k"], lay["cu_seqlens"], cfg.window, cfg.pool_width)
-             for lay in layers]
-    tprobs = [ckv.Problem(lay["q_win"], lay["k"], lay["cu_seqlens"], cfg.window, cfg.pool_width,
-                          trace=trace) for lay in layers]
+
+    def call_problem(l0, l1, tr=None):
+        m = l1 - l0
+        cu = np.concatenate([np.asarray(layers[0]["cu_seqlens"][:-1], np.int64) + j * T
+                             for j in range(m)] + [[m * T]]).astype(np.int32)
+        return ckv.Problem(q_all[l0 * B:l1 * B], k_all[l0 * T:l1 * T], cu, cfg.window,
+                           cfg.pool_width, trace=tr)
+
+    probs = [call_problem(l0, l1) for l0, l1 in calls]
+    tprobs = [call_problem(l0, l1, trace) for l0, l1 in calls]
+    budgets = [np.concatenate([np.asarray(layers[l]["budgets"]).reshape(-1) for l in range(l0, l1)])
+               for l0, l1 in calls]
+    masks = [np.stack([np.asarray(layers[l]["srh_mask"]) for l in range(l0, l1)])
+             for l0, l1 in calls]
+    outs = [ckv.LayerOutputs(probs[c], budgets[c], cfg.head_dim, k_all.dtype, dev, scores=False)
+            for c in range(len(calls))]
     wss = [ckv.workspace(probs[0], dev) for _ in range(n_streams)]
     lanes = [torch.cuda.Stream() for _ in range(n_streams)]
 
@@ -550,12 +570,12 @@ def run_lse_fed(args, cfg, layers, outs, dev, dist, world, tokens):
         fork.record(cur)
         for st in lanes[:streams]:
             st.wait_event(fork)
-        for l, lay in enumerate(layers):
-            o = outs[l]
-            st = lanes[l % streams]
-            ckv.compress_layer_lse(pr[l], lay["q_win"], lay["k"], lay["v"], lses[l],
-                                   lay["srh_mask"], lay["budgets"], o.indices, o.k_out, o.v_out,
-                                   wss[l % streams], stream=st)
+        for c, (l0, l1) in enumerate(calls):
+            o = outs[c]
+            ckv.compress_layers_lse(pr[c], l1 - l0, q_all[l0 * B:l1 * B], k_all[l0 * T:l1 * T],
+                                    v_all[l0 * T:l1 * T], lse_all[l0 * B:l1 * B], masks[c],
+                                    budgets[c], o.indices, o.k_out, o.v_out, wss[c % streams],
+                                    stream=lanes[c % streams])
         for st in lanes[:streams]:
             done = torch.cuda.Event()
             done.record(st)
@@ -595,7 +615,8 @@ def run_lse_fed(args, cfg, layers, outs, dev, dist, world, tokens):
     peak, _ = measured_peaks()
     achieved = k_bytes / (sum(score_ms) / len(score_ms) / 1e3) / 1e9
     return {"value": round(world * tokens * args.steps / (el / 1e3), 1), "unit": UNIT,
-            "ms_per_step": round(el / args.steps, 4),
+            "ms_per_step": round(el / args.steps, 4), "layers_per_call": lpc,
+            "call_streams": n_streams,
             "kernels": {k: {"launches_per_step": len(v), "avg_us": round(1e3 * sum(v) / len(v), 2)}
                         for k, v in per_kind.items()},
             "score_roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,

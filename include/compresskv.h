@@ -105,7 +105,8 @@ enum {
   CKV_KERNEL_SCORE = 1,         /* window logits over K: softmax statistics + exponent table */
   CKV_KERNEL_COMBINE = 2,       /* normalised scores summed over queries, then pooled */
   CKV_KERNEL_SELECT = 3,        /* pooling + top-k + window append */
-  CKV_KERNEL_GATHER = 4         /* retained K/V rows -> compressed cache */
+  CKV_KERNEL_GATHER = 4,        /* retained K/V rows -> compressed cache */
+  CKV_KERNEL_FUSED = 5          /* all four steps for every unit of a call, one persistent kernel */
 };
 
 /* Optional launch trace.  When ckv_problem.trace is non-null every kernel
@@ -148,10 +149,11 @@ typedef struct ckv_problem {
  * Returns 0 if `p` is invalid. */
 size_t compresskv_workspace_size(const ckv_problem* p);
 
-/* Zero the workspace header -- the status word and the per-unit counters the
- * scoring kernel uses to merge softmax denominators (4.3 KB, enqueued on
- * `stream`).  Call once after allocating a workspace, and after reading a
- * non-zero device status (an aborted call can leave the counters set). */
+/* Zero the workspace header -- the status word and the work counters the
+ * kernels share between their CTAs (about 390 KB, enqueued on `stream`).
+ * Call once after allocating a workspace, and after reading a non-zero
+ * device status (an aborted call can leave the counters set); every call
+ * that completes leaves them zero. */
 int compresskv_workspace_init(void* workspace, size_t workspace_bytes, void* stream);
 
 /* Host-only: per-sequence offsets of the prefix scores (cu_prefix, [batch+1])
@@ -218,8 +220,20 @@ int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const voi
  * [n_layers*B][H_q][W][d], block l is layer l.  One launch of each kernel
  * then covers all the layers' units, so the scoring kernel's start-up and
  * tail are paid once.
- * n_masks: 1 <= n_masks <= 4, dividing batch (else CKV_ERR_INVALID_ARG /
- *   CKV_ERR_UNSUPPORTED).
+ * Under CKV_SELECT_PER_GROUP every step of every unit (scoring, normalising
+ * and pooling, top-k, window, gather) runs in one persistent kernel
+ * (CKV_KERNEL_FUSED): one CTA per SM streams K without a break from the first
+ * layer to the last while other warps of the same CTAs pool, select and
+ * gather the units whose scores are complete.  Its scores equal those of the
+ * separate kernels up to the fp16 rounding of the exponent table (the
+ * references restart every 8 tiles of 128 keys of a unit), and depend only
+ * on the unit itself: compressing a layer alone or among others gives the
+ * same result.  That kernel takes SRH lists of at most 192 query rows per
+ * group and at most 32 query heads per group; other per-group problems use
+ * the separate kernels.
+ * n_masks: 1 <= n_masks, dividing batch (else CKV_ERR_INVALID_ARG); at most
+ *   256 under CKV_SELECT_PER_GROUP and 4 under CKV_SELECT_PER_LAYER (or when
+ *   the separate kernels run) (else CKV_ERR_UNSUPPORTED).
  * srh_masks: host uint8 [n_masks][num_q_heads].
  * budgets, cu_out and every output follow the packed batch (sequence
  * l*B + s is sequence s of block l); the workspace is sized for `p`.

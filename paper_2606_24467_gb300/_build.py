@@ -17,8 +17,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB_PATH = os.path.join(OUT_DIR, "libcompresskv.so")
-SOURCES = ["api.cu", "score_kernel.cu", "combine_kernel.cu", "select_kernel.cu", "gather_kernel.cu",
-           "budget_alloc.cpp"]
+SOURCES = ["api.cu", "fused_kernel.cu", "score_kernel.cu", "combine_kernel.cu", "select_kernel.cu",
+           "gather_kernel.cu", "budget_alloc.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -32,7 +32,7 @@ CKV_DTYPE_BF16 = 1
 CKV_POOL_AVG = 0
 CKV_SELECT_PER_GROUP = 0
 CKV_SELECT_PER_LAYER = 1
-KERNEL_KINDS = {1: "score", 2: "combine", 3: "select", 4: "gather"}
+KERNEL_KINDS = {1: "score", 2: "combine", 3: "select", 4: "gather", 5: "fused"}
 
 EXPORTED = (
     "compresskv_workspace_size",

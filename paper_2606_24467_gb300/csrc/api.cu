@@ -24,6 +24,17 @@ namespace {
 // last-CTA-per-unit merge resets the tickets it uses).
 constexpr size_t kTicketOffset = 256;
 constexpr size_t kStatusBytes = kTicketOffset + static_cast<size_t>(kMaxItems) * sizeof(int);
+// ... followed by the fused call's counters; the whole header is zeroed by
+// compresskv_workspace_init and left zero by every call that completes.
+constexpr size_t kFusedCtrOffset = kStatusBytes;
+constexpr size_t kHeaderBytes = ((kFusedCtrOffset + kFusedCtrBytes) + 255) & ~static_cast<size_t>(255);
+// The fused call keeps a ring of per-unit exponent tables; a unit waits for
+// the unit that used its slot before to be combined.  The ring is sized to
+// at most this many bytes (enough slots to cover the units in flight).
+#ifndef CKV_FUSED_RING_BYTES
+#define CKV_FUSED_RING_BYTES (256ll << 20)
+#endif
+constexpr long long kFusedRingBytes = CKV_FUSED_RING_BYTES;
 // Units are scored in sets whose exponent tables take at most this many
 // bytes; one set's table is written by the scoring kernel and read back by
 // the combine kernel while (mostly) still in the 126 MB L2.  The workspace
@@ -73,6 +84,7 @@ int device_facts(DeviceFacts** out) {
       return CKV_ERR_CUDA;
     f.smem_optin = optin;
     if (score_set_smem_limit(static_cast<size_t>(optin)) != cudaSuccess) return CKV_ERR_CUDA;
+    if (fused_set_smem_limit(static_cast<size_t>(optin)) != cudaSuccess) return CKV_ERR_CUDA;
     if (combine_set_smem_limit(static_cast<size_t>(optin), &f.combine_smem_max) != cudaSuccess)
       return CKV_ERR_CUDA;
     if (select_set_smem_limit(static_cast<size_t>(select_max_smem_floats()) * 4) != cudaSuccess)
@@ -263,7 +275,7 @@ WorkspaceLayout workspace_layout(const Info& I) {
     r = std::max(r, S.ref_floats);
   }
   WorkspaceLayout W;
-  W.pooled = kStatusBytes + kPartialBytes + kBiasBytes;
+  W.pooled = kHeaderBytes + kPartialBytes + kBiasBytes;
   W.expo = W.pooled + align256(static_cast<size_t>(I.Hkv) * I.p_total * sizeof(float));
   W.refs = W.expo + align256(static_cast<size_t>(e) * sizeof(uint16_t));
   W.shared = W.refs + align256(static_cast<size_t>(r) * sizeof(float));
@@ -272,16 +284,60 @@ WorkspaceLayout workspace_layout(const Info& I) {
   return W;
 }
 
-size_t workspace_bytes(const Info& I) { return workspace_layout(I).total; }
+// Layout of the fused call's workspace (after the header; it aliases the
+// layout above, which the other entry points use).  A function of the problem
+// alone: rows are bounded with every head of a group counted as SRH.
+struct FusedLayout {
+  size_t pooled, partials, bias, expo, refs, total;
+  long long slot_expo, slot_refs, n_chunks;
+  int n_slots, part_stride;
+};
+
+int chunks_per_unit(const Info& I, int s) {
+  if (I.n[s] <= 0) return 0;
+  const int tiles = (I.len[s] + kTileTokens - 1) / kTileTokens;
+  return (tiles + kChunkTiles - 1) / kChunkTiles;
+}
+
+FusedLayout fused_layout(const Info& I) {
+  FusedLayout F;
+  const long long nr = expo_row_bound(I);
+  F.part_stride = (std::min(I.G * I.W, kMaxQRows) + 3) & ~3;
+  long long max_n = 0, max_tiles = 0;
+  F.n_chunks = 0;
+  for (int s = 0; s < I.B; ++s) {
+    if (I.n[s] <= 0) continue;
+    max_n = std::max<long long>(max_n, I.n[s]);
+    max_tiles = std::max<long long>(max_tiles, (I.len[s] + kTileTokens - 1) / kTileTokens);
+    F.n_chunks += static_cast<long long>(I.Hkv) * chunks_per_unit(I, s);
+  }
+  F.slot_expo = (max_n * nr + 127) & ~127LL;
+  F.slot_refs = (max_tiles * kQuarters * nr + 63) & ~63LL;
+  const long long slot_bytes = std::max<long long>(1, F.slot_expo * 2 + F.slot_refs * 4);
+  const long long units = static_cast<long long>(I.B) * I.Hkv;
+  F.n_slots = static_cast<int>(std::max(1LL, std::min(units, kFusedRingBytes / slot_bytes)));
+  F.pooled = kHeaderBytes;
+  F.partials = F.pooled + align256(static_cast<size_t>(I.Hkv) * I.p_total * sizeof(float));
+  F.bias = F.partials + align256(static_cast<size_t>(F.n_chunks) * 2 * F.part_stride * sizeof(float2));
+  F.expo = F.bias + align256(static_cast<size_t>(units) * F.part_stride * sizeof(float));
+  F.refs = F.expo + align256(static_cast<size_t>(F.n_slots) * F.slot_expo * sizeof(uint16_t));
+  F.total = F.refs + align256(static_cast<size_t>(F.n_slots) * F.slot_refs * sizeof(float));
+  return F;
+}
+
+size_t workspace_bytes(const Info& I) {
+  return std::max(workspace_layout(I).total, fused_layout(I).total);
+}
 
 int carve(const Info& I, void* ws, size_t bytes, Workspace& out) {
   const WorkspaceLayout W = workspace_layout(I);
-  if (!ws || bytes < W.total || (reinterpret_cast<uintptr_t>(ws) & 255u)) return CKV_ERR_WORKSPACE;
+  if (!ws || bytes < workspace_bytes(I) || (reinterpret_cast<uintptr_t>(ws) & 255u))
+    return CKV_ERR_WORKSPACE;
   char* b = static_cast<char*>(ws);
   out.status = reinterpret_cast<int*>(b);
   out.tickets = reinterpret_cast<int*>(b + kTicketOffset);
-  out.partials = reinterpret_cast<float2*>(b + kStatusBytes);
-  out.bias = reinterpret_cast<float*>(b + kStatusBytes + kPartialBytes);
+  out.partials = reinterpret_cast<float2*>(b + kHeaderBytes);
+  out.bias = reinterpret_cast<float*>(b + kHeaderBytes + kPartialBytes);
   out.pooled = reinterpret_cast<float*>(b + W.pooled);
   out.expo = reinterpret_cast<uint16_t*>(b + W.expo);
   out.refs = reinterpret_cast<float*>(b + W.refs);
@@ -805,6 +861,115 @@ int run_gather(const ckv_problem* p, const Info& I, const int32_t* indices,
   return traced(tr, CKV_KERNEL_GATHER, [&] { return launch_gather(P, rows, stream); });
 }
 
+// Per-group selection of a (multi-layer) fused call in one persistent kernel
+// (fused_kernel.cu).  Sets *handled = false, enqueueing nothing, when the
+// problem is outside what that kernel takes (the caller then uses the
+// scoring / combine / selection kernels).
+int run_fused(const ckv_problem* p, const Info& I, const SrhLists& S, const void* q_win,
+              const void* k, const void* v, const std::vector<int>& co, int32_t* indices,
+              void* k_out, void* v_out, float* raw, float* pooled_user, void* ws, size_t ws_bytes,
+              cudaStream_t stream, bool* handled, bool do_select = true) {
+  *handled = false;
+  if (I.layer || I.G > 32 || I.n_masks * I.Hkv > kFusedMaxLists || I.B > kFusedMaxSeqs)
+    return CKV_OK;
+  int max_rows = 16;
+  for (int v_ = 0; v_ < I.n_masks * I.Hkv; ++v_) max_rows = std::max(max_rows, S.rows[v_]);
+  const int npad_max = (max_rows + 15) & ~15;
+  const int q_half = ((npad_max * 128) + 1023) & ~1023;
+  DeviceFacts* Fd = nullptr;
+  int rc = device_facts(&Fd);
+  if (rc != CKV_OK) return rc;
+  int stages = 8;
+  while (stages >= 2 && fused_smem_bytes(q_half, stages) > static_cast<size_t>(Fd->smem_optin))
+    --stages;
+  if (stages < 2) return CKV_OK;  // query rows too many for two Q buffers and a ring
+  *handled = true;
+  if (!q_win || !k || !aligned16(q_win) || !aligned16(k)) return CKV_ERR_INVALID_ARG;
+  if (do_select && (rc = check_outputs(I, co, indices, k, v, k_out, v_out)) != CKV_OK) return rc;
+  const FusedLayout FL = fused_layout(I);
+  if (!ws || ws_bytes < workspace_bytes(I) || (reinterpret_cast<uintptr_t>(ws) & 255u))
+    return CKV_ERR_WORKSPACE;
+  char* wb = static_cast<char*>(ws);
+
+  static thread_local FusedParams P;  // large (about 15 KB): kept off the stack
+  std::memset(&P, 0, sizeof(P));
+  if ((rc = make_k_map(I, p, k, &P.tmap_k)) != CKV_OK) return rc;
+  P.q = static_cast<const uint16_t*>(q_win);
+  P.q_bs = p->q_batch_stride;
+  P.q_hs = p->q_head_stride;
+  P.q_ws = p->q_win_stride;
+  P.k = static_cast<const uint4*>(k);
+  P.v = static_cast<const uint4*>(v);
+  P.k_out = static_cast<uint4*>(k_out);
+  P.v_out = static_cast<uint4*>(v_out);
+  P.tok_stride_v16 = p->kv_token_stride / 8;
+  P.head_stride_v16 = p->kv_head_stride / 8;
+  P.indices = indices;
+  P.pooled = pooled_user ? pooled_user : reinterpret_cast<float*>(wb + FL.pooled);
+  P.raw_out = raw;
+  P.status = reinterpret_cast<int*>(wb);
+  P.ctr = reinterpret_cast<int*>(wb + kFusedCtrOffset);
+  P.partials = reinterpret_cast<float2*>(wb + FL.partials);
+  P.bias = reinterpret_cast<float*>(wb + FL.bias);
+  P.expo = reinterpret_cast<uint16_t*>(wb + FL.expo);
+  P.refs = reinterpret_cast<float*>(wb + FL.refs);
+  P.slot_expo = FL.slot_expo;
+  P.slot_refs = FL.slot_refs;
+  P.n_slots = FL.n_slots;
+  P.part_stride = FL.part_stride;
+  P.c = static_cast<float>(static_cast<double>(I.scale) * 1.4426950408889634);
+  P.window = I.W;
+  P.pool_width = I.P;
+  P.num_kv_heads = I.Hkv;
+  P.group_size = I.G;
+  P.p_total = static_cast<int>(I.p_total);
+  P.o_total = co[I.B];
+  P.is_bf16 = I.bf16 ? 1 : 0;
+  P.n_units = I.B * I.Hkv;
+  P.batch = I.B;
+  P.do_select = do_select ? 1 : 0;
+  // combine pieces: as many quarters as the workers' shared memory takes
+  // (weights of the quarters touched and raw scores with the halo), at most 64
+  const int nr_max = expo_stride(max_rows);
+  const int h = (I.P - 1) / 2;
+  const int pq = std::min(64, std::max(1, (kFusedCRegion - 3088 - 8 * nr_max - 8 * h - 64) /
+                                              (4 * nr_max + 128)));
+  P.piece_quarters = pq;
+  P.chunk_off[0] = 0;
+  P.piece_off[0] = 0;
+  for (int s_ = 0; s_ < I.B; ++s_) {
+    P.cu_seqlens[s_] = I.cu[s_];
+    P.cu_prefix[s_] = I.cu_prefix[s_];
+    P.cu_out[s_] = co[s_];
+    const int npc = I.n[s_] > 0 ? ((I.n[s_] + 31) / 32 + pq - 1) / pq : 0;
+    P.chunk_off[s_ + 1] = P.chunk_off[s_] + I.Hkv * chunks_per_unit(I, s_);
+    P.piece_off[s_ + 1] = P.piece_off[s_] + I.Hkv * npc;
+  }
+  P.cu_seqlens[I.B] = I.cu[I.B];
+  P.cu_prefix[I.B] = I.cu_prefix[I.B];
+  P.cu_out[I.B] = co[I.B];
+  P.n_chunks = P.chunk_off[I.B];
+  P.n_pieces = P.piece_off[I.B];
+  if (P.n_chunks != FL.n_chunks) return CKV_ERR_WORKSPACE;  // cannot happen: same plan
+  P.seqs_per_mask = I.spm;
+  for (int m = 0; m < I.n_masks; ++m) {
+    for (int g = 0; g < I.Hkv; ++g) {
+      const int v_ = m * I.Hkv + g;
+      uint32_t bits = 0u;
+      for (int j = S.off[v_]; j < S.off[v_ + 1]; ++j) bits |= 1u << (S.heads[j] - g * I.G);
+      P.srh_bits[v_] = bits;
+    }
+  }
+  P.q_half_bytes = q_half;
+  P.stages = stages;
+  P.tstride = npad_max <= 64 ? 64 : (npad_max <= 128 ? 128 : 256);
+  P.nbuf = 512 / P.tstride;
+  if (P.n_units == 0 || (P.n_chunks == 0 && (!do_select || co[I.B] == 0))) return CKV_OK;
+  const size_t smem = fused_smem_bytes(q_half, stages);
+  Tracer tr{p->trace, stream};
+  return traced(tr, CKV_KERNEL_FUSED, [&] { return launch_fused(P, Fd->sms, smem, stream); });
+}
+
 }  // namespace
 
 // ====================================================================== C ABI
@@ -817,8 +982,8 @@ size_t compresskv_workspace_size(const ckv_problem* p) {
 }
 
 int compresskv_workspace_init(void* workspace, size_t workspace_bytes, void* stream) {
-  if (!workspace || workspace_bytes < kStatusBytes) return CKV_ERR_WORKSPACE;
-  return cudaMemsetAsync(workspace, 0, kStatusBytes, static_cast<cudaStream_t>(stream)) ==
+  if (!workspace || workspace_bytes < kHeaderBytes) return CKV_ERR_WORKSPACE;
+  return cudaMemsetAsync(workspace, 0, kHeaderBytes, static_cast<cudaStream_t>(stream)) ==
                  cudaSuccess
              ? CKV_OK
              : CKV_ERR_CUDA;
@@ -847,8 +1012,19 @@ int compresskv_score(const ckv_problem* p, const void* q_win, const void* k,
   Workspace ws;
   if ((rc = carve(I, workspace, workspace_bytes, ws)) != CKV_OK) return rc;
   if (!raw_scores) return CKV_ERR_INVALID_ARG;
-  return run_score(p, I, q_win, k, srh_mask, raw_scores, ws.pooled, ws,
-                   static_cast<cudaStream_t>(stream));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (!I.layer) {
+    // per-group problems are scored by the kernel the fused layer call runs
+    // (the same scores, bit for bit), without its selection
+    SrhLists S;
+    if ((rc = srh_lists(I, srh_mask, S)) != CKV_OK) return rc;
+    bool handled = false;
+    std::vector<int> co(I.B + 1, 0);
+    rc = run_fused(p, I, S, q_win, k, nullptr, co, nullptr, nullptr, nullptr, raw_scores,
+                   nullptr, workspace, workspace_bytes, st, &handled, false);
+    if (handled) return rc;
+  }
+  return run_score(p, I, q_win, k, srh_mask, raw_scores, ws.pooled, ws, st);
 }
 
 int compresskv_select(const ckv_problem* p, const float* raw_scores, const int32_t* budgets,
@@ -910,7 +1086,7 @@ int compresskv_compress_layers(const ckv_problem* p, int n_masks, const void* q_
   int rc = validate(p, I);
   if (rc != CKV_OK) return rc;
   if (n_masks < 1 || I.B % n_masks != 0) return CKV_ERR_INVALID_ARG;
-  if (n_masks > kMaxMasks) return CKV_ERR_UNSUPPORTED;
+  if (n_masks > kMaxFusedMasks) return CKV_ERR_UNSUPPORTED;
   I.n_masks = n_masks;
   I.spm = I.B / n_masks;
   const uint8_t* srh_mask = srh_masks;
@@ -922,6 +1098,17 @@ int compresskv_compress_layers(const ckv_problem* p, int n_masks, const void* q_
   SrhLists S;
   if ((rc = srh_lists(I, srh_mask, S)) != CKV_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (!I.layer) {
+    // per-group selection: one persistent kernel for every unit of the call
+    bool handled = false;
+    rc = run_fused(p, I, S, q_win, k, v, co, indices, k_out, v_out, raw_scores, pooled_scores,
+                   workspace, workspace_bytes, st, &handled);
+    if (handled) {
+      if (rc == CKV_OK) std::copy(co.begin(), co.end(), cu_out);
+      return rc;
+    }
+  }
+  if (n_masks > kMaxMasks) return CKV_ERR_UNSUPPORTED;
   float* pooled = pooled_scores ? pooled_scores : ws.pooled;
   if ((rc = check_outputs(I, co, indices, k, v, k_out, v_out)) != CKV_OK) return rc;
   std::copy(co.begin(), co.end(), cu_out);
@@ -1149,8 +1336,9 @@ extern "C" int compresskv_compress_layer_noalloc(
   void* scratch = nullptr;
   if ((rc = static_scratch_address(&scratch)) != CKV_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  // The array keeps the previous call's contents; the status word must start at zero.
-  if (cudaMemsetAsync(scratch, 0, kStatusBytes, st) != cudaSuccess) return CKV_ERR_CUDA;
+  // The array keeps the previous call's contents; the status word and the
+  // counters must start at zero.
+  if (cudaMemsetAsync(scratch, 0, kHeaderBytes, st) != cudaSuccess) return CKV_ERR_CUDA;
   rc = compresskv_compress_layer(p, q_win, k, v, srh_mask, budgets, indices, cu_out, k_out, v_out,
                                  raw_scores, pooled_scores, scratch,
                                  static_cast<size_t>(CKV_STATIC_SCRATCH_BYTES), stream);

@@ -129,7 +129,7 @@ __device__ __forceinline__ void warp_pick_bin256(const uint32_t* h, int rem, int
 // then picks the bin itself.  `slot` selects this search's key_or / key_and
 // (zero / all ones on entry).  Kept out of line: the kernels that call it run
 // once per SM, so code size (instruction fetch) matters more than inlining.
-__device__ __noinline__ uint32_t cta_kth_largest(const uint32_t* keys, int count, uint32_t sub,
+static __device__ __noinline__ uint32_t cta_kth_largest(const uint32_t* keys, int count, uint32_t sub,
                                                  uint32_t clamp, int r, RadixShared& sh, int slot,
                                                  int& pc, int* rem) {
   const int tid = threadIdx.x;

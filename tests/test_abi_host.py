@@ -140,11 +140,18 @@ def test_compress_layers_host_errors():
     assert call(2, [mask_empty, mask_ok]) == B.CKV_ERR_EMPTY_SRH_GROUP  # first block
     # one mask for both sequences is the single-layer call: the empty group fails too
     assert call(1, [mask_empty]) == B.CKV_ERR_EMPTY_SRH_GROUP
-    p5, _, _ = _problem(L=(100,) * 5)
+    # per-layer selection runs the separate kernels: at most 4 masks per call
+    p5, _, _ = _problem(L=(100,) * 5, selection="layer")
     b5, bp5 = B._i32([64] * 5)
     cu_out = (ctypes.c_int32 * 6)()
     assert call(5, [mask_ok] * 5, p=p5, budgets_ptr=bp5,
-                wsn=ckv.workspace_size(p5)) == B.CKV_ERR_UNSUPPORTED  # more than 4 masks
+                wsn=ckv.workspace_size(p5)) == B.CKV_ERR_UNSUPPORTED
+    # per-group selection runs the persistent kernel: at most 256 masks
+    p257, _, _ = _problem(L=(40,) * 257)
+    b257, bp257 = B._i32([32] * 257)
+    cu_out = (ctypes.c_int32 * 258)()
+    assert call(257, [mask_ok] * 257, p=p257, budgets_ptr=bp257,
+                wsn=ckv.workspace_size(p257)) == B.CKV_ERR_UNSUPPORTED
 
 
 def test_compress_layers_lse_host_errors():

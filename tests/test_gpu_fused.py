@@ -1,0 +1,157 @@
+"""The persistent per-group kernel of compresskv_compress_layers against the
+float64 oracle, through the C ABI (needs a GB300).
+
+Besides parity with the oracle (tolerances as in test_gpu_parity.py), the
+kernel's scores depend only on the unit itself: its exponent references
+restart on a fixed grid of 8 K tiles of every unit and each tile of that grid
+always goes to the same epilogue warpgroup, so a layer compressed alone and
+the same layer inside a larger call give identical bits.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2606_24467_gb300 as ckv
+import workloads as wl
+from oracle import compare
+
+pytestmark = pytest.mark.gpu
+
+EXPO_RTOL = 2.0 ** -11 + 2e-5
+
+
+def _bits(t):
+    return t.detach().cpu().contiguous().view(torch.int16).numpy()
+
+
+def _layers(cfg):
+    lengths = wl.sequence_lengths(cfg)
+    masks = wl.srh_masks(cfg)
+    budgets = wl.layer_budgets(cfg, lengths)
+    return [wl.make_layer(cfg, l, lengths=lengths, masks=masks, budgets=budgets)
+            for l in range(cfg.n_layers)]
+
+
+def _pack(layers, dev, lengths_per_layer=None):
+    """K/V/Q of several layers packed as one batch (block l = layer l)."""
+    Ts = [lay["k"].shape[0] for lay in layers]
+    k_all = torch.cat([lay["k"] for lay in layers]).to(dev)
+    v_all = torch.cat([lay["v"] for lay in layers]).to(dev)
+    q_all = torch.cat([lay["q_win"] for lay in layers]).to(dev)
+    offs = np.concatenate([[0], np.cumsum(Ts)])
+    cu = np.concatenate([np.asarray(lay["cu_seqlens"][:-1], np.int64) + offs[l]
+                         for l, lay in enumerate(layers)] + [[offs[-1]]]).astype(np.int32)
+    b_all = np.concatenate([np.asarray(lay["budgets"]).reshape(-1) for lay in layers])
+    m_all = np.stack([np.asarray(lay["srh_mask"]) for lay in layers])
+    return q_all, k_all, v_all, cu, b_all, m_all
+
+
+def _run_call(layers, cfg, dev, scores=True):
+    q_all, k_all, v_all, cu, b_all, m_all = _pack(layers, dev)
+    prob = ckv.Problem(q_all, k_all, cu, cfg.window, cfg.pool_width)
+    out = ckv.LayerOutputs(prob, b_all, 128, k_all.dtype, dev, scores=scores)
+    ws = ckv.workspace(prob, dev)
+    cu_out = ckv.compress_layers(prob, len(layers), q_all, k_all, v_all, m_all, b_all,
+                                 out.indices, out.k_out, out.v_out, ws, raw=out.raw,
+                                 pooled=out.pooled)
+    torch.cuda.synchronize()
+    assert ckv.read_device_status(ws) == 0
+    return out, cu_out, cu
+
+
+def _block(out, cu_out, cu, l, B, window):
+    """Layer l's block of a packed call's outputs (host arrays)."""
+    n = np.maximum(np.diff(cu) - window, 0)
+    cu_prefix = np.concatenate([[0], np.cumsum(n)])
+    s0, s1 = l * B, (l + 1) * B
+    p0, p1 = cu_prefix[s0], cu_prefix[s1]
+    o0, o1 = cu_out[s0], cu_out[s1]
+    blk = {"indices": out.indices[:, o0:o1].cpu().numpy(),
+           "k_out": _bits(out.k_out[o0:o1]), "v_out": _bits(out.v_out[o0:o1]),
+           "cu_out": cu_out[s0:s1 + 1] - o0}
+    if out.raw is not None:
+        blk["raw"] = out.raw[:, p0:p1].cpu().numpy()
+        blk["pooled"] = out.pooled[:, p0:p1].cpu().numpy()
+    return blk
+
+
+def _check_block(blk, lay, cfg):
+    res = oracle.compress_layer(lay["q_win"].float().numpy(), lay["k"].float().numpy(),
+                                lay["v"].float().numpy(), lay["cu_seqlens"], lay["srh_mask"],
+                                lay["budgets"], cfg.window, cfg.pool_width)
+    assert np.array_equal(blk["cu_out"], res.cu_out)
+    if "raw" in blk:
+        compare.check_layer(res, blk["raw"], blk["pooled"], blk["indices"], lay["cu_seqlens"],
+                            cfg.window)
+        compare.check_scores("raw (fp16 table bound)", blk["raw"], res.raw, rtol=EXPO_RTOL,
+                             atol=1e-8)
+        compare.check_scores("pooled (fp16 table bound)", blk["pooled"], res.pooled,
+                             rtol=EXPO_RTOL, atol=1e-8)
+    else:
+        for (s, g), unit in res.units.items():
+            L = int(lay["cu_seqlens"][s + 1] - lay["cu_seqlens"][s])
+            o0, o1 = int(res.cu_out[s]), int(res.cu_out[s + 1])
+            compare.check_unit_indices(blk["indices"][g, o0:o1], unit, L, cfg.window)
+    compare.check_gather_bits(_bits(lay["k"]), _bits(lay["v"]), blk["k_out"], blk["v_out"],
+                              blk["indices"], lay["cu_seqlens"], blk["cu_out"])
+
+
+def test_layer_alone_equals_layer_in_a_larger_call(cuda_device):
+    """Scores, indices and K/V of a layer are bit-identical whether it is
+    compressed alone or as one block of a six-layer call (ragged batch)."""
+    dev = cuda_device
+    cfg = wl.get("c2").scaled(seq_len=0, n_layers=6, batch=3, length_range=(900, 5200))
+    layers = _layers(cfg)
+    big, cu_out, cu = _run_call(layers, cfg, dev)
+    for l in (0, 3, 5):
+        alone, cu_out1, cu1 = _run_call([layers[l]], cfg, dev)
+        a = _block(alone, cu_out1, cu1, 0, cfg.batch, cfg.window)
+        b = _block(big, cu_out, cu, l, cfg.batch, cfg.window)
+        for key in ("raw", "pooled", "indices", "k_out", "v_out", "cu_out"):
+            assert np.array_equal(a[key].view(np.uint8) if a[key].dtype != np.int32 else a[key],
+                                  b[key].view(np.uint8) if b[key].dtype != np.int32 else b[key]), (l, key)
+        _check_block(b, layers[l], cfg)
+
+
+def test_many_short_layers_with_edge_lengths(cuda_device):
+    """Forty layers of a batch of 5 prompts with lengths 0, 1, W, W+1 and
+    tile edges in one call: more units than chunks, empty and window-only
+    sequences, per-layer masks and budgets."""
+    dev = cuda_device
+    lens = [0, 33, 32, 129, 1023]
+    cfg = wl.get("c2").scaled(seq_len=0, n_layers=40, batch=len(lens), srh_per_group=(1, 3))
+    lengths = lens
+    masks = wl.srh_masks(cfg)
+    budgets = wl.layer_budgets(cfg, lengths)
+    layers = [wl.make_layer(cfg, l, lengths=lengths, masks=masks, budgets=budgets)
+              for l in range(cfg.n_layers)]
+    out, cu_out, cu = _run_call(layers, cfg, dev)
+    for l in (0, 17, 39):
+        _check_block(_block(out, cu_out, cu, l, cfg.batch, cfg.window), layers[l], cfg)
+
+
+def test_repeat_call_is_bit_identical(cuda_device):
+    dev = cuda_device
+    cfg = wl.get("c2").scaled(seq_len=9000, n_layers=3)
+    layers = _layers(cfg)
+    a, ca, _ = _run_call(layers, cfg, dev)
+    b, cb, _ = _run_call(layers, cfg, dev)
+    assert np.array_equal(ca, cb)
+    assert torch.equal(a.raw.view(torch.int32), b.raw.view(torch.int32))
+    assert torch.equal(a.pooled.view(torch.int32), b.pooled.view(torch.int32))
+    assert torch.equal(a.indices, b.indices)
+    assert torch.equal(a.k_out.view(torch.int16), b.k_out.view(torch.int16))
+
+
+def test_full_32_layer_llama8b_32k_in_one_call(cuda_device):
+    """The benchmark step itself: all 32 layers of the L=32K Llama-3.1-8B
+    workload in one call (256 units; more units than exponent-table slots, so
+    units wait for their slot's previous user).  The first and last layers
+    are checked against the oracle unit by unit."""
+    dev = cuda_device
+    cfg = wl.get("c2")
+    layers = _layers(cfg)
+    out, cu_out, cu = _run_call(layers, cfg, dev, scores=False)
+    for l in (0, cfg.n_layers - 1):
+        _check_block(_block(out, cu_out, cu, l, cfg.batch, cfg.window), layers[l], cfg)
