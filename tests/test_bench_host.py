@@ -1,6 +1,6 @@
 """Host logic of the benchmark: how many layers one compress_layers call
-packs (the most, up to four, whose exponent tables with the actual SRH rows
-fit one 128 MiB set; two when a single layer's table does not)."""
+packs (every layer of the step, up to the 256 SRH masks one per-group call
+takes), and the step's algorithmic bytes."""
 import numpy as np
 
 import bench
@@ -15,22 +15,32 @@ def _lpc(name):
     return bench.layers_per_call(cfg, layers, lengths)
 
 
-def test_expo_stride_matches_the_library_rule():
-    assert [bench.expo_stride(r) for r in (0, 1, 8, 9, 32, 33, 64, 96, 192, 256)] == \
-        [8, 8, 8, 16, 32, 64, 64, 128, 256, 256]
-
-
 def test_layers_per_call_of_the_workloads():
-    assert _lpc("c2") == 4   # ~25 MB of table per layer
-    assert _lpc("c3") == 1   # ~100 MB per layer: one layer per set
-    assert _lpc("c4") == 2   # a layer's table exceeds the set: two passes
-    assert _lpc("c5") == 2
+    assert _lpc("c1") == 1
+    assert _lpc("c2") == 32
+    assert _lpc("c3") == 32
+    assert _lpc("c4") == 28
+    assert _lpc("c5") == 80
 
 
 def test_layers_per_call_bounds():
-    cfg = wl.get("c2").scaled(seq_len=1000, n_layers=8)
+    cfg = wl.get("c2").scaled(seq_len=1000, n_layers=300)
     lengths = wl.sequence_lengths(cfg)
-    one_head = np.zeros(cfg.num_q_heads, bool)
-    one_head[::cfg.num_q_heads // cfg.num_kv_heads] = True
-    layers = [{"srh_mask": one_head} for _ in range(cfg.n_layers)]
-    assert bench.layers_per_call(cfg, layers, lengths) == bench.MAX_LAYERS_PER_CALL
+    layers = [{"srh_mask": np.ones(cfg.num_q_heads, bool)} for _ in range(cfg.n_layers)]
+    assert bench.layers_per_call(cfg, layers, lengths) == bench.MAX_LAYERS_PER_CALL == 256
+
+
+def test_algorithmic_bytes_of_the_bench_step():
+    # K once for scoring, the SRH query rows, and 4 x 256 B per kept token and
+    # group (K and V rows read and written)
+    cfg = wl.get("c2").scaled(n_layers=2, seq_len=1000)
+    lengths = wl.sequence_lengths(cfg)
+    mask = np.zeros(cfg.num_q_heads, bool)
+    mask[[0, 5, 9, 13, 17, 21, 25, 29]] = True
+    layers = [{"srh_mask": mask, "budgets": np.array([200])},
+              {"srh_mask": mask, "budgets": np.array([2000])}]
+    total, score = bench.algorithmic_bytes(cfg, layers, lengths)
+    k_bytes = 1000 * 8 * 128 * 2
+    q_bytes = 8 * 32 * 128 * 2
+    assert score == 2 * (k_bytes + q_bytes)
+    assert total == score + 4 * (200 + 1000) * 8 * 128 * 2
