@@ -28,13 +28,7 @@ constexpr size_t kStatusBytes = kTicketOffset + static_cast<size_t>(kMaxItems) *
 // compresskv_workspace_init and left zero by every call that completes.
 constexpr size_t kFusedCtrOffset = kStatusBytes;
 constexpr size_t kHeaderBytes = ((kFusedCtrOffset + kFusedCtrBytes) + 255) & ~static_cast<size_t>(255);
-// The fused call keeps a ring of per-unit exponent tables; a unit waits for
-// the unit that used its slot before to be combined.  The ring is sized to
-// at most this many bytes (enough slots to cover the units in flight).
-#ifndef CKV_FUSED_RING_BYTES
-#define CKV_FUSED_RING_BYTES (256ll << 20)
-#endif
-constexpr long long kFusedRingBytes = CKV_FUSED_RING_BYTES;
+
 // Units are scored in sets whose exponent tables take at most this many
 // bytes; one set's table is written by the scoring kernel and read back by
 // the combine kernel while (mostly) still in the 126 MB L2.  The workspace
@@ -288,9 +282,9 @@ WorkspaceLayout workspace_layout(const Info& I) {
 // layout above, which the other entry points use).  A function of the problem
 // alone: rows are bounded with every head of a group counted as SRH.
 struct FusedLayout {
-  size_t pooled, partials, bias, expo, refs, total;
-  long long slot_expo, slot_refs, n_chunks;
-  int n_slots, part_stride;
+  size_t raw, pooled, partials, bias, total;
+  long long n_chunks;
+  int part_stride;
 };
 
 int chunks_per_unit(const Info& I, int s) {
@@ -301,27 +295,17 @@ int chunks_per_unit(const Info& I, int s) {
 
 FusedLayout fused_layout(const Info& I) {
   FusedLayout F;
-  const long long nr = expo_row_bound(I);
   F.part_stride = (std::min(I.G * I.W, kMaxQRows) + 3) & ~3;
-  long long max_n = 0, max_tiles = 0;
   F.n_chunks = 0;
-  for (int s = 0; s < I.B; ++s) {
-    if (I.n[s] <= 0) continue;
-    max_n = std::max<long long>(max_n, I.n[s]);
-    max_tiles = std::max<long long>(max_tiles, (I.len[s] + kTileTokens - 1) / kTileTokens);
-    F.n_chunks += static_cast<long long>(I.Hkv) * chunks_per_unit(I, s);
-  }
-  F.slot_expo = (max_n * nr + 127) & ~127LL;
-  F.slot_refs = (max_tiles * kQuarters * nr + 63) & ~63LL;
-  const long long slot_bytes = std::max<long long>(1, F.slot_expo * 2 + F.slot_refs * 4);
+  for (int s = 0; s < I.B; ++s) F.n_chunks += static_cast<long long>(I.Hkv) * chunks_per_unit(I, s);
   const long long units = static_cast<long long>(I.B) * I.Hkv;
-  F.n_slots = static_cast<int>(std::max(1LL, std::min(units, kFusedRingBytes / slot_bytes)));
-  F.pooled = kHeaderBytes;
-  F.partials = F.pooled + align256(static_cast<size_t>(I.Hkv) * I.p_total * sizeof(float));
-  F.bias = F.partials + align256(static_cast<size_t>(F.n_chunks) * 2 * F.part_stride * sizeof(float2));
-  F.expo = F.bias + align256(static_cast<size_t>(units) * F.part_stride * sizeof(float));
-  F.refs = F.expo + align256(static_cast<size_t>(F.n_slots) * F.slot_expo * sizeof(uint16_t));
-  F.total = F.refs + align256(static_cast<size_t>(F.n_slots) * F.slot_refs * sizeof(float));
+  const size_t scores = align256(static_cast<size_t>(I.Hkv) * I.p_total * sizeof(float));
+  F.raw = kHeaderBytes;
+  F.pooled = F.raw + scores;
+  F.partials = F.pooled + scores;
+  F.bias = F.partials + align256(static_cast<size_t>(F.n_chunks) * kFusedPartsPerChunk *
+                                 F.part_stride * sizeof(float2));
+  F.total = F.bias + align256(static_cast<size_t>(units) * F.part_stride * sizeof(float));
   return F;
 }
 
@@ -864,11 +848,13 @@ int run_gather(const ckv_problem* p, const Info& I, const int32_t* indices,
 // Per-group selection of a (multi-layer) fused call in one persistent kernel
 // (fused_kernel.cu).  Sets *handled = false, enqueueing nothing, when the
 // problem is outside what that kernel takes (the caller then uses the
-// scoring / combine / selection kernels).
+// scoring / combine / selection kernels).  `lse` given: the window queries'
+// log-sum-exp replaces the first pass.
 int run_fused(const ckv_problem* p, const Info& I, const SrhLists& S, const void* q_win,
               const void* k, const void* v, const std::vector<int>& co, int32_t* indices,
-              void* k_out, void* v_out, float* raw, float* pooled_user, void* ws, size_t ws_bytes,
-              cudaStream_t stream, bool* handled, bool do_select = true) {
+              void* k_out, void* v_out, float* raw_user, float* pooled_user, void* ws,
+              size_t ws_bytes, cudaStream_t stream, bool* handled, bool do_select = true,
+              const LseInput& lse = LseInput{}) {
   *handled = false;
   if (I.layer || I.G > 32 || I.n_masks * I.Hkv > kFusedMaxLists || I.B > kFusedMaxSeqs)
     return CKV_OK;
@@ -876,13 +862,28 @@ int run_fused(const ckv_problem* p, const Info& I, const SrhLists& S, const void
   for (int v_ = 0; v_ < I.n_masks * I.Hkv; ++v_) max_rows = std::max(max_rows, S.rows[v_]);
   const int npad_max = (max_rows + 15) & ~15;
   const int q_half = ((npad_max * 128) + 1023) & ~1023;
+  const int row_stride = (max_rows + 31) & ~31;
+  // TMEM: 512 columns of accumulator buffers, tstride columns each
+  const int tstride = npad_max <= 64 ? 64 : (npad_max <= 128 ? 128 : 256);
+  const int nwg = 2;  // epilogue warpgroups that take tiles
+  const int nbuf = 512 / tstride;
   DeviceFacts* Fd = nullptr;
   int rc = device_facts(&Fd);
   if (rc != CKV_OK) return rc;
-  int stages = 8;
-  while (stages >= 2 && fused_smem_bytes(q_half, stages) > static_cast<size_t>(Fd->smem_optin))
-    --stages;
-  if (stages < 2) return CKV_OK;  // query rows too many for two Q buffers and a ring
+  // three Q buffers when they fit beside a ring of at least four K tiles,
+  // else two beside at least two
+  int stages = 0, q_bufs = 0;
+  for (int nq = 3; nq >= 2 && stages == 0; --nq) {
+    for (int st = 8; st >= (nq == 3 ? 4 : 2); --st) {
+      if (fused_smem_bytes(q_half, nq, st, row_stride, nwg) <=
+          static_cast<size_t>(Fd->smem_optin)) {
+        stages = st;
+        q_bufs = nq;
+        break;
+      }
+    }
+  }
+  if (stages == 0) return CKV_OK;  // query rows too many for two Q buffers and a ring
   *handled = true;
   if (!q_win || !k || !aligned16(q_win) || !aligned16(k)) return CKV_ERR_INVALID_ARG;
   if (do_select && (rc = check_outputs(I, co, indices, k, v, k_out, v_out)) != CKV_OK) return rc;
@@ -898,6 +899,10 @@ int run_fused(const ckv_problem* p, const Info& I, const SrhLists& S, const void
   P.q_bs = p->q_batch_stride;
   P.q_hs = p->q_head_stride;
   P.q_ws = p->q_win_stride;
+  P.lse = lse.lse;
+  P.lse_bs = lse.batch_stride;
+  P.lse_hs = lse.head_stride;
+  P.given_lse = lse.lse ? 1 : 0;
   P.k = static_cast<const uint4*>(k);
   P.v = static_cast<const uint4*>(v);
   P.k_out = static_cast<uint4*>(k_out);
@@ -905,17 +910,12 @@ int run_fused(const ckv_problem* p, const Info& I, const SrhLists& S, const void
   P.tok_stride_v16 = p->kv_token_stride / 8;
   P.head_stride_v16 = p->kv_head_stride / 8;
   P.indices = indices;
+  P.raw = raw_user ? raw_user : reinterpret_cast<float*>(wb + FL.raw);
   P.pooled = pooled_user ? pooled_user : reinterpret_cast<float*>(wb + FL.pooled);
-  P.raw_out = raw;
   P.status = reinterpret_cast<int*>(wb);
   P.ctr = reinterpret_cast<int*>(wb + kFusedCtrOffset);
   P.partials = reinterpret_cast<float2*>(wb + FL.partials);
   P.bias = reinterpret_cast<float*>(wb + FL.bias);
-  P.expo = reinterpret_cast<uint16_t*>(wb + FL.expo);
-  P.refs = reinterpret_cast<float*>(wb + FL.refs);
-  P.slot_expo = FL.slot_expo;
-  P.slot_refs = FL.slot_refs;
-  P.n_slots = FL.n_slots;
   P.part_stride = FL.part_stride;
   P.c = static_cast<float>(static_cast<double>(I.scale) * 1.4426950408889634);
   P.window = I.W;
@@ -928,28 +928,17 @@ int run_fused(const ckv_problem* p, const Info& I, const SrhLists& S, const void
   P.n_units = I.B * I.Hkv;
   P.batch = I.B;
   P.do_select = do_select ? 1 : 0;
-  // combine pieces: as many quarters as the workers' shared memory takes
-  // (weights of the quarters touched and raw scores with the halo), at most 64
-  const int nr_max = expo_stride(max_rows);
-  const int h = (I.P - 1) / 2;
-  const int pq = std::min(64, std::max(1, (kFusedCRegion - 3088 - 8 * nr_max - 8 * h - 64) /
-                                              (4 * nr_max + 128)));
-  P.piece_quarters = pq;
   P.chunk_off[0] = 0;
-  P.piece_off[0] = 0;
   for (int s_ = 0; s_ < I.B; ++s_) {
     P.cu_seqlens[s_] = I.cu[s_];
     P.cu_prefix[s_] = I.cu_prefix[s_];
     P.cu_out[s_] = co[s_];
-    const int npc = I.n[s_] > 0 ? ((I.n[s_] + 31) / 32 + pq - 1) / pq : 0;
     P.chunk_off[s_ + 1] = P.chunk_off[s_] + I.Hkv * chunks_per_unit(I, s_);
-    P.piece_off[s_ + 1] = P.piece_off[s_] + I.Hkv * npc;
   }
   P.cu_seqlens[I.B] = I.cu[I.B];
   P.cu_prefix[I.B] = I.cu_prefix[I.B];
   P.cu_out[I.B] = co[I.B];
   P.n_chunks = P.chunk_off[I.B];
-  P.n_pieces = P.piece_off[I.B];
   if (P.n_chunks != FL.n_chunks) return CKV_ERR_WORKSPACE;  // cannot happen: same plan
   P.seqs_per_mask = I.spm;
   for (int m = 0; m < I.n_masks; ++m) {
@@ -961,11 +950,14 @@ int run_fused(const ckv_problem* p, const Info& I, const SrhLists& S, const void
     }
   }
   P.q_half_bytes = q_half;
+  P.q_bufs = q_bufs;
+  P.row_stride = row_stride;
   P.stages = stages;
-  P.tstride = npad_max <= 64 ? 64 : (npad_max <= 128 ? 128 : 256);
-  P.nbuf = 512 / P.tstride;
+  P.tstride = tstride;
+  P.nbuf = nbuf;
+  P.nwg = nwg;
   if (P.n_units == 0 || (P.n_chunks == 0 && (!do_select || co[I.B] == 0))) return CKV_OK;
-  const size_t smem = fused_smem_bytes(q_half, stages);
+  const size_t smem = fused_smem_bytes(q_half, q_bufs, stages, row_stride, nwg);
   Tracer tr{p->trace, stream};
   return traced(tr, CKV_KERNEL_FUSED, [&] { return launch_fused(P, Fd->sms, smem, stream); });
 }
@@ -1146,7 +1138,7 @@ int compresskv_compress_layers_lse(const ckv_problem* p, int n_masks, const void
   int rc = validate(p, I);
   if (rc != CKV_OK) return rc;
   if (n_masks < 1 || I.B % n_masks != 0) return CKV_ERR_INVALID_ARG;
-  if (n_masks > kMaxMasks) return CKV_ERR_UNSUPPORTED;
+  if (n_masks > kMaxFusedMasks) return CKV_ERR_UNSUPPORTED;
   I.n_masks = n_masks;
   I.spm = I.B / n_masks;
   const uint8_t* srh_mask = srh_masks;
@@ -1170,6 +1162,15 @@ int compresskv_compress_layers_lse(const ckv_problem* p, int n_masks, const void
   lse.lse = lse_win;
   lse.batch_stride = lse_batch_stride;
   lse.head_stride = lse_head_stride;
+  if (!I.layer) {
+    // per-group selection: the persistent kernel with the given LSE in place
+    // of its first pass
+    bool handled = false;
+    rc = run_fused(p, I, S, q_win, k, v, co, indices, k_out, v_out, raw_scores, pooled_scores,
+                   workspace, workspace_bytes, st, &handled, true, lse);
+    if (handled) return rc;
+  }
+  if (n_masks > kMaxMasks) return CKV_ERR_UNSUPPORTED;
   if ((rc = run_score(p, I, q_win, k, srh_mask, raw, nullptr, ws, st, lse)) != CKV_OK) return rc;
   return run_select(p, I, raw, nullptr, co, indices, pooled_scores, ws, st, k, v, k_out, v_out);
 }

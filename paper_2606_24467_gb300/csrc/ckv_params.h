@@ -142,61 +142,66 @@ struct GatherParams {
 };
 
 // ---------------------------------------------------------------------------
-// Persistent fused layer call (per-group selection of compresskv_compress_layers):
-// one kernel scores every unit of the call, combines and pools the scores and
-// selects and gathers, with work claimed from counters in the workspace.
+// Persistent fused layer call (per-group selection of compresskv_compress_layers
+// and compresskv_compress_layers_lse): one kernel streams K for every unit of
+// a call in two passes (softmax statistics, then normalised scores with K
+// re-read from L2), pools, selects and gathers, with work claimed from
+// counters in the workspace.
 constexpr int kChunkTiles = 8;          // K tiles per scoring chunk (references restart per chunk)
+constexpr int kChunkKeys = kChunkTiles * kTileTokens;
 constexpr int kFusedMaxSeqs = kMaxBatch;
 constexpr int kFusedMaxLists = 1024;    // (mask, group) SRH lists of one call
 constexpr int kFusedMaxUnits = kMaxBatch * kMaxKvHeads;
 constexpr int kFusedCtrHead = 64;       // claim / exit / abort counters before the per-unit ones
 // Workspace counters of the fused call: the header words, then per unit the
-// scoring contributions (two per chunk), the combine pieces done and the
-// state of its merged softmax denominators.
+// first-pass contributions (one per epilogue warpgroup and chunk), the
+// second-pass contributions (one per epilogue warp and chunk) and the state
+// of its merged softmax denominators.
 constexpr size_t kFusedCtrBytes = static_cast<size_t>(kFusedCtrHead + 3 * kFusedMaxUnits) * 4;
 constexpr int kFusedCandCap = 4096;     // top-k candidates of one unit kept in shared memory
-constexpr int kFusedCRegion = 40 * 1024;  // shared memory of the combine / select warps
+constexpr int kFusedCRegion = 40 * 1024;  // shared memory of the merge / select warps
 
 struct FusedParams {
   CUtensorMap tmap_k;          // 3-D map over K: (d, kv head, token)
   const uint16_t* q;           // window queries (f16/bf16 bits)
   long long q_bs, q_hs, q_ws;  // window-query strides, elements
+  const float* lse;            // given-LSE mode: natural-log LSE per (sequence, head, window row)
+  long long lse_bs, lse_hs;    // its strides (elements); window rows contiguous
   const uint4* k;              // gather sources (K on the device; V may be mapped host memory)
   const uint4* v;
   uint4* k_out;
   uint4* v_out;
   long long tok_stride_v16, head_stride_v16;  // K/V strides in 16-byte units
   int32_t* indices;            // [num_kv_heads][o_total]
-  float* pooled;               // score layout: pooled scores (caller's buffer or workspace)
-  float* raw_out;              // optional raw scores, score layout
+  float* raw;                  // raw scores, score layout (caller's buffer or workspace)
+  float* pooled;               // pooled scores, score layout (caller's buffer or workspace)
   int* status;                 // device status word
   int* ctr;                    // counters (kFusedCtrBytes, zero between calls)
-  float2* partials;            // [chunk * 2 + warpgroup][part_stride]: (M, S), sum 2^(z c) = S 2^M
+  float2* partials;            // [chunk * 4 + warpgroup][part_stride]: (M, S), sum 2^(z c) = S 2^M
   float* bias;                 // [unit][part_stride]: log2 D_q
-  uint16_t* expo;              // ring of n_slots exponent tables (fp16, [key][Nr] per unit)
-  float* refs;                 // ring of reference tables ([tile][quarter][Nr] per unit)
-  long long slot_expo;         // fp16 elements per ring slot
-  long long slot_refs;         // floats per ring slot
-  int n_slots;                 // unit u writes slot u % n_slots
   int part_stride;             // row length of partials and bias
   float c;                     // scale * log2(e)
   int window, pool_width, num_kv_heads, group_size, p_total, o_total, is_bf16;
-  int n_units, n_chunks, n_pieces, piece_quarters, batch;
+  int n_units, n_chunks, batch;
   int do_select;               // 0: scores only (no selection, no gather)
+  int given_lse;               // 1: no first pass; denominators from `lse`
   int q_half_bytes;            // bytes of one 64-column half of a Q buffer
+  int q_bufs;                  // Q buffers (2 or 3)
+  int row_stride;              // floats per epilogue warp row (>= max query rows, multiple of 32)
   int stages;                  // K tiles in the shared-memory ring
-  int tstride, nbuf;           // TMEM columns per accumulator buffer, buffers (even)
+  int tstride, nbuf;           // TMEM columns per accumulator buffer, buffers
+  int nwg;                     // epilogue warpgroups taking tiles (nbuf / nwg buffers each)
   int seqs_per_mask;
   int cu_seqlens[kFusedMaxSeqs + 1];
   int cu_prefix[kFusedMaxSeqs + 1];
   int cu_out[kFusedMaxSeqs + 1];
-  int chunk_off[kFusedMaxSeqs + 1];   // first scoring chunk of sequence s (units of s are consecutive)
-  int piece_off[kFusedMaxSeqs + 1];   // first combine piece of sequence s
+  int chunk_off[kFusedMaxSeqs + 1];   // first chunk of sequence s (units of s are consecutive)
   uint32_t srh_bits[kFusedMaxLists];  // per (mask, group): bit i = query head group*G + i is SRH
 };
 
 cudaError_t launch_fused(const FusedParams& p, int grid, size_t smem, cudaStream_t s);
-size_t fused_smem_bytes(int q_half_bytes, int stages);
+size_t fused_smem_bytes(int q_half_bytes, int q_bufs, int stages, int row_stride, int nwg);
+constexpr int kFusedPartsPerChunk = 4;  // first-pass pairs per chunk (epilogue warpgroups)
 cudaError_t fused_set_smem_limit(size_t bytes);
 
 // Kernel parameters travel by value; CUDA takes at most 32764 bytes of them.

@@ -4,46 +4,52 @@
 // model at the end of prefill -- pools the scores, takes the budgeted top-k,
 // appends the window and gathers the retained K/V rows.
 //
-// What is computed is what the three-kernel path computes (scoring kernel,
-// combine kernel, selection kernel), with the same arithmetic:
-//   * per K tile of 128 keys and query row q of the unit's SRH heads, the
-//     logits z = <q, k> * scale on tcgen05 tensor cores (fp32 in TMEM), the
-//     exponents e = 2^(z c - R) stored as fp16 for prefix keys (R: the
-//     owning warp's running reference, 7 below its largest scaled logit),
-//     and per query the pair (M, S) with sum 2^(z c) = S 2^M;
-//   * per unit, log2 D_q from the pairs, raw_j = sum_q e_qj 2^(R - log2 D_q),
-//     pooled_j = (sum_{t=-h..h} raw_{j+t}) / P with zeros outside [0, n);
-//   * the k = kept - W largest pooled scores (ties to the lower position) in
-//     ascending position, the window positions, and the K/V rows.
+// For unit (s, g), with Q_S the N = |S_g| * W window-query rows of the
+// group's SRH heads, z = <q, k> * scale and c = log2(e), query q (window
+// position p_q) attends key j <= p_q with 2^(z_qj c) / D_q,
+// D_q = sum_{j <= p_q} 2^(z_qj c).  The kernel makes two passes over the
+// unit's K, both on tcgen05 tensor cores (logits in TMEM):
+//   pass 1  per query row and epilogue warpgroup the pair (M, S) with
+//           sum 2^(z c) = S 2^M over its tiles of a chunk of kChunkTiles K tiles (the epilogue keeps a reference R
+//           per warp and query, 7 below the largest scaled logit it has seen,
+//           and sums 2^(z c - R) exactly as the scoring kernel of the
+//           separate path does); the workers merge a unit's pairs into
+//           log2 D_q once every chunk of the unit is in;
+//   pass 2  raw_j = sum_q 2^(z_qj c - log2 D_q) over the unit's prefix keys
+//           j < n = L - W, straight from the logits in fp32; pass 2 of a
+//           chunk is published only once its unit's denominators are merged,
+//           so it follows pass 1 closely and finds K in L2;
+// then pooled_j = (sum_{t=-h..h} raw_{j+t}) / P with zeros outside [0, n)
+// (inside a chunk by the epilogue from shared memory, within h of a chunk
+// edge by the select), the k = kept - W largest pooled scores (ties to the
+// lower position) in ascending position, the window, and the K/V rows.
+// With the window queries' log-sum-exp given (given_lse) pass 1 is skipped
+// and log2 D_q = LSE_q * log2(e).
 //
-// One CTA per SM runs for the whole call.  Its warps have fixed roles and
-// never wait on another CTA, except where noted:
-//   warp 0      claims scoring chunks (kChunkTiles tiles of one unit) from a
-//               counter, publishes each in a small descriptor ring and
-//               streams the chunk's K tiles into a shared-memory ring by TMA;
-//               before the first chunk of unit u it waits until the unit that
-//               last used u's exponent-table slot has been combined (other
-//               CTAs: bounded);
+// One CTA per SM runs for the whole call.  Its warps have fixed roles:
+//   warp 3      claims chunks (a pass-2 chunk once its unit's denominators
+//               are merged, else the next pass-1 chunk) and publishes them,
+//               up to kDescs ahead, in a descriptor ring;
+//   warp 0      streams each chunk's K tiles into a shared-memory ring by TMA;
 //   warp 1      TMEM allocation and UMMA issue (M = 128 keys, N = query rows);
-//   warp 2      copies each chunk's SRH query rows into one of two Q buffers;
+//   warp 2      copies each chunk's SRH query rows into one of two or three
+//               Q buffers;
 //   warps 4-11  two epilogue warpgroups; tile t of a chunk belongs to
-//               warpgroup t % 2, each with its own TMEM buffers;  at the end
-//               of a chunk each warpgroup writes its (M, S) pairs and counts
-//               itself in the unit's ticket;
-//   warps 12-19 combine / select workers: they claim combine pieces (a run of
-//               32-key quarters of one unit: wait for the unit's ticket, merge
-//               the pairs once per unit, weight, sum and pool the exponent
-//               rows) and, once every piece of a unit is done, the unit's
-//               selection and gather (one CTA per unit).
-// Every wait that depends on another CTA depends only on work that was
-// claimed earlier by a running CTA and that never waits on later work, so
-// the call completes whatever the number of CTAs resident at once; every
-// wait is bounded (kWaitTimeoutNs) and on expiry records
-// CKV_ERR_DEVICE_TIMEOUT and stops the call.
-// The references restart at every chunk and tile t of a chunk always goes to
-// warpgroup t % 2, so the scores depend only on the chunk grid (fixed per
-// unit), not on which CTA ran a chunk: results are deterministic and the
-// same whatever the other units of the call.
+//               warpgroup t % nwg (nwg = 2), each with its own TMEM buffers;
+//   warps 12-19 workers: they merge a unit's pass-1 pairs into its
+//               denominators once all its chunks are in, and select and
+//               gather a unit once all its pass-2 chunks are in (one CTA per
+//               unit).
+// A pass-2 chunk is published once its unit's denominators are merged (the
+// epilogue still checks, bounded); workers claim a merge or a selection only
+// when it is ready.  Every wait therefore depends only on
+// work claimed earlier by a running CTA that never waits on later work, so a
+// call completes whatever the number of CTAs resident at once; every wait
+// is bounded (kWaitTimeoutNs) and on expiry records CKV_ERR_DEVICE_TIMEOUT
+// and stops the call.
+// References restart at every chunk and tile t of a chunk always goes to
+// warpgroup t % nwg, so the scores depend only on the chunk grid (fixed per
+// unit), not on which CTA ran a chunk or what else the call holds.
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
@@ -61,51 +67,51 @@ constexpr int kFThreads = 32 * kFWarps;
 constexpr int kProdWarp = 0;
 constexpr int kMmaWarp = 1;
 constexpr int kStageWarp = 2;
+constexpr int kClaimWarp = 3;
 constexpr int kEpiWarp0 = 4;  // warps 4..11: two warpgroups (TMEM lane quarter = warp % 4)
 constexpr int kEpiWarps = 8;
 constexpr int kCWarp0 = 12;   // warps 12..19
 constexpr int kCThreads = 256;
-constexpr int kDescs = 4;     // chunk descriptors in flight
-constexpr int kBarC = 3;      // named barrier of the combine / select warps (1, 2: warpgroups)
+constexpr int kDescs = 4;     // chunk descriptors in flight (claimed ahead)
+constexpr int kBarC = 3;      // named barrier of the worker warps
 constexpr float kShift = 7.0f;
-constexpr float kRaise = 15.0f;
+constexpr float kRaise = 64.0f;  // fp32 sums: exponents stay below 2^64 before R is raised
 constexpr float kNegInf = -INFINITY;
-constexpr int kLoadBatch = 4;
 
 // counters (ints at p.ctr)
-constexpr int kCtrChunk = 0;  // next scoring chunk
-constexpr int kCtrPiece = 1;  // next combine piece
-constexpr int kCtrSel = 2;    // next unit to select
-constexpr int kCtrExit = 3;   // CTAs finished
-constexpr int kCtrAbort = 4;  // set when any wait ran out
+constexpr int kCtrPass1 = 0;  // next pass-1 chunk
+constexpr int kCtrPass2 = 1;  // next pass-2 chunk
+constexpr int kCtrMerge = 2;  // next unit whose denominators to merge
+constexpr int kCtrSel = 3;    // next unit to select
+constexpr int kCtrExit = 4;   // CTAs finished
+constexpr int kCtrAbort = 5;  // set when any wait ran out
 
 constexpr int kTaskEnd = 0;
-constexpr int kTaskCombine = 1;
+constexpr int kTaskMerge = 1;
 constexpr int kTaskSelect = 2;
 
 struct ChunkDesc {
-  int end, s, g, t0, t1, chunk, n_rows, list;
+  int end, pass, s, g, t0, t1, chunk, n_rows;
 };
 
-// Shared memory of the combine / select workers (one of the two at a time).
+// Shared memory of the worker warps (a merge or a selection at a time).
 struct SelShared {
   int samp[256];
   uint32_t key[kFusedCandCap];
   int pos[kFusedCandCap];
   RadixShared rs;
   int wcnt[8], wbase[8];
-  int red[2];
+  int flag[4];
   uint32_t lo;
 };
 static_assert(sizeof(SelShared) <= kFusedCRegion, "select scratch");
+static_assert(3 * kMaxQRows * 4 + 16 <= kFusedCRegion, "merge scratch");
 
-// Fixed part of the dynamic shared memory (after the K ring and Q buffers).
-constexpr int kRefBytes = kEpiWarps * kMaxQRows * 4;  // running references per epilogue warp
-constexpr int kAccBytes = kEpiWarps * kMaxQRows * 4;  // per-query sums per epilogue warp
 constexpr int kWposBytes = kMaxQRows * 4;
+constexpr int kChunkBufBytes = 2 * kChunkKeys * 4;  // raw scores of two pass-2 chunks
 constexpr int kBarBytes = 512;
-constexpr int kMiscBytes = 256;  // TMEM address, abort flag, task, descriptors
-constexpr int kFixedBytes = kRefBytes + kAccBytes + kWposBytes + kBarBytes + kMiscBytes +
+constexpr int kMiscBytes = 256;  // TMEM address, abort flag, task
+constexpr int kFixedBytes = kWposBytes + kChunkBufBytes + kBarBytes + kMiscBytes +
                             kDescs * static_cast<int>(sizeof(ChunkDesc));
 
 __device__ __forceinline__ int ld_acquire(const int* p) {
@@ -145,20 +151,11 @@ struct Fused {
   __device__ int chunks_per_unit(int s) const {
     return (p.chunk_off[s + 1] - p.chunk_off[s]) / p.num_kv_heads;
   }
-  __device__ int pieces_per_unit(int s) const {
-    return (p.piece_off[s + 1] - p.piece_off[s]) / p.num_kv_heads;
-  }
   __device__ int list(int s, int g) const { return srh_group(s, g, p.seqs_per_mask, p.num_kv_heads); }
   __device__ int rows(int s, int g) const { return __popc(p.srh_bits[list(s, g)]) * p.window; }
   __device__ int* ticket(int u) const { return p.ctr + kFusedCtrHead + u; }
-  __device__ int* combdone(int u) const { return p.ctr + kFusedCtrHead + p.n_units + u; }
+  __device__ int* p2done(int u) const { return p.ctr + kFusedCtrHead + p.n_units + u; }
   __device__ int* bias_state(int u) const { return p.ctr + kFusedCtrHead + 2 * p.n_units + u; }
-  __device__ uint16_t* expo_slot(int u) const {
-    return p.expo + static_cast<long long>(u % p.n_slots) * p.slot_expo;
-  }
-  __device__ float* refs_slot(int u) const {
-    return p.refs + static_cast<long long>(u % p.n_slots) * p.slot_refs;
-  }
   __device__ bool aborted() const { return ld_volatile(p.ctr + kCtrAbort) != 0; }
   __device__ void raise_abort() const {
     atomicCAS(p.status, 0, CKV_DEV_ERR_TIMEOUT);
@@ -171,7 +168,7 @@ struct Fused {
     if (ld_acquire(ptr) >= target) return true;
     const uint64_t t0 = globaltimer_ns();
     for (;;) {
-      __nanosleep(128);
+      __nanosleep(64);
       if (ld_acquire(ptr) >= target) return true;
       if (aborted() || *reinterpret_cast<volatile int*>(abort_cta)) return false;
       if (globaltimer_ns() - t0 > kWaitTimeoutNs) {
@@ -188,78 +185,66 @@ struct Fused {
   }
 };
 
-// ---------------------------------------------------------------- combine
-__device__ __forceinline__ float dot8w(const uint4 v, const float* w) {
-  const __half2* h = reinterpret_cast<const __half2*>(&v);
-  const float4 w0 = *reinterpret_cast<const float4*>(w);
-  const float4 w1 = *reinterpret_cast<const float4*>(w + 4);
-  const float2 a = __half22float2(h[0]);
-  const float2 b = __half22float2(h[1]);
-  const float2 c = __half22float2(h[2]);
-  const float2 d = __half22float2(h[3]);
-  float s = a.x * w0.x;
-  s = fmaf(a.y, w0.y, s);
-  s = fmaf(b.x, w0.z, s);
-  s = fmaf(b.y, w0.w, s);
-  s = fmaf(c.x, w1.x, s);
-  s = fmaf(c.y, w1.y, s);
-  s = fmaf(d.x, w1.z, s);
-  s = fmaf(d.y, w1.w, s);
-  return s;
+// ---------------------------------------------------------------- claims
+// The next chunk of this CTA.  Each claimer holds at most one pass-2 chunk it
+// has claimed (*pending, taken with atomicAdd as soon as the previous one was
+// published) and publishes it once its unit's denominators are merged (with
+// the LSE given: at once); until then it claims pass-1 chunks.  Pass 1 keeps
+// advancing while pass-2 chunks wait, and a pass-2 chunk never reaches the
+// epilogue before its denominators.  When pass 1 is exhausted the claimer
+// waits (bounded) for its pending chunk's unit, whose pass-1 chunks are then
+// all claimed.  Returns false when both passes are exhausted (or aborted).
+__device__ bool claim_chunk(const Fused& F, int* pending, int* pass, int* x) {
+  const FusedParams& p = F.p;
+  for (;;) {
+    if (F.aborted() || *reinterpret_cast<volatile int*>(F.abort_cta)) return false;
+    if (*pending < 0 && ld_volatile(p.ctr + kCtrPass2) < p.n_chunks) {
+      const int y = atomicAdd(p.ctr + kCtrPass2, 1);
+      if (y < p.n_chunks) *pending = y;
+    }
+    int u = -1;
+    if (*pending >= 0) {
+      const int s = find_seq(p.chunk_off, p.batch, *pending);
+      u = s * p.num_kv_heads + (*pending - p.chunk_off[s]) / F.chunks_per_unit(s);
+      if (p.given_lse || ld_acquire(F.bias_state(u)) >= 2) {
+        *pass = 2;
+        *x = *pending;
+        *pending = -1;
+        return true;
+      }
+    }
+    if (!p.given_lse && ld_volatile(p.ctr + kCtrPass1) < p.n_chunks) {
+      const int y = atomicAdd(p.ctr + kCtrPass1, 1);
+      if (y < p.n_chunks) {
+        *pass = 1;
+        *x = y;
+        return true;
+      }
+      continue;
+    }
+    if (*pending < 0) return false;  // both passes exhausted
+    // pass 1 is exhausted: every pass-1 chunk of the pending chunk's unit is claimed
+    if (!F.wait_counter(F.bias_state(u), 2)) return false;
+  }
 }
 
-// One combine piece: quarters [q_first, q_last) of unit (s, g).  All 256
-// worker threads (ct = 0..255).  Returns false if the call was aborted.
-__device__ __noinline__ bool combine_piece(const Fused& F, int x, uint8_t* creg, int ct) {
+// ---------------------------------------------------------------- merge
+// log2 D_q of unit u from its pass-1 pairs (one per chunk and warpgroup that
+// takes tiles; one that got no tile of a chunk leaves (-inf, 0)), 256 worker
+// threads: nm threads per query row, sixteen pairs in flight per thread.
+__device__ __noinline__ void merge_unit(const Fused& F, int u, uint8_t* creg, int ct) {
   const FusedParams& p = F.p;
-  const int s = find_seq(p.piece_off, p.batch, x);
-  const int npc = F.pieces_per_unit(s);
-  const int local = x - p.piece_off[s];
-  const int g = local / npc;
-  const int pc = local - g * npc;
-  const int u = s * p.num_kv_heads + g;
-  const int n = F.prefix(s);
+  const int s = u / p.num_kv_heads;
+  const int g = u - s * p.num_kv_heads;
   const int N = F.rows(s, g);
-  const int Nr = expo_stride(N);
-  const int cpr = Nr >> 3;
-  const int lg_cpr = __ffs(cpr) - 1;
-  const int col = ct & (cpr - 1);
-  const int h = (p.pool_width - 1) >> 1;
-  const int quarters = (n + 31) >> 5;
-  const int qa = pc * p.piece_quarters;
-  const int qb = min(quarters, qa + p.piece_quarters);
-  const int a = qa * 32;
-  const int b = min(qb * 32, n);
-  const int base = a - h;
-  const int span = b - a + 2 * h;
-  const int ea = max(base, 0);
-  const int eb = min(b + h, n);
-  const int q0 = ea >> 5;
-  const int nqt = ((eb + 31) >> 5) - q0;
-  float* s_bias = reinterpret_cast<float*>(creg);             // [256]
-  float* s_mm = s_bias + kMaxQRows;                           // [256] merge scratch (M)
-  float* s_mz = s_mm + kMaxQRows;                             // [256] merge scratch (S)
-  int* s_flag = reinterpret_cast<int*>(s_mz + kMaxQRows);     // [4]
-  float* s_w = s_mz + kMaxQRows + 4;                          // [nqt][Nr] (16-byte aligned)
-  float* s_raw = s_w + nqt * Nr;                              // [span]
-
-  for (int i = ct; i < span; i += kCThreads) s_raw[i] = 0.f;
-  // every scoring contribution of the unit (two per chunk) has landed
-  if (ct == 0) {
-    const bool ok = F.wait_counter(F.ticket(u), 2 * F.chunks_per_unit(s));
-    s_flag[0] = ok ? 1 : 0;
-    s_flag[1] = ok ? atomicCAS(F.bias_state(u), 0, 1) : 2;
-  }
-  cbar();
-  if (!s_flag[0]) return false;
-  float* bias_g = p.bias + static_cast<long long>(u) * p.part_stride;
-  if (s_flag[1] == 0) {
-    // this piece merges the unit's pairs once: nm threads per query row,
-    // sixteen pairs in flight per thread
-    const int nparts = 2 * F.chunks_per_unit(s);
-    const float2* parts =
-        p.partials + static_cast<long long>(p.chunk_off[s] + g * F.chunks_per_unit(s)) * 2 *
-                         p.part_stride;
+  const int ncu = F.chunks_per_unit(s);
+  float* s_mm = reinterpret_cast<float*>(creg);  // [256]
+  float* s_mz = s_mm + kMaxQRows;                 // [256]
+  if (ncu > 0 && N > 0) {
+    const int nwg = p.nwg;
+    const int nparts = nwg * ncu;  // the unit's chunks are consecutive
+    const float2* parts = p.partials + static_cast<long long>(p.chunk_off[s] + g * ncu) *
+                                           kFusedPartsPerChunk * p.part_stride;
     const int nm = kCThreads / N;
     const int q = ct % N;
     const int sub = ct / N;
@@ -269,9 +254,11 @@ __device__ __noinline__ bool combine_piece(const Fused& F, int x, uint8_t* creg,
         float2 pr[16];
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
-          const int i = i0 + k * nm;
-          pr[k] = i < nparts ? __ldcg(parts + static_cast<long long>(i) * p.part_stride + q)
-                             : make_float2(kNegInf, 0.f);
+          const int i = i0 + k * nm;  // pair i: chunk i / nwg, warpgroup i % nwg
+          pr[k] = i < nparts
+                      ? __ldcg(parts + (static_cast<long long>(i / nwg) * kFusedPartsPerChunk +
+                                        i % nwg) * p.part_stride + q)
+                      : make_float2(kNegInf, 0.f);
         }
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
@@ -301,91 +288,12 @@ __device__ __noinline__ bool combine_piece(const Fused& F, int x, uint8_t* creg,
           z = fmaf(pz, ex2_approx(pm - m), z);
         }
       }
-      const float bq = m + __log2f(z);
-      s_bias[ct] = bq;
-      bias_g[ct] = bq;
+      p.bias[static_cast<long long>(u) * p.part_stride + ct] = m + __log2f(z);
     }
-    __threadfence();
-    cbar();
-    if (ct == 0) atomicExch(F.bias_state(u), 2);
-  } else {
-    if (ct == 0) s_flag[2] = F.wait_counter(F.bias_state(u), 2) ? 1 : 0;
-    cbar();
-    if (!s_flag[2]) return false;  // (a slot no thread still reads)
-    if (ct < N) s_bias[ct] = __ldcg(bias_g + ct);
-  }
-  // references of the quarters touched (the piece plus an h-key halo each
-  // side), turned into weights 2^(R - log2 D_q) in place
-  const float* R = F.refs_slot(u) + static_cast<long long>(q0) * Nr;
-  for (int i = 4 * ct; i < nqt * Nr; i += 4 * kCThreads)
-    *reinterpret_cast<float4*>(s_w + i) = __ldcg(reinterpret_cast<const float4*>(R + i));
-  cbar();
-  for (int i = ct; i < nqt * Nr; i += kCThreads) {
-    const int cc = i & (Nr - 1);
-    s_w[i] = cc < N ? ex2_approx(s_w[i] - s_bias[cc]) : 0.f;
-  }
-  cbar();
-  // raw scores of keys [ea, eb): one contiguous run of exponent rows
-  const uint4* E4 = reinterpret_cast<const uint4*>(F.expo_slot(u));
-  const int f_lo = ea * cpr;
-  const int f_hi = eb * cpr;
-  uint4 ev[kLoadBatch];
-#pragma unroll
-  for (int k = 0; k < kLoadBatch; ++k) {
-    const int f = f_lo + k * kCThreads + ct;
-    ev[k] = f < f_hi ? __ldcg(E4 + f) : make_uint4(0u, 0u, 0u, 0u);
-  }
-  for (int f0 = f_lo; f0 < f_hi; f0 += kLoadBatch * kCThreads) {
-    uint4 nx[kLoadBatch];
-    const int f1 = f0 + kLoadBatch * kCThreads;
-    if (f1 < f_hi) {
-#pragma unroll
-      for (int k = 0; k < kLoadBatch; ++k) {
-        const int f = f1 + k * kCThreads + ct;
-        nx[k] = f < f_hi ? __ldcg(E4 + f) : make_uint4(0u, 0u, 0u, 0u);
-      }
-    }
-#pragma unroll
-    for (int k = 0; k < kLoadBatch; ++k) {
-      const int f = f0 + k * kCThreads + ct;
-      const int row = f >> lg_cpr;
-      const int qq = min((row >> 5) - q0, nqt - 1);
-      float v = dot8w(ev[k], s_w + qq * Nr + 8 * col);
-      for (int off = cpr >> 1; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-      if (f < f_hi && col == 0) s_raw[row - base] = v;
-    }
-    if (f1 < f_hi) {
-#pragma unroll
-      for (int k = 0; k < kLoadBatch; ++k) ev[k] = nx[k];
-    }
-  }
-  cbar();
-  // table lines no other piece reads (inside [a + h, b - h)) need no
-  // write-back to DRAM
-  {
-    const long long row_bytes = static_cast<long long>(Nr) * 2;
-    const uintptr_t tb = reinterpret_cast<uintptr_t>(F.expo_slot(u));
-    const long long lo_b = ((static_cast<long long>(a + h + 1) * row_bytes + 127) / 128) * 128;
-    const long long hi_b = ((static_cast<long long>(b - h - 1) * row_bytes) / 128) * 128;
-    for (long long xb = lo_b + static_cast<long long>(ct) * 128; xb + 128 <= hi_b;
-         xb += static_cast<long long>(kCThreads) * 128) {
-      const char* line = reinterpret_cast<const char*>(tb) + xb;
-      asm volatile("discard.global.L2 [%0], 128;" ::"l"(line) : "memory");
-    }
-  }
-  const long long soff = static_cast<long long>(g) * p.p_total + p.cu_prefix[s];
-  const float fP = static_cast<float>(p.pool_width);
-  for (int j = a + ct; j < b; j += kCThreads) {
-    const int i = j - a;
-    float acc = 0.f;
-    for (int t = 0; t <= 2 * h; ++t) acc += s_raw[i + t];
-    p.pooled[soff + j] = acc / fP;
-    if (p.raw_out) p.raw_out[soff + j] = s_raw[i + h];
   }
   __threadfence();
   cbar();
-  if (ct == 0) atomicAdd(F.combdone(u), 1);
-  return true;
+  if (ct == 0) atomicExch(F.bias_state(u), 2);
 }
 
 // ---------------------------------------------------------------- select
@@ -552,11 +460,24 @@ __device__ __noinline__ void gather_rows(const FusedParams& p, int seq0, int g,
   }
 }
 
-// Selection of unit u: top-k of its pooled scores by a sampled lower bound,
-// candidates in position order, an exact radix search among them (all the
-// unit's scores when the bound keeps too few or too many), the window, and
-// the K/V rows.  Pooled scores are >= 0: their bit patterns order like
-// their values.
+// Pooled score of prefix key j from the raw scores (zeros outside [0, n)),
+// summed in the order the epilogue's chunk pooling uses.
+__device__ __forceinline__ float pool_from_global(const float* raw, int n, int j, int h,
+                                                  float fP) {
+  float acc = 0.f;
+  for (int t = 0; t <= 2 * h; ++t) {
+    const int jj = j - h + t;
+    acc += (jj >= 0 && jj < n) ? __ldcg(raw + jj) : 0.f;
+  }
+  return acc / fP;
+}
+
+// Selection of unit u.  First the pooled scores within h of a chunk edge
+// (the epilogue pooled each chunk's interior), then the top-k by a sampled
+// lower bound: candidates in position order, an exact radix search among
+// them (among all the unit's scores when the bound keeps too few or too
+// many), the window, and the K/V rows.  Pooled scores are >= 0: their bit
+// patterns order like their values.
 __device__ __noinline__ void select_unit(const Fused& F, int u, uint8_t* creg, int ct) {
   const FusedParams& p = F.p;
   SelShared& sh = *reinterpret_cast<SelShared*>(creg);
@@ -570,6 +491,28 @@ __device__ __noinline__ void select_unit(const Fused& F, int u, uint8_t* creg, i
   const int n = F.prefix(s);
   const int out0 = p.cu_out[s];
   const int kept = p.cu_out[s + 1] - out0;
+  const long long soff = static_cast<long long>(g) * p.p_total + p.cu_prefix[s];
+  float* pooled = p.pooled + soff;
+  const int h = (p.pool_width - 1) >> 1;
+  const float fP = static_cast<float>(p.pool_width);
+  // chunk-edge pooled scores: [a, a + h) and [b - h, b) of every chunk
+  if (h > 0 && n > 0) {
+    const float* raw = p.raw + soff;
+    const int nct = (n + kChunkKeys - 1) / kChunkKeys;
+    for (int e = ct; e < nct * 2 * h; e += kCThreads) {
+      const int c = e / (2 * h);
+      const int o = e - c * 2 * h;
+      const int a = c * kChunkKeys;
+      const int b = min(a + kChunkKeys, n);
+      const int lo_end = min(a + h, b);
+      const int hi_start = max(b - h, lo_end);
+      const int j = o < h ? a + o : hi_start + (o - h);
+      if (o < h ? j < lo_end : j < b) pooled[j] = pool_from_global(raw, n, j, h, fP);
+    }
+    __threadfence();
+  }
+  cbar();
+  if (!p.do_select) return;
   int32_t* out = p.indices + static_cast<long long>(g) * p.o_total + out0;
   if (kept >= L) {  // keep everything
     for (int i = ct; i < L; i += kCThreads) out[i] = i;
@@ -581,13 +524,12 @@ __device__ __noinline__ void select_unit(const Fused& F, int u, uint8_t* creg, i
   const int k = kept - W;  // 0 <= k < n
   for (int w = ct; w < W; w += kCThreads) out[k + w] = n + w;
   if (k == 0) {
+    __threadfence_block();
     cbar();
     gather_rows(p, seq0, g, out, out0, W, ct);
     return;
   }
-  const uint32_t* keys = reinterpret_cast<const uint32_t*>(
-      p.pooled + static_cast<long long>(g) * p.p_total + p.cu_prefix[s]);
-  // samples: ns evenly spaced keys
+  const uint32_t* keys = reinterpret_cast<const uint32_t*>(pooled);
   const int ns = min(256, n);
   sh.samp[ct] = ct < ns ? static_cast<int>(__ldcg(keys + static_cast<int>(
                                                   (static_cast<long long>(ct) * n) / ns)))
@@ -598,8 +540,8 @@ __device__ __noinline__ void select_unit(const Fused& F, int u, uint8_t* creg, i
   int rs = min(ns, static_cast<int>(ceilf(mu + 3.f * sqrtf(mu))) + 2);
   uint32_t lo = 0;
   int total = 0;
-  // positions per warp (multiple of 32)
-  const int seg = ((n + 8 * 32 - 1) / (8 * 32)) * 32;
+  constexpr int kU = 8;  // loads in flight per lane
+  const int seg = ((n + 8 * 32 * kU - 1) / (8 * 32 * kU)) * 32 * kU;  // positions per warp
   const int wlo = min(n, cw * seg);
   const int whi = min(n, wlo + seg);
   bool fast = false;
@@ -619,9 +561,16 @@ __device__ __noinline__ void select_unit(const Fused& F, int u, uint8_t* creg, i
     cbar();
     lo = sh.lo;
     int wc = 0;
-    for (int b0 = wlo; b0 < whi; b0 += 32) {
-      const int i = b0 + lane;
-      wc += __popc(__ballot_sync(0xffffffffu, i < whi && __ldcg(keys + i) >= lo));
+    for (int b0 = wlo; b0 < whi; b0 += 32 * kU) {
+      uint32_t kv[kU];
+#pragma unroll
+      for (int q = 0; q < kU; ++q) {
+        const int i = b0 + q * 32 + lane;
+        kv[q] = i < whi ? __ldcg(keys + i) : 0u;
+      }
+#pragma unroll
+      for (int q = 0; q < kU; ++q)
+        wc += __popc(__ballot_sync(0xffffffffu, b0 + q * 32 + lane < whi && kv[q] >= lo));
     }
     if (lane == 0) sh.wcnt[cw] = wc;
     cbar();
@@ -643,17 +592,25 @@ __device__ __noinline__ void select_unit(const Fused& F, int u, uint8_t* creg, i
     // candidates (keys >= lo) in position order
     int o = 0;
     for (int w = 0; w < cw; ++w) o += sh.wcnt[w];
-    for (int b0 = wlo; b0 < whi; b0 += 32) {
-      const int i = b0 + lane;
-      const uint32_t key = i < whi ? __ldcg(keys + i) : 0u;
-      const bool c = i < whi && key >= lo;
-      const uint32_t mm = __ballot_sync(0xffffffffu, c);
-      const int slot = o + __popc(mm & lanemask_lt(lane));
-      if (c) {
-        sh.key[slot] = key;
-        sh.pos[slot] = i;
+    for (int b0 = wlo; b0 < whi; b0 += 32 * kU) {
+      uint32_t kv[kU];
+#pragma unroll
+      for (int q = 0; q < kU; ++q) {
+        const int i = b0 + q * 32 + lane;
+        kv[q] = i < whi ? __ldcg(keys + i) : 0u;
       }
-      o += __popc(mm);
+#pragma unroll
+      for (int q = 0; q < kU; ++q) {
+        const int i = b0 + q * 32 + lane;
+        const bool c = i < whi && kv[q] >= lo;
+        const uint32_t mm = __ballot_sync(0xffffffffu, c);
+        const int slot = o + __popc(mm & lanemask_lt(lane));
+        if (c) {
+          sh.key[slot] = kv[q];
+          sh.pos[slot] = i;
+        }
+        o += __popc(mm);
+      }
     }
     cbar();
     constexpr uint32_t kClamp = 0xFFFFu;
@@ -674,20 +631,18 @@ __device__ __noinline__ void select_unit(const Fused& F, int u, uint8_t* creg, i
   gather_rows(p, seq0, g, out, out0, kept, ct);
 }
 
-
-// Claim the workers' next task (one thread): the next unit to select once all
-// its combine pieces are done, else the next combine piece, else wait for
-// the next selection to become ready.  Without selection (scores only) the
-// workers stop when every piece is claimed.
+// The workers' next task (one thread): the next unit to select once all its
+// pass-2 chunks are in, else the next unit to merge once all its pass-1
+// chunks are in; waits (bounded) while neither is ready.
 __device__ void claim_task(const Fused& F, int* task) {
   const FusedParams& p = F.p;
   uint64_t t0 = 0;
   for (;;) {
     if (F.aborted() || *reinterpret_cast<volatile int*>(F.abort_cta)) break;
-    const int u = p.do_select ? ld_volatile(p.ctr + kCtrSel) : p.n_units;
-    if (u >= p.n_units && ld_volatile(p.ctr + kCtrPiece) >= p.n_pieces)
-      break;  // every unit selected (every piece combined), or scores only and no piece left
-    if (u < p.n_units && ld_acquire(F.combdone(u)) >= F.pieces_per_unit(u / p.num_kv_heads)) {
+    const int u = ld_volatile(p.ctr + kCtrSel);
+    if (u >= p.n_units) break;  // every unit selected (and therefore merged)
+    const int s = u / p.num_kv_heads;
+    if (ld_acquire(F.p2done(u)) >= kEpiWarps * F.chunks_per_unit(s)) {  // every epilogue warp
       if (atomicCAS(p.ctr + kCtrSel, u, u + 1) == u) {
         task[0] = kTaskSelect;
         task[1] = u;
@@ -695,15 +650,18 @@ __device__ void claim_task(const Fused& F, int* task) {
       }
       continue;
     }
-    if (ld_volatile(p.ctr + kCtrPiece) < p.n_pieces) {
-      const int x = atomicAdd(p.ctr + kCtrPiece, 1);
-      if (x < p.n_pieces) {
-        task[0] = kTaskCombine;
-        task[1] = x;
-        return;
+    if (!p.given_lse) {
+      const int m = ld_volatile(p.ctr + kCtrMerge);
+      if (m < p.n_units &&
+          ld_acquire(F.ticket(m)) >= p.nwg * F.chunks_per_unit(m / p.num_kv_heads)) {
+        if (atomicCAS(p.ctr + kCtrMerge, m, m + 1) == m) {
+          task[0] = kTaskMerge;
+          task[1] = m;
+          return;
+        }
+        continue;
       }
     }
-    // every piece is claimed; the next unit's last pieces are still running
     const uint64_t now = globaltimer_ns();
     if (t0 == 0) {
       t0 = now;
@@ -711,10 +669,42 @@ __device__ void claim_task(const Fused& F, int* task) {
       F.raise_abort();
       break;
     }
-    __nanosleep(256);
+    __nanosleep(128);
   }
   task[0] = kTaskEnd;
   task[1] = 0;
+}
+
+// Pass 1, rare: an exponent of this 32-column group passed 2^kRaise (or the
+// references are still -inf): raise every query's R to kShift below its
+// largest scaled logit among the warp's 32 keys, shrink the sums kept against
+// the old R, and return this group's column sums against the new R (column
+// lane).  The whole warp calls it; taddr is the group's first TMEM column.
+__device__ __noinline__ float p1_raise_group(uint32_t taddr, float* rf, float* acc_c,
+                                             const int* wpos, int lim, bool edge, bool key,
+                                             int vis, float c, int lane) {
+  uint32_t r[32];
+  tmem_load32_async(taddr, r);
+  tmem_wait_ld(r);
+  uint32_t valid = 0u;
+  float v[32];
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    const bool ok = j < lim && (!edge || (key && wpos[j] >= -vis));
+    valid |= (ok ? 1u : 0u) << j;
+    v[j] = ok ? __uint_as_float(r[j]) * c : kNegInf;
+  }
+  const float m = warp_transpose_max32(v, lane);  // column lane
+  const float old = rf[lane];
+  const float nw = fmaxf(old, m - kShift);
+  acc_c[lane] *= (nw == old) ? 1.f : ((old == kNegInf) ? 0.f : ex2_approx(old - nw));
+  __syncwarp();
+  rf[lane] = nw;
+  __syncwarp();
+#pragma unroll
+  for (int j = 0; j < 32; ++j)
+    v[j] = ((valid >> j) & 1u) ? ex2_approx(fmaf(__uint_as_float(r[j]), c, -rf[j])) : 0.f;
+  return warp_transpose_sum32(v, lane);
 }
 
 __device__ __forceinline__ void wait_plain(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
@@ -728,12 +718,16 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
                                              ~static_cast<uintptr_t>(1023));
   const int nst = p.stages;
   const int qh = p.q_half_bytes;
+  const int rstride = p.row_stride;
   uint8_t* sK = base;
-  uint8_t* sQ = base + nst * kTileBytes;  // two buffers of two 64-column halves
-  float* sRef = reinterpret_cast<float*>(sQ + 4 * qh);
-  float* sAcc = sRef + kEpiWarps * kMaxQRows;
-  int* sWpos = reinterpret_cast<int*>(sAcc + kEpiWarps * kMaxQRows);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sWpos + kMaxQRows);
+  const int nqb = p.q_bufs;
+  uint8_t* sQ = base + nst * kTileBytes;  // nqb buffers of two 64-column halves
+  const int nrow = 4 * p.nwg;  // epilogue warps that take tiles
+  float* sRef = reinterpret_cast<float*>(sQ + 2 * nqb * qh);  // [nrow][rstride]
+  float* sAcc = sRef + nrow * rstride;                        // [nrow][rstride]
+  int* sWpos = reinterpret_cast<int*>(sAcc + nrow * rstride);
+  float* sChunk = reinterpret_cast<float*>(sWpos + kMaxQRows);  // [2][kChunkKeys]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sChunk + 2 * kChunkKeys);
   uint8_t* misc = reinterpret_cast<uint8_t*>(bars) + kBarBytes;
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(misc);
   int* abort_cta = reinterpret_cast<int*>(misc + 4);
@@ -750,8 +744,9 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
   auto dfull = [&](int i) { return bar0 + 8u * (32 + i); };     // descriptor written
   auto dempty = [&](int i) { return bar0 + 8u * (36 + i); };    // descriptor read by all
   auto qfull = [&](int i) { return bar0 + 8u * (40 + i); };     // Q buffer staged
-  auto qempty = [&](int i) { return bar0 + 8u * (42 + i); };    // Q buffer's MMAs done
-  auto wgbar = [&](int w) { return bar0 + 8u * (44 + w); };     // epilogue warpgroup sync
+  auto qempty = [&](int i) { return bar0 + 8u * (43 + i); };    // Q buffer's MMAs done
+  auto wgbar = [&](int w) { return bar0 + 8u * (46 + w); };     // epilogue warpgroup sync
+  const uint32_t epibar = bar0 + 8u * 50;                       // all epilogue warps
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -770,13 +765,14 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
     }
     for (int i = 0; i < kDescs; ++i) {
       mbar_init(dfull(i), 1);
-      mbar_init(dempty(i), 2 + kEpiWarps);  // MMA, stager, epilogue warps
+      mbar_init(dempty(i), 3 + kEpiWarps);  // TMA producer, MMA, stager, epilogue warps
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < 3; ++i) {
       mbar_init(qfull(i), 1);
       mbar_init(qempty(i), 1);
-      mbar_init(wgbar(i), 4);
     }
+    for (int i = 0; i < 4; ++i) mbar_init(wgbar(i), 4);
+    mbar_init(epibar, kEpiWarps);
     *abort_cta = 0;
     fence_mbar_init();
   }
@@ -790,44 +786,51 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
   tc_fence_after();
   const uint32_t tbase = *tmem_holder;
 
-  if (warp == kProdWarp) {
-    // ------------------------------------------------------------ chunks + TMA
+  if (warp == kClaimWarp) {
+    // ------------------------------------------------------------ chunk claims
     if (lane == 0) {
-      const uint64_t kpol = l2_policy_evict_first();
-      int gt = 0;  // K tiles issued
+      int pending = -1;  // pass-2 chunk claimed, not yet published
       for (int c = 0;; ++c) {
         const int ds = c % kDescs;
         if (!F.wait_bar(dempty(ds), ((c / kDescs) & 1) ^ 1)) break;
         ChunkDesc d;
         d.end = 1;
-        const int x = F.aborted() ? p.n_chunks : atomicAdd(p.ctr + kCtrChunk, 1);
-        if (x < p.n_chunks) {
+        int pass = 0, x = 0;
+        if (claim_chunk(F, &pending, &pass, &x)) {
           const int s = find_seq(p.chunk_off, p.batch, x);
           const int ncu = F.chunks_per_unit(s);
           const int local = x - p.chunk_off[s];
           const int g = local / ncu;
           const int cc = local - g * ncu;
-          const int u = s * Hkv + g;
-          // the exponent-table slot's previous unit has been combined
-          bool ok = true;
-          if (u >= p.n_slots) {
-            const int up = u - p.n_slots;
-            ok = F.wait_counter(F.combdone(up), F.pieces_per_unit(up / Hkv));
-          }
-          if (ok) {
-            d.end = 0;
-            d.s = s;
-            d.g = g;
-            d.t0 = cc * kChunkTiles;
-            d.t1 = min(F.tiles(s), d.t0 + kChunkTiles);
-            d.chunk = x;
-            d.list = F.list(s, g);
-            d.n_rows = __popc(p.srh_bits[d.list]) * W;
-          }
+          d.end = 0;
+          d.pass = pass;
+          d.s = s;
+          d.g = g;
+          d.t0 = cc * kChunkTiles;
+          d.t1 = min(F.tiles(s), d.t0 + kChunkTiles);
+          d.chunk = x;
+          d.n_rows = F.rows(s, g);
         }
         descs[ds] = d;
         mbar_arrive(dfull(ds));
         if (d.end) break;
+      }
+    }
+    __syncwarp();
+  } else if (warp == kProdWarp) {
+    // ------------------------------------------------------------ TMA
+    if (lane == 0) {
+      // pass 1 keeps K in L2 for pass 2, which reads it for the last time
+      const uint64_t pol1 = l2_policy_evict_last();
+      const uint64_t pol2 = l2_policy_evict_first();
+      int gt = 0;  // K tiles issued
+      for (int c = 0;; ++c) {
+        const int ds = c % kDescs;
+        if (!F.wait_bar(dfull(ds), static_cast<uint32_t>(c / kDescs) & 1u)) break;
+        const ChunkDesc d = descs[ds];
+        mbar_arrive(dempty(ds));
+        if (d.end) break;
+        const uint64_t pol = d.pass == 1 ? pol1 : pol2;
         const int row0 = p.cu_seqlens[d.s];
         bool stop = false;
         for (int t = d.t0; t < d.t1; ++t) {
@@ -839,8 +842,8 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
           mbar_arrive_expect_tx(full(st), kTileBytes);
           const uint32_t dst = smem_u32(sK + st * kTileBytes);
           const int row = row0 + t * kTileTokens;
-          tma_load_3d(dst, &p.tmap_k, full(st), 0, d.g, row, kpol);
-          tma_load_3d(dst + kHalfTileBytes, &p.tmap_k, full(st), 64, d.g, row, kpol);
+          tma_load_3d(dst, &p.tmap_k, full(st), 0, d.g, row, pol);
+          tma_load_3d(dst + kHalfTileBytes, &p.tmap_k, full(st), 64, d.g, row, pol);
           ++gt;
         }
         if (stop) break;
@@ -856,9 +859,10 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
     // ------------------------------------------------------------ UMMA issue
     if (lane == 0) {
       const uint64_t dk0 = smem_desc_sw128(smem_u32(sK));
-      const int half = p.nbuf >> 1;
+      const int nwg = p.nwg;
+      const int bpw = p.nbuf / nwg;  // TMEM buffers per warpgroup
       int gt = 0;
-      int kw[2] = {0, 0};
+      int kw[4] = {0, 0, 0, 0};
       int last_b = -1;
       uint32_t last_use = 0;
       for (int c = 0;; ++c) {
@@ -867,18 +871,18 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
         const ChunkDesc d = descs[ds];
         mbar_arrive(dempty(ds));
         if (d.end) break;
-        const int qb = c & 1;
-        if (!F.wait_bar(qfull(qb), static_cast<uint32_t>(c >> 1) & 1u)) break;
+        const int qb = c % nqb;
+        if (!F.wait_bar(qfull(qb), static_cast<uint32_t>(c / nqb) & 1u)) break;
         tc_fence_after();
         const int Npad = (d.n_rows + 15) & ~15;
         const uint32_t idesc = umma_idesc_f16(kTileTokens, Npad, p.is_bf16 != 0);
         const uint64_t dq0 = smem_desc_sw128(smem_u32(sQ + qb * 2 * qh));
         bool stop = false;
         for (int t = d.t0; t < d.t1; ++t) {
-          const int wg = (t - d.t0) & 1;
+          const int wg = (t - d.t0) % nwg;
           const int kk = kw[wg]++;
-          const int b = wg + 2 * (kk % half);
-          const uint32_t use = static_cast<uint32_t>(kk / half) & 1u;
+          const int b = wg + nwg * (kk % bpw);
+          const uint32_t use = static_cast<uint32_t>(kk / bpw) & 1u;
           if (!F.wait_bar(tempty(b), use ^ 1u)) {
             stop = true;
             break;
@@ -913,6 +917,7 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
   } else if (warp == kStageWarp) {
     // ------------------------------------------------------------ Q rows
     const int G = p.group_size;
+    const uint64_t qpol = l2_policy_evict_last();  // the window rows are read once per chunk
     for (int c = 0;; ++c) {
       const int ds = c % kDescs;
       const bool got = F.wait_bar(dfull(ds), static_cast<uint32_t>(c / kDescs) & 1u);
@@ -921,12 +926,12 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
       __syncwarp();
       if (lane == 0) mbar_arrive(dempty(ds));
       if (d.end) break;
-      const int qb = c & 1;
-      const bool ok = F.wait_bar(qempty(qb), (static_cast<uint32_t>(c >> 1) & 1u) ^ 1u);
+      const int qb = c % nqb;
+      const bool ok = F.wait_bar(qempty(qb), (static_cast<uint32_t>(c / nqb) & 1u) ^ 1u);
       if (!__all_sync(0xffffffffu, ok)) break;
       const int N = d.n_rows;
       const int Npad = (N + 15) & ~15;
-      const uint32_t bits = p.srh_bits[d.list];
+      const uint32_t bits = p.srh_bits[F.list(d.s, d.g)];
       uint8_t* qbuf = sQ + qb * 2 * qh;
       const long long sbase = static_cast<long long>(d.s) * p.q_bs;
       for (int idx = lane; idx < Npad * 16; idx += 32) {
@@ -937,8 +942,10 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
           const int hi = r / W;
           const int w = r - hi * W;
           const int head = d.g * G + nth_bit(bits, hi);
-          cp_async16(smem_u32(dst), p.q + sbase + static_cast<long long>(head) * p.q_hs +
-                                        static_cast<long long>(w) * p.q_ws + ch * 8);
+          cp_async16_hint(smem_u32(dst),
+                          p.q + sbase + static_cast<long long>(head) * p.q_hs +
+                              static_cast<long long>(w) * p.q_ws + ch * 8,
+                          qpol);
         } else {
           *reinterpret_cast<uint4*>(dst) = make_uint4(0u, 0u, 0u, 0u);
         }
@@ -954,20 +961,34 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
     const int wg = ew >> 2;
     const int qd = warp & 3;  // TMEM lane quarter of this warp
     const int tw = (ew & 3) * 32 + lane;
-    float* ref = sRef + ew * kMaxQRows;
-    float* acc_s = sAcc + ew * kMaxQRows;
+    const int te = ew * 32 + lane;  // thread among all epilogue threads
+    const int nwg = p.nwg;
+    const bool takes = wg < nwg;  // this warpgroup takes tiles
+    float* ref = sRef + (takes ? ew : 0) * rstride;
+    float* acc_s = sAcc + (takes ? ew : 0) * rstride;
     const float c = p.c;
-    const uint64_t keep = l2_policy_evict_last();
-    const int half = p.nbuf >> 1;
+    const int bpw = p.nbuf / nwg;
+    const int h = (p.pool_width - 1) >> 1;
+    const float fP = static_cast<float>(p.pool_width);
+    const int G = p.group_size;
     int kc = 0;       // tiles this warpgroup has taken
     int nsync = 0;    // warpgroup syncs so far (mbarrier phase)
+    int nsync8 = 0;   // all-epilogue syncs so far
+    int n2 = 0;       // pass-2 chunks so far (raw buffer parity)
     bool stop = false;
-    // bounded warpgroup barrier: a warp that stopped cannot hang the others
+    // bounded barriers (a warp that stopped cannot hang the others)
     auto wg_sync = [&]() -> bool {
       __syncwarp();
       if (lane == 0) mbar_arrive(wgbar(wg));
       const bool ok = F.wait_bar(wgbar(wg), static_cast<uint32_t>(nsync) & 1u);
       ++nsync;
+      return __all_sync(0xffffffffu, ok);
+    };
+    auto epi_sync = [&]() -> bool {
+      __syncwarp();
+      if (lane == 0) mbar_arrive(epibar);
+      const bool ok = F.wait_bar(epibar, static_cast<uint32_t>(nsync8) & 1u);
+      ++nsync8;
       return __all_sync(0xffffffffu, ok);
     };
     for (int ci = 0; !stop; ++ci) {
@@ -981,164 +1002,214 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
       const int s = d.s;
       const int g = d.g;
       const int N = d.n_rows;
-      const int Nr = expo_stride(N);
       const int L = F.len(s);
       const int n = L - W;
       const int u = s * Hkv + g;
-      uint16_t* expo_u = F.expo_slot(u);
-      float* refs_u = F.refs_slot(u);
-      for (int q = lane; q < N; q += 32) {
-        ref[q] = kNegInf;
-        acc_s[q] = 0.f;
-      }
-      __syncwarp();
-      const int ngrp = (Nr + 31) >> 5;
-      for (int tile = d.t0 + wg; tile < d.t1; tile += 2) {
-        const int kk = kc++;
-        const int b = wg + 2 * (kk % half);
-        const uint32_t use = static_cast<uint32_t>(kk / half) & 1u;
-        const bool ok = F.wait_bar(tfull(b), use);
-        if (!__all_sync(0xffffffffu, ok)) {
-          stop = true;
-          break;
+      const long long soff = static_cast<long long>(g) * p.p_total + p.cu_prefix[s];
+      if (d.pass == 1) {
+        // ---------------------------------------- pass 1: softmax statistics
+        // Per query row q the warp keeps a reference R_q and sums
+        // 2^(z c - R_q) over its keys, reduced across the lanes every tile.
+        if (!takes) continue;  // warpgroups beyond nwg take no first-pass work
+        for (int q = lane; q < N; q += 32) {
+          ref[q] = kNegInf;
+          acc_s[q] = 0.f;
         }
-        tc_fence_after();
-        const int tok = tile * kTileTokens + qd * 32 + lane;  // position in the sequence
-        const uint32_t taddr = tbase + (static_cast<uint32_t>(qd * 32) << 16) +
-                               static_cast<uint32_t>(b * p.tstride);
-        const bool edge = (tile + 1) * kTileTokens > n;  // causal mask or sequence end
-        const int vis = n - tok;  // query row q sees this key iff tok < L and wpos(q) >= -vis
-        const bool key = tok < L;
-        const bool store = tok < n;  // the table holds prefix keys only
-        uint16_t* erow = expo_u + static_cast<long long>(tok) * Nr;
-        for (int grp = 0; grp < ngrp; ++grp) {
-          const int c0 = 32 * grp;
-          const int ncols = min(32, Nr - c0);  // 8, 16 or 32
-          if (c0 >= N) {
-            if (store) {
-              if (ncols == 32) {
-                const uint32_t zz[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
-                st_global_v8_hint(erow + c0, zz, keep);
-                st_global_v8_hint(erow + c0 + 16, zz, keep);
-              } else {
-                for (int v = 0; v < ncols; v += 8) st_global_v4_hint(erow + c0 + v, 0u, 0u, 0u, 0u, keep);
-              }
-            }
-            continue;
+        __syncwarp();
+        bool first = true;  // no tile of this chunk accumulated yet
+        for (int tile = d.t0 + wg; tile < d.t1; tile += nwg) {
+          const int kk = kc++;
+          const int b = wg + nwg * (kk % bpw);
+          const uint32_t use = static_cast<uint32_t>(kk / bpw) & 1u;
+          const bool ok = F.wait_bar(tfull(b), use);
+          if (!__all_sync(0xffffffffu, ok)) {
+            stop = true;
+            break;
           }
-          uint32_t r[32];
-          tmem_load32_async(taddr + c0, r);
-          tmem_wait_ld(r);
-          const int lim = min(32, N - c0);
-          const bool masked = edge || lim < 32;
-          float* rf = ref + c0;
-          float t[32];
-          float tmax = kNegInf;
-          if (masked) {
-#pragma unroll
-            for (int j = 0; j < 32; j += 4) {
-              const int4 wq = *reinterpret_cast<const int4*>(sWpos + c0 + j);
-              const float4 rq = *reinterpret_cast<const float4*>(rf + j);
-              const int wv[4] = {wq.x, wq.y, wq.z, wq.w};
-              const float rv[4] = {rq.x, rq.y, rq.z, rq.w};
-#pragma unroll
-              for (int k = 0; k < 4; ++k) {
-                const bool okk = (j + k) < lim && (!edge || (key && wv[k] >= -vis));
-                t[j + k] = okk ? fmaf(__uint_as_float(r[j + k]), c, -rv[k]) : kNegInf;
-                tmax = fmaxf(tmax, t[j + k]);
-              }
-            }
-          } else {
-#pragma unroll
-            for (int j = 0; j < 32; j += 4) {
-              const float4 rq = *reinterpret_cast<const float4*>(rf + j);
-              t[j + 0] = fmaf(__uint_as_float(r[j + 0]), c, -rq.x);
-              t[j + 1] = fmaf(__uint_as_float(r[j + 1]), c, -rq.y);
-              t[j + 2] = fmaf(__uint_as_float(r[j + 2]), c, -rq.z);
-              t[j + 3] = fmaf(__uint_as_float(r[j + 3]), c, -rq.w);
-              tmax = fmaxf(fmaxf(tmax, fmaxf(t[j], t[j + 1])), fmaxf(t[j + 2], t[j + 3]));
-            }
-          }
-          if (__any_sync(0xffffffffu, tmax > kRaise)) {
-            // raise each query's R to kShift below its largest scaled logit in
-            // this warp's 32 keys (always on the warp's first tile of a chunk)
-            uint32_t valid = 0u;
-#pragma unroll
-            for (int j = 0; j < 32; ++j) valid |= (t[j] != kNegInf ? 1u : 0u) << j;
-            float v[32];
+          tc_fence_after();
+          const int tok = tile * kTileTokens + qd * 32 + lane;
+          const uint32_t taddr = tbase + (static_cast<uint32_t>(qd * 32) << 16) +
+                                 static_cast<uint32_t>(b * p.tstride);
+          const bool edge = (tile + 1) * kTileTokens > n;
+          const int vis = n - tok;
+          const bool key = tok < L;
+          for (int c0 = 0; c0 < N; c0 += 32) {
+            uint32_t r[32];  // the logits
             tmem_load32_async(taddr + c0, r);
             tmem_wait_ld(r);
+            const int lim = min(32, N - c0);
+            const bool masked = edge || lim < 32;
+            float* rf = ref + c0;
+            float e[32];  // 2^(z c - R)
+            if (first && !masked) {
+              // the warp's first tile of the chunk: lane 0's scaled logit is
+              // the reference of each query row (any reference within 2^kRaise
+              // of the largest keeps the fp32 sums exact enough)
 #pragma unroll
-            for (int j = 0; j < 32; ++j)
-              v[j] = ((valid >> j) & 1u) ? __uint_as_float(r[j]) * c : kNegInf;
-            const float m = warp_transpose_max32(v, lane);  // column c0 + lane
-            const float old = rf[lane];
-            const float nw = fmaxf(old, m - kShift);
-            acc_s[c0 + lane] *= (nw == old) ? 1.f : ((old == kNegInf) ? 0.f : ex2_approx(old - nw));
-            __syncwarp();
-            rf[lane] = nw;
-            __syncwarp();
-            tmem_load32_async(taddr + c0, r);
-            tmem_wait_ld(r);
+              for (int j = 0; j < 32; ++j) {
+                const float v = __uint_as_float(r[j]) * c;
+                const float rj = __shfl_sync(0xffffffffu, v, 0);
+                e[j] = ex2_approx(v - rj);
+                if (lane == 0) rf[j] = rj;
+              }
+              __syncwarp();
+            } else if (masked) {
 #pragma unroll
-            for (int j = 0; j < 32; j += 4) {
-              const float4 rq = *reinterpret_cast<const float4*>(rf + j);
-              const float rv[4] = {rq.x, rq.y, rq.z, rq.w};
+              for (int j = 0; j < 32; j += 4) {
+                const int4 wq = *reinterpret_cast<const int4*>(sWpos + c0 + j);
+                const float4 rq = *reinterpret_cast<const float4*>(rf + j);
+                const int wv[4] = {wq.x, wq.y, wq.z, wq.w};
+                const float rv[4] = {rq.x, rq.y, rq.z, rq.w};
 #pragma unroll
-              for (int k = 0; k < 4; ++k)
-                t[j + k] = ((valid >> (j + k)) & 1u) ? fmaf(__uint_as_float(r[j + k]), c, -rv[k])
-                                                      : kNegInf;
-            }
-          }
-          float e[32];
-#pragma unroll
-          for (int j = 0; j < 32; ++j) e[j] = ex2_approx(t[j]);
-          if (store) {
-#pragma unroll
-            for (int v = 0; v < 2; ++v) {
-              if (16 * v < ncols) {
-                uint32_t pk[8];
-#pragma unroll
-                for (int k = 0; k < 8; ++k) pk[k] = pack_half2(e[16 * v + 2 * k], e[16 * v + 2 * k + 1]);
-                if (ncols >= 16) {
-                  st_global_v8_hint(erow + c0 + 16 * v, pk, keep);
-                } else {  // ncols == 8
-                  st_global_v4_hint(erow + c0, pk[0], pk[1], pk[2], pk[3], keep);
+                for (int k = 0; k < 4; ++k) {
+                  const bool okk = (j + k) < lim && (!edge || (key && wv[k] >= -vis));
+                  e[j + k] = okk ? ex2_approx(fmaf(__uint_as_float(r[j + k]), c, -rv[k])) : 0.f;
                 }
               }
+            } else {
+#pragma unroll
+              for (int j = 0; j < 32; j += 4) {
+                const float4 rq = *reinterpret_cast<const float4*>(rf + j);
+                e[j + 0] = ex2_approx(fmaf(__uint_as_float(r[j + 0]), c, -rq.x));
+                e[j + 1] = ex2_approx(fmaf(__uint_as_float(r[j + 1]), c, -rq.y));
+                e[j + 2] = ex2_approx(fmaf(__uint_as_float(r[j + 2]), c, -rq.z));
+                e[j + 3] = ex2_approx(fmaf(__uint_as_float(r[j + 3]), c, -rq.w));
+              }
             }
+            float colsum = warp_transpose_sum32(e, lane);  // column c0 + lane
+            // an exponent above 2^kRaise shows in its column's sum (inf/NaN
+            // when above 2^128 or with the references still -inf)
+            if (__any_sync(0xffffffffu, !(colsum <= 18446744073709551616.0f)))
+              colsum = p1_raise_group(taddr + c0, rf, acc_s + c0, sWpos + c0, lim, edge, key, vis,
+                                      c, lane);
+            acc_s[c0 + lane] += colsum;
+            __syncwarp();
           }
-          const float colsum = warp_transpose_sum32(e, lane);
-          acc_s[c0 + lane] += colsum;
+          first = false;
+          tc_fence_before();
           __syncwarp();
+          if (lane == 0) mbar_arrive(tempty(b));
         }
-        // the references this tile quarter's exponents are relative to
-        float* rt = refs_u + (static_cast<long long>(tile) * kQuarters + qd) * Nr;
-        for (int q = lane; q < N; q += 32) rt[q] = ref[q];
-        tc_fence_before();
+        if (stop) break;
+        // the warpgroup's (M, S) pairs for this chunk, then its ticket
+        if (!wg_sync()) break;
+        float2* part = p.partials +
+                       (static_cast<long long>(d.chunk) * kFusedPartsPerChunk + wg) * p.part_stride;
+        for (int q = tw; q < N; q += 128) {
+          float m = kNegInf;
+          for (int w = 0; w < 4; ++w) m = fmaxf(m, sRef[(wg * 4 + w) * rstride + q]);
+          float z = 0.f;
+          for (int w = 0; w < 4; ++w) {
+            const float rw = sRef[(wg * 4 + w) * rstride + q];
+            if (rw != kNegInf) z += sAcc[(wg * 4 + w) * rstride + q] * ex2_approx(rw - m);
+          }
+          part[q] = make_float2(m, z);
+        }
+        __threadfence();
+        if (!wg_sync()) break;
+        if (tw == 0) atomicAdd(F.ticket(u), 1);
+      } else {
+        // ---------------------------------------- pass 2: raw scores
+        // log2 D_q of every query row into this warp's row of sRef
+        if (p.given_lse) {
+          const uint32_t bits = p.srh_bits[F.list(s, g)];
+          for (int q = lane; q < N; q += 32) {
+            const int hi = q / W;
+            const int w = q - hi * W;
+            const int head = g * G + nth_bit(bits, hi);
+            ref[q] = p.lse[static_cast<long long>(s) * p.lse_bs +
+                           static_cast<long long>(head) * p.lse_hs + w] *
+                     1.4426950408889634f;
+          }
+        } else {
+          bool okb = true;
+          if (lane == 0) okb = F.wait_counter(F.bias_state(u), 2);
+          if (!__shfl_sync(0xffffffffu, okb ? 1 : 0, 0)) {
+            stop = true;
+            break;
+          }
+          const float* bias = p.bias + static_cast<long long>(u) * p.part_stride;
+          for (int q = lane; q < N; q += 32) ref[q] = __ldcg(bias + q);
+        }
         __syncwarp();
-        if (lane == 0) mbar_arrive(tempty(b));
-      }
-      if (stop) break;
-      // the warpgroup's (M, S) pairs for this chunk, then its ticket
-      if (!wg_sync()) break;
-      float2* part = p.partials + (static_cast<long long>(d.chunk) * 2 + wg) * p.part_stride;
-      for (int q = tw; q < N; q += 128) {
-        float m = kNegInf;
-        for (int w = 0; w < 4; ++w) m = fmaxf(m, sRef[(wg * 4 + w) * kMaxQRows + q]);
-        float z = 0.f;
-        for (int w = 0; w < 4; ++w) {
-          const float rw = sRef[(wg * 4 + w) * kMaxQRows + q];
-          if (rw != kNegInf) z += sAcc[(wg * 4 + w) * kMaxQRows + q] * ex2_approx(rw - m);
+        float* cbuf = sChunk + (n2 & 1) * kChunkKeys;
+        ++n2;
+        const int a = d.t0 * kTileTokens;  // first key of the chunk
+        for (int tile = d.t0 + wg; takes && tile < d.t1; tile += nwg) {
+          const int kk = kc++;
+          const int b = wg + nwg * (kk % bpw);
+          const uint32_t use = static_cast<uint32_t>(kk / bpw) & 1u;
+          const bool ok = F.wait_bar(tfull(b), use);
+          if (!__all_sync(0xffffffffu, ok)) {
+            stop = true;
+            break;
+          }
+          tc_fence_after();
+          const int tok = tile * kTileTokens + qd * 32 + lane;
+          const uint32_t taddr = tbase + (static_cast<uint32_t>(qd * 32) << 16) +
+                                 static_cast<uint32_t>(b * p.tstride);
+          const bool edge = (tile + 1) * kTileTokens > n;
+          const int vis = n - tok;
+          const bool key = tok < L;
+          float acc[4] = {0.f, 0.f, 0.f, 0.f};
+          // add 2^(z c - log2 D_q) of 32 columns starting at c0 (lim valid)
+          auto add_group = [&](const uint32_t (&r)[32], int c0, int lim) {
+            if (edge || lim < 32) {
+#pragma unroll
+              for (int j = 0; j < 32; j += 4) {
+                const int4 wq = *reinterpret_cast<const int4*>(sWpos + c0 + j);
+                const float4 lq = *reinterpret_cast<const float4*>(ref + c0 + j);
+                const int wv[4] = {wq.x, wq.y, wq.z, wq.w};
+                const float lv[4] = {lq.x, lq.y, lq.z, lq.w};
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                  const bool okk = (j + k) < lim && (!edge || (key && wv[k] >= -vis));
+                  acc[k] += okk ? ex2_approx(fmaf(__uint_as_float(r[j + k]), c, -lv[k])) : 0.f;
+                }
+              }
+            } else {
+#pragma unroll
+              for (int j = 0; j < 32; j += 4) {
+                const float4 lq = *reinterpret_cast<const float4*>(ref + c0 + j);
+                acc[0] += ex2_approx(fmaf(__uint_as_float(r[j + 0]), c, -lq.x));
+                acc[1] += ex2_approx(fmaf(__uint_as_float(r[j + 1]), c, -lq.y));
+                acc[2] += ex2_approx(fmaf(__uint_as_float(r[j + 2]), c, -lq.z));
+                acc[3] += ex2_approx(fmaf(__uint_as_float(r[j + 3]), c, -lq.w));
+              }
+            }
+          };
+          for (int c0 = 0; c0 < N; c0 += 32) {
+            uint32_t r0[32];
+            tmem_load32_async(taddr + c0, r0);
+            tmem_wait_ld(r0);
+            add_group(r0, c0, min(32, N - c0));
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(tempty(b));
+          if (tok < n) {
+            const float rv = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+            p.raw[soff + tok] = rv;
+            cbuf[tok - a] = rv;
+          }
         }
-        part[q] = make_float2(m, z);
+        if (stop) break;
+        // pooled scores of the chunk's interior [a + h, b - h) from the raw
+        // scores of both warpgroups; the select pools the h keys at each edge
+        if (!epi_sync()) break;
+        const int bnd = min(d.t1 * kTileTokens, n);
+        for (int j = a + h + te; j < bnd - h; j += 32 * kEpiWarps) {
+          float accp = 0.f;
+          for (int t = 0; t <= 2 * h; ++t) accp += cbuf[j - h + t - a];
+          p.pooled[soff + j] = accp / fP;
+        }
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) atomicAdd(F.p2done(u), 1);
       }
-      __threadfence();
-      if (!wg_sync()) break;
-      if (tw == 0) atomicAdd(F.ticket(u), 1);
     }
-  } else if (warp >= kCWarp0) {
-    // ------------------------------------------------------------ combine / select
+  } else if (warp >= kCWarp0 && warp < kCWarp0 + kCThreads / 32) {
+    // ------------------------------------------------------------ merge / select
     const int ct = threadIdx.x - kCWarp0 * 32;
     for (;;) {
       if (ct == 0) claim_task(F, s_task);
@@ -1147,8 +1218,8 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
       const int idx = s_task[1];
       cbar();
       if (type == kTaskEnd) break;
-      if (type == kTaskCombine) {
-        if (!combine_piece(F, idx, creg, ct)) break;
+      if (type == kTaskMerge) {
+        merge_unit(F, idx, creg, ct);
       } else {
         select_unit(F, idx, creg, ct);
       }
@@ -1177,9 +1248,10 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
 
 }  // namespace
 
-size_t fused_smem_bytes(int q_half_bytes, int stages) {
-  return 1024 + static_cast<size_t>(stages) * kTileBytes + 4 * static_cast<size_t>(q_half_bytes) +
-         kFixedBytes + kFusedCRegion;
+size_t fused_smem_bytes(int q_half_bytes, int q_bufs, int stages, int row_stride, int nwg) {
+  return 1024 + static_cast<size_t>(stages) * kTileBytes +
+         2 * static_cast<size_t>(q_bufs) * q_half_bytes +
+         2 * static_cast<size_t>(4 * nwg) * row_stride * 4 + kFixedBytes + kFusedCRegion;
 }
 
 cudaError_t fused_set_smem_limit(size_t bytes) {
