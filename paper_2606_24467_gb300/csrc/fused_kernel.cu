@@ -73,6 +73,7 @@ constexpr int kEpiWarps = 8;
 constexpr int kCWarp0 = 12;   // warps 12..19
 constexpr int kCThreads = 256;
 constexpr int kDescs = 4;     // chunk descriptors in flight (claimed ahead)
+constexpr int kNwg = 2;       // epilogue warpgroups that take tiles (tile t of a chunk: t % 2)
 constexpr int kBarC = 3;      // named barrier of the worker warps
 constexpr float kShift = 7.0f;
 constexpr float kRaise = 64.0f;  // fp32 sums: exponents stay below 2^64 before R is raised
@@ -241,7 +242,7 @@ __device__ __noinline__ void merge_unit(const Fused& F, int u, uint8_t* creg, in
   float* s_mm = reinterpret_cast<float*>(creg);  // [256]
   float* s_mz = s_mm + kMaxQRows;                 // [256]
   if (ncu > 0 && N > 0) {
-    const int nwg = p.nwg;
+    constexpr int nwg = kNwg;
     const int nparts = nwg * ncu;  // the unit's chunks are consecutive
     const float2* parts = p.partials + static_cast<long long>(p.chunk_off[s] + g * ncu) *
                                            kFusedPartsPerChunk * p.part_stride;
@@ -722,7 +723,7 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
   uint8_t* sK = base;
   const int nqb = p.q_bufs;
   uint8_t* sQ = base + nst * kTileBytes;  // nqb buffers of two 64-column halves
-  const int nrow = 4 * p.nwg;  // epilogue warps that take tiles
+  const int nrow = 4 * kNwg;  // epilogue warps that take tiles
   float* sRef = reinterpret_cast<float*>(sQ + 2 * nqb * qh);  // [nrow][rstride]
   float* sAcc = sRef + nrow * rstride;                        // [nrow][rstride]
   int* sWpos = reinterpret_cast<int*>(sAcc + nrow * rstride);
@@ -824,6 +825,8 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
       const uint64_t pol1 = l2_policy_evict_last();
       const uint64_t pol2 = l2_policy_evict_first();
       int gt = 0;  // K tiles issued
+      int st = 0;  // their ring stage and its phase
+      uint32_t sph = 0;
       for (int c = 0;; ++c) {
         const int ds = c % kDescs;
         if (!F.wait_bar(dfull(ds), static_cast<uint32_t>(c / kDescs) & 1u)) break;
@@ -834,8 +837,7 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
         const int row0 = p.cu_seqlens[d.s];
         bool stop = false;
         for (int t = d.t0; t < d.t1; ++t) {
-          const int st = gt % nst;
-          if (!F.wait_bar(empty(st), (static_cast<uint32_t>(gt / nst) & 1u) ^ 1u)) {
+          if (!F.wait_bar(empty(st), sph ^ 1u)) {
             stop = true;
             break;
           }
@@ -845,6 +847,10 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
           tma_load_3d(dst, &p.tmap_k, full(st), 0, d.g, row, pol);
           tma_load_3d(dst + kHalfTileBytes, &p.tmap_k, full(st), 64, d.g, row, pol);
           ++gt;
+          if (++st == nst) {
+            st = 0;
+            sph ^= 1u;
+          }
         }
         if (stop) break;
       }
@@ -859,10 +865,13 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
     // ------------------------------------------------------------ UMMA issue
     if (lane == 0) {
       const uint64_t dk0 = smem_desc_sw128(smem_u32(sK));
-      const int nwg = p.nwg;
-      const int bpw = p.nbuf / nwg;  // TMEM buffers per warpgroup
-      int gt = 0;
-      int kw[4] = {0, 0, 0, 0};
+      const int bpw = p.nbuf / kNwg;  // TMEM buffers per warpgroup (a power of two)
+      const int lbpw = __ffs(bpw) - 1;
+      int st = 0;  // ring stage of the next K tile and its phase
+      uint32_t sph = 0;
+      int qb = 0;  // Q buffer of the next chunk and its phase
+      uint32_t qph = 0;
+      int kw0 = 0, kw1 = 0;  // tiles given to each warpgroup
       int last_b = -1;
       uint32_t last_use = 0;
       for (int c = 0;; ++c) {
@@ -871,44 +880,50 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
         const ChunkDesc d = descs[ds];
         mbar_arrive(dempty(ds));
         if (d.end) break;
-        const int qb = c % nqb;
-        if (!F.wait_bar(qfull(qb), static_cast<uint32_t>(c / nqb) & 1u)) break;
+        if (!F.wait_bar(qfull(qb), qph)) break;
         tc_fence_after();
         const int Npad = (d.n_rows + 15) & ~15;
         const uint32_t idesc = umma_idesc_f16(kTileTokens, Npad, p.is_bf16 != 0);
         const uint64_t dq0 = smem_desc_sw128(smem_u32(sQ + qb * 2 * qh));
         bool stop = false;
         for (int t = d.t0; t < d.t1; ++t) {
-          const int wg = (t - d.t0) % nwg;
-          const int kk = kw[wg]++;
-          const int b = wg + nwg * (kk % bpw);
-          const uint32_t use = static_cast<uint32_t>(kk / bpw) & 1u;
+          const int wg = (t - d.t0) & 1;
+          const int kk = wg ? kw1++ : kw0++;
+          const int b = wg + kNwg * (kk & (bpw - 1));
+          const uint32_t use = static_cast<uint32_t>(kk >> lbpw) & 1u;
           if (!F.wait_bar(tempty(b), use ^ 1u)) {
             stop = true;
             break;
           }
           tc_fence_after();
-          const int st = gt % nst;
-          if (!F.wait_bar(full(st), static_cast<uint32_t>(gt / nst) & 1u)) {
+          if (!F.wait_bar(full(st), sph)) {
             stop = true;
             break;
           }
           tc_fence_after();
           const uint32_t dt = tbase + static_cast<uint32_t>(b * p.tstride);
+          const uint64_t dk = dk0 + static_cast<uint64_t>((st * kTileBytes) >> 4);
 #pragma unroll
           for (int k8 = 0; k8 < kHeadDim / 16; ++k8) {
-            const uint32_t koff = st * kTileBytes + (k8 >> 2) * kHalfTileBytes + (k8 & 3) * 32;
+            const uint32_t koff = (k8 >> 2) * kHalfTileBytes + (k8 & 3) * 32;
             const uint32_t qoff = (k8 >> 2) * qh + (k8 & 3) * 32;
-            umma_f16(dt, dk0 + (koff >> 4), dq0 + (qoff >> 4), idesc, k8 > 0 ? 1u : 0u);
+            umma_f16(dt, dk + (koff >> 4), dq0 + (qoff >> 4), idesc, k8 > 0 ? 1u : 0u);
           }
           umma_commit(empty(st));
           umma_commit(tfull(b));
           last_b = b;
           last_use = use;
-          ++gt;
+          if (++st == nst) {
+            st = 0;
+            sph ^= 1u;
+          }
         }
         if (stop) break;
         umma_commit(qempty(qb));
+        if (++qb == nqb) {
+          qb = 0;
+          qph ^= 1u;
+        }
       }
       if (*reinterpret_cast<volatile int*>(abort_cta) && last_b >= 0)
         wait_plain(tfull(last_b), last_use, 100000000ull);  // MMAs done before TMEM is freed
@@ -918,6 +933,8 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
     // ------------------------------------------------------------ Q rows
     const int G = p.group_size;
     const uint64_t qpol = l2_policy_evict_last();  // the window rows are read once per chunk
+    int qb = 0;  // Q buffer of the next chunk and its phase
+    uint32_t qph = 0;
     for (int c = 0;; ++c) {
       const int ds = c % kDescs;
       const bool got = F.wait_bar(dfull(ds), static_cast<uint32_t>(c / kDescs) & 1u);
@@ -926,8 +943,7 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
       __syncwarp();
       if (lane == 0) mbar_arrive(dempty(ds));
       if (d.end) break;
-      const int qb = c % nqb;
-      const bool ok = F.wait_bar(qempty(qb), (static_cast<uint32_t>(c / nqb) & 1u) ^ 1u);
+      const bool ok = F.wait_bar(qempty(qb), qph ^ 1u);
       if (!__all_sync(0xffffffffu, ok)) break;
       const int N = d.n_rows;
       const int Npad = (N + 15) & ~15;
@@ -954,6 +970,10 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(qfull(qb));
+      if (++qb == nqb) {
+        qb = 0;
+        qph ^= 1u;
+      }
     }
   } else if (warp >= kEpiWarp0 && warp < kEpiWarp0 + kEpiWarps) {
     // ------------------------------------------------------------ epilogue
@@ -962,12 +982,13 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
     const int qd = warp & 3;  // TMEM lane quarter of this warp
     const int tw = (ew & 3) * 32 + lane;
     const int te = ew * 32 + lane;  // thread among all epilogue threads
-    const int nwg = p.nwg;
+    constexpr int nwg = kNwg;
     const bool takes = wg < nwg;  // this warpgroup takes tiles
     float* ref = sRef + (takes ? ew : 0) * rstride;
     float* acc_s = sAcc + (takes ? ew : 0) * rstride;
     const float c = p.c;
-    const int bpw = p.nbuf / nwg;
+    const int bpw = p.nbuf / nwg;  // a power of two
+    const int lbpw = __ffs(bpw) - 1;
     const int h = (p.pool_width - 1) >> 1;
     const float fP = static_cast<float>(p.pool_width);
     const int G = p.group_size;
@@ -1019,8 +1040,8 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
         bool first = true;  // no tile of this chunk accumulated yet
         for (int tile = d.t0 + wg; tile < d.t1; tile += nwg) {
           const int kk = kc++;
-          const int b = wg + nwg * (kk % bpw);
-          const uint32_t use = static_cast<uint32_t>(kk / bpw) & 1u;
+          const int b = wg + nwg * (kk & (bpw - 1));
+          const uint32_t use = static_cast<uint32_t>(kk >> lbpw) & 1u;
           const bool ok = F.wait_bar(tfull(b), use);
           if (!__all_sync(0xffffffffu, ok)) {
             stop = true;
@@ -1137,8 +1158,8 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
         const int a = d.t0 * kTileTokens;  // first key of the chunk
         for (int tile = d.t0 + wg; takes && tile < d.t1; tile += nwg) {
           const int kk = kc++;
-          const int b = wg + nwg * (kk % bpw);
-          const uint32_t use = static_cast<uint32_t>(kk / bpw) & 1u;
+          const int b = wg + nwg * (kk & (bpw - 1));
+          const uint32_t use = static_cast<uint32_t>(kk >> lbpw) & 1u;
           const bool ok = F.wait_bar(tfull(b), use);
           if (!__all_sync(0xffffffffu, ok)) {
             stop = true;
