@@ -435,6 +435,24 @@ int make_k_map(const Info& I, const ckv_problem* p, const void* k, CUtensorMap* 
   return r == CUDA_SUCCESS ? CKV_OK : CKV_ERR_INVALID_ARG;
 }
 
+// 4-D map over the window queries (d, w, head, sequence); the fused kernel
+// loads one box of W rows x 64 columns per SRH head and column half.
+int make_q_map(const Info& I, const ckv_problem* p, const void* q_win, CUtensorMap* map) {
+  const long long bs = I.B > 1 ? p->q_batch_stride : p->q_head_stride * I.Hq;
+  cuuint64_t dims[4] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(I.W),
+                        static_cast<cuuint64_t>(I.Hq), static_cast<cuuint64_t>(I.B)};
+  cuuint64_t strides[3] = {static_cast<cuuint64_t>(p->q_win_stride) * 2,
+                           static_cast<cuuint64_t>(p->q_head_stride) * 2,
+                           static_cast<cuuint64_t>(bs) * 2};
+  cuuint32_t box[4] = {64u, static_cast<cuuint32_t>(I.W), 1u, 1u};
+  cuuint32_t estr[4] = {1u, 1u, 1u, 1u};
+  CUresult r = g_encode(map, I.bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16,
+                        4, const_cast<void*>(q_win), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? CKV_OK : CKV_ERR_INVALID_ARG;
+}
+
 // Scores every unit: per set, the scoring kernel (one pass over K) and the
 // combine kernel, which leaves pooled scores (and raw scores when `raw` is
 // given) in score layout.
@@ -858,6 +876,13 @@ int run_fused(const ckv_problem* p, const Info& I, const SrhLists& S, const void
   *handled = false;
   if (I.layer || I.G > 32 || I.n_masks * I.Hkv > kFusedMaxLists || I.B > kFusedMaxSeqs)
     return CKV_OK;
+  // query rows by TMA: a head block of W rows keeps the 128-byte swizzle
+  // atoms aligned and leaves no padding row (W a multiple of 16), and every
+  // query stride is a multiple of 16 bytes
+  if (I.W % 16 != 0 || I.W > 256 || p->q_win_stride % 8 != 0 || p->q_head_stride % 8 != 0 ||
+      p->q_win_stride <= 0 || p->q_head_stride <= 0 ||
+      (I.B > 1 && (p->q_batch_stride % 8 != 0 || p->q_batch_stride <= 0)))
+    return CKV_OK;
   int max_rows = 16;
   for (int v_ = 0; v_ < I.n_masks * I.Hkv; ++v_) max_rows = std::max(max_rows, S.rows[v_]);
   const int npad_max = (max_rows + 15) & ~15;
@@ -895,6 +920,7 @@ int run_fused(const ckv_problem* p, const Info& I, const SrhLists& S, const void
   static thread_local FusedParams P;  // large (about 15 KB): kept off the stack
   std::memset(&P, 0, sizeof(P));
   if ((rc = make_k_map(I, p, k, &P.tmap_k)) != CKV_OK) return rc;
+  if ((rc = make_q_map(I, p, q_win, &P.tmap_q)) != CKV_OK) return rc;
   P.q = static_cast<const uint16_t*>(q_win);
   P.q_bs = p->q_batch_stride;
   P.q_hs = p->q_head_stride;

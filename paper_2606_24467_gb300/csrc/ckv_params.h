@@ -163,6 +163,7 @@ constexpr int kFusedCRegion = 40 * 1024;  // shared memory of the merge / select
 
 struct FusedParams {
   CUtensorMap tmap_k;          // 3-D map over K: (d, kv head, token)
+  CUtensorMap tmap_q;          // 4-D map over the window queries: (d, w, head, sequence)
   const uint16_t* q;           // window queries (f16/bf16 bits)
   long long q_bs, q_hs, q_ws;  // window-query strides, elements
   const float* lse;            // given-LSE mode: natural-log LSE per (sequence, head, window row)

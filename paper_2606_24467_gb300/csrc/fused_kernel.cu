@@ -30,18 +30,22 @@
 //   warp 3      claims chunks (a pass-2 chunk once its unit's denominators
 //               are merged, else the next pass-1 chunk) and publishes them,
 //               up to kDescs ahead, in a descriptor ring;
-//   warp 0      streams each chunk's K tiles into a shared-memory ring by TMA;
-//   warp 1      TMEM allocation and UMMA issue (M = 128 keys, N = query rows);
-//   warp 2      copies each chunk's SRH query rows into one of two or three
-//               Q buffers;
+//   warp 0      loads each chunk's SRH query rows (one TMA box of W rows per
+//               head and 64-column half) into one of two or three Q buffers
+//               and streams its K tiles into a shared-memory ring, by TMA;
+//   warps 1, 2  UMMA issue (M = 128 keys, N = query rows), warp 1 for the
+//               tiles of warpgroup 0 and warp 2 for those of warpgroup 1
+//               (a UMMA of this shape holds the tensor core for a fixed 76
+//               cycles whatever N up to 128, so two issuing threads, each
+//               with its own waits, keep it fed); warp 1 also allocates TMEM;
 //   warps 4-11  two epilogue warpgroups; tile t of a chunk belongs to
 //               warpgroup t % nwg (nwg = 2), each with its own TMEM buffers;
 //   warps 12-19 workers: they merge a unit's pass-1 pairs into its
 //               denominators once all its chunks are in, and select and
 //               gather a unit once all its pass-2 chunks are in (one CTA per
 //               unit).
-// A pass-2 chunk is published once its unit's denominators are merged (the
-// epilogue still checks, bounded); workers claim a merge or a selection only
+// A pass-2 chunk is published once its claimer has seen (acquire) its unit's
+// denominators merged; workers claim a merge or a selection only
 // when it is ready.  Every wait therefore depends only on
 // work claimed earlier by a running CTA that never waits on later work, so a
 // call completes whatever the number of CTAs resident at once; every wait
@@ -66,14 +70,15 @@ constexpr int kFWarps = 20;
 constexpr int kFThreads = 32 * kFWarps;
 constexpr int kProdWarp = 0;
 constexpr int kMmaWarp = 1;
-constexpr int kStageWarp = 2;
+constexpr int kMmaWarp2 = 2;  // second UMMA issuer (tiles of warpgroup 1)
 constexpr int kClaimWarp = 3;
 constexpr int kEpiWarp0 = 4;  // warps 4..11: two warpgroups (TMEM lane quarter = warp % 4)
 constexpr int kEpiWarps = 8;
 constexpr int kCWarp0 = 12;   // warps 12..19
 constexpr int kCThreads = 256;
 constexpr int kDescs = 4;     // chunk descriptors in flight (claimed ahead)
-constexpr int kNwg = 2;       // epilogue warpgroups that take tiles (tile t of a chunk: t % 2)
+constexpr int kNwg = 2;
+constexpr int kPub = 6;       // chunks written, not yet published (publish ring)       // epilogue warpgroups that take tiles (tile t of a chunk: t % 2)
 constexpr int kBarC = 3;      // named barrier of the worker warps
 constexpr float kShift = 7.0f;
 constexpr float kRaise = 64.0f;  // fp32 sums: exponents stay below 2^64 before R is raised
@@ -180,9 +185,69 @@ struct Fused {
   }
   // Bounded wait on one of this CTA's mbarriers; a timeout stops the call.
   __device__ bool wait_bar(uint32_t bar, uint32_t parity) const {
+    if (mbar_test_wait(bar, parity)) return true;
     const bool ok = mbar_wait_bounded(bar, parity, abort_cta, p.status);
     if (!ok && !aborted()) atomicExch(p.ctr + kCtrAbort, 1);
     return ok;
+  }
+};
+
+// ---------------------------------------------------------------- publishing
+// The claimer thread publishes the chunks the epilogue has finished, in
+// order: after the epilogue warps' arrivals (CTA-scope release/acquire) one
+// GPU-scope fence covers a batch of finished chunks, then each chunk adds to
+// its unit's counter (pass 1: the ticket the merge waits for; pass 2: the
+// count the selection waits for).  The fence's wait for the writes thus
+// stalls neither the epilogue nor the tile pipeline.
+struct Publisher {
+  const Fused& F;
+  uint32_t full0, empty0;  // the publish ring's barriers
+  int info[kPub];          // chunk i (slot i % kPub): unit * 2 + pass - 1
+  int next, issued;        // first chunk not yet published; chunks issued
+
+  __device__ uint32_t full(int i) const { return full0 + 8u * static_cast<uint32_t>(i % kPub); }
+  __device__ uint32_t empty(int i) const { return empty0 + 8u * static_cast<uint32_t>(i % kPub); }
+  __device__ void pump() {
+    int k = next;
+    while (k < issued && mbar_test_wait(full(k), static_cast<uint32_t>(k / kPub) & 1u)) ++k;
+    if (k == next) return;
+    fence_acq_rel_gpu();
+    for (; next < k; ++next) {
+      const int v = info[next % kPub];
+      if (v & 1) {
+        atomicAdd(F.p2done(v >> 1), kEpiWarps);
+      } else {
+        atomicAdd(F.ticket(v >> 1), kNwg);
+      }
+      mbar_arrive(empty(next));
+    }
+  }
+  // Bounded wait on one of the CTA's mbarriers, publishing meanwhile.
+  __device__ bool wait_bar(uint32_t bar, uint32_t parity) {
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t it = 1;; ++it) {
+      if (mbar_try_wait(bar, parity)) return true;
+      pump();
+      if ((it & 63u) == 0 && !still_waiting(t0)) return false;
+    }
+  }
+  // Bounded wait until at most `left` issued chunks are unpublished.
+  __device__ bool wait_published(int left) {
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t it = 1; issued - next > left; ++it) {
+      pump();
+      __nanosleep(32);
+      if ((it & 63u) == 0 && !still_waiting(t0)) return false;
+    }
+    return true;
+  }
+  __device__ bool still_waiting(uint64_t t0) const {
+    if (F.aborted() || *reinterpret_cast<volatile int*>(F.abort_cta)) return false;
+    if (globaltimer_ns() - t0 > kWaitTimeoutNs) {
+      F.raise_abort();
+      return false;
+    }
+    return true;
   }
 };
 
@@ -195,7 +260,7 @@ struct Fused {
 // epilogue before its denominators.  When pass 1 is exhausted the claimer
 // waits (bounded) for its pending chunk's unit, whose pass-1 chunks are then
 // all claimed.  Returns false when both passes are exhausted (or aborted).
-__device__ bool claim_chunk(const Fused& F, int* pending, int* pass, int* x) {
+__device__ bool claim_chunk(const Fused& F, Publisher& pb, int* pending, int* pass, int* x) {
   const FusedParams& p = F.p;
   for (;;) {
     if (F.aborted() || *reinterpret_cast<volatile int*>(F.abort_cta)) return false;
@@ -224,8 +289,15 @@ __device__ bool claim_chunk(const Fused& F, int* pending, int* pass, int* x) {
       continue;
     }
     if (*pending < 0) return false;  // both passes exhausted
-    // pass 1 is exhausted: every pass-1 chunk of the pending chunk's unit is claimed
-    if (!F.wait_counter(F.bias_state(u), 2)) return false;
+    // pass 1 is exhausted: every pass-1 chunk of the pending chunk's unit is
+    // claimed; wait (bounded) for its merge, publishing meanwhile (the merge
+    // may wait for tickets this CTA holds)
+    const uint64_t t0 = globaltimer_ns();
+    while (ld_acquire(F.bias_state(u)) < 2) {
+      pb.pump();
+      __nanosleep(64);
+      if (!pb.still_waiting(t0)) return false;
+    }
   }
 }
 
@@ -292,7 +364,7 @@ __device__ __noinline__ void merge_unit(const Fused& F, int u, uint8_t* creg, in
       p.bias[static_cast<long long>(u) * p.part_stride + ct] = m + __log2f(z);
     }
   }
-  __threadfence();
+  fence_acq_rel_gpu();
   cbar();
   if (ct == 0) atomicExch(F.bias_state(u), 2);
 }
@@ -643,7 +715,7 @@ __device__ void claim_task(const Fused& F, int* task) {
     const int u = ld_volatile(p.ctr + kCtrSel);
     if (u >= p.n_units) break;  // every unit selected (and therefore merged)
     const int s = u / p.num_kv_heads;
-    if (ld_acquire(F.p2done(u)) >= kEpiWarps * F.chunks_per_unit(s)) {  // every epilogue warp
+    if (ld_acquire(F.p2done(u)) >= kEpiWarps * F.chunks_per_unit(s)) {  // kEpiWarps per pass-2 chunk
       if (atomicCAS(p.ctr + kCtrSel, u, u + 1) == u) {
         task[0] = kTaskSelect;
         task[1] = u;
@@ -748,6 +820,8 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
   auto qempty = [&](int i) { return bar0 + 8u * (43 + i); };    // Q buffer's MMAs done
   auto wgbar = [&](int w) { return bar0 + 8u * (46 + w); };     // epilogue warpgroup sync
   const uint32_t epibar = bar0 + 8u * 50;                       // all epilogue warps
+  auto pubfull = [&](int i) { return bar0 + 8u * (51 + i); };   // chunk's results written
+  auto pubempty = [&](int i) { return bar0 + 8u * (51 + kPub + i); };  // chunk published
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -766,14 +840,18 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
     }
     for (int i = 0; i < kDescs; ++i) {
       mbar_init(dfull(i), 1);
-      mbar_init(dempty(i), 3 + kEpiWarps);  // TMA producer, MMA, stager, epilogue warps
+      mbar_init(dempty(i), 3 + kEpiWarps);  // TMA producer, both MMA warps, epilogue warps
     }
     for (int i = 0; i < 3; ++i) {
       mbar_init(qfull(i), 1);
-      mbar_init(qempty(i), 1);
+      mbar_init(qempty(i), 2);  // one commit from each MMA warp
     }
     for (int i = 0; i < 4; ++i) mbar_init(wgbar(i), 4);
     mbar_init(epibar, kEpiWarps);
+    for (int i = 0; i < kPub; ++i) {
+      mbar_init(pubfull(i), kEpiWarps);
+      mbar_init(pubempty(i), 1);
+    }
     *abort_cta = 0;
     fence_mbar_init();
   }
@@ -790,14 +868,15 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
   if (warp == kClaimWarp) {
     // ------------------------------------------------------------ chunk claims
     if (lane == 0) {
+      Publisher pb{F, pubfull(0), pubempty(0), {}, 0, 0};
       int pending = -1;  // pass-2 chunk claimed, not yet published
       for (int c = 0;; ++c) {
         const int ds = c % kDescs;
-        if (!F.wait_bar(dempty(ds), ((c / kDescs) & 1) ^ 1)) break;
+        if (!pb.wait_bar(dempty(ds), ((c / kDescs) & 1) ^ 1)) break;
         ChunkDesc d;
         d.end = 1;
         int pass = 0, x = 0;
-        if (claim_chunk(F, &pending, &pass, &x)) {
+        if (claim_chunk(F, pb, &pending, &pass, &x)) {
           const int s = find_seq(p.chunk_off, p.batch, x);
           const int ncu = F.chunks_per_unit(s);
           const int local = x - p.chunk_off[s];
@@ -811,11 +890,15 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
           d.t1 = min(F.tiles(s), d.t0 + kChunkTiles);
           d.chunk = x;
           d.n_rows = F.rows(s, g);
+          if (!pb.wait_published(kPub - 1)) break;  // a free slot in the publish ring
+          pb.info[pb.issued % kPub] = (s * Hkv + g) * 2 + (pass - 1);
+          ++pb.issued;
         }
         descs[ds] = d;
         mbar_arrive(dfull(ds));
         if (d.end) break;
       }
+      pb.wait_published(0);  // every chunk this CTA processed
     }
     __syncwarp();
   } else if (warp == kProdWarp) {
@@ -824,9 +907,13 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
       // pass 1 keeps K in L2 for pass 2, which reads it for the last time
       const uint64_t pol1 = l2_policy_evict_last();
       const uint64_t pol2 = l2_policy_evict_first();
+      const int G = p.group_size;
       int gt = 0;  // K tiles issued
       int st = 0;  // their ring stage and its phase
       uint32_t sph = 0;
+      int qb = 0;  // Q buffer of the next chunk and its phase
+      uint32_t qph = 0;
+      uint32_t q_issued = 0, q_phase = 0;  // per Q buffer: loads issued, phase of the last
       for (int c = 0;; ++c) {
         const int ds = c % kDescs;
         if (!F.wait_bar(dfull(ds), static_cast<uint32_t>(c / kDescs) & 1u)) break;
@@ -835,6 +922,26 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
         if (d.end) break;
         const uint64_t pol = d.pass == 1 ? pol1 : pol2;
         const int row0 = p.cu_seqlens[d.s];
+        // the chunk's query rows: head block hi of the buffer holds the W
+        // window rows of the group's hi-th SRH head
+        if (!F.wait_bar(qempty(qb), qph ^ 1u)) break;
+        {
+          uint32_t bits = p.srh_bits[F.list(d.s, d.g)];
+          mbar_arrive_expect_tx(qfull(qb), static_cast<uint32_t>(d.n_rows) * (kHeadDim * 2));
+          const uint32_t qdst = smem_u32(sQ + qb * 2 * qh);
+          for (int hi = 0; bits != 0u; ++hi, bits &= bits - 1u) {
+            const int head = d.g * G + (__ffs(bits) - 1);
+            const uint32_t dst = qdst + static_cast<uint32_t>(hi * W * 128);
+            tma_load_4d(dst, &p.tmap_q, qfull(qb), 0, 0, head, d.s, pol1);
+            tma_load_4d(dst + qh, &p.tmap_q, qfull(qb), 64, 0, head, d.s, pol1);
+          }
+          q_issued |= 1u << qb;
+          q_phase = (q_phase & ~(1u << qb)) | (qph << qb);
+          if (++qb == nqb) {
+            qb = 0;
+            qph ^= 1u;
+          }
+        }
         bool stop = false;
         for (int t = d.t0; t < d.t1; ++t) {
           if (!F.wait_bar(empty(st), sph ^ 1u)) {
@@ -858,11 +965,14 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
         // let the copies already issued land before the CTA can exit
         for (int i = max(0, gt - nst); i < gt; ++i)
           wait_plain(full(i % nst), static_cast<uint32_t>(i / nst) & 1u, 100000000ull);
+        for (int b = 0; b < nqb; ++b)
+          if ((q_issued >> b) & 1u) wait_plain(qfull(b), (q_phase >> b) & 1u, 100000000ull);
       }
     }
     __syncwarp();
-  } else if (warp == kMmaWarp) {
+  } else if (warp == kMmaWarp || warp == kMmaWarp2) {
     // ------------------------------------------------------------ UMMA issue
+    const int mw = warp == kMmaWarp ? 0 : 1;  // the warpgroup whose tiles this warp issues
     if (lane == 0) {
       const uint64_t dk0 = smem_desc_sw128(smem_u32(sK));
       const int bpw = p.nbuf / kNwg;  // TMEM buffers per warpgroup (a power of two)
@@ -871,7 +981,7 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
       uint32_t sph = 0;
       int qb = 0;  // Q buffer of the next chunk and its phase
       uint32_t qph = 0;
-      int kw0 = 0, kw1 = 0;  // tiles given to each warpgroup
+      int kw = 0;  // tiles issued for warpgroup mw
       int last_b = -1;
       uint32_t last_use = 0;
       for (int c = 0;; ++c) {
@@ -887,15 +997,20 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
         const uint64_t dq0 = smem_desc_sw128(smem_u32(sQ + qb * 2 * qh));
         bool stop = false;
         for (int t = d.t0; t < d.t1; ++t) {
-          const int wg = (t - d.t0) & 1;
-          const int kk = wg ? kw1++ : kw0++;
-          const int b = wg + kNwg * (kk & (bpw - 1));
+          if (((t - d.t0) & 1) != mw) {  // the other warp's tile: only the ring advances
+            if (++st == nst) {
+              st = 0;
+              sph ^= 1u;
+            }
+            continue;
+          }
+          const int kk = kw++;
+          const int b = mw + kNwg * (kk & (bpw - 1));
           const uint32_t use = static_cast<uint32_t>(kk >> lbpw) & 1u;
           if (!F.wait_bar(tempty(b), use ^ 1u)) {
             stop = true;
             break;
           }
-          tc_fence_after();
           if (!F.wait_bar(full(st), sph)) {
             stop = true;
             break;
@@ -929,52 +1044,6 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
         wait_plain(tfull(last_b), last_use, 100000000ull);  // MMAs done before TMEM is freed
     }
     __syncwarp();
-  } else if (warp == kStageWarp) {
-    // ------------------------------------------------------------ Q rows
-    const int G = p.group_size;
-    const uint64_t qpol = l2_policy_evict_last();  // the window rows are read once per chunk
-    int qb = 0;  // Q buffer of the next chunk and its phase
-    uint32_t qph = 0;
-    for (int c = 0;; ++c) {
-      const int ds = c % kDescs;
-      const bool got = F.wait_bar(dfull(ds), static_cast<uint32_t>(c / kDescs) & 1u);
-      if (!__all_sync(0xffffffffu, got)) break;
-      const ChunkDesc d = descs[ds];
-      __syncwarp();
-      if (lane == 0) mbar_arrive(dempty(ds));
-      if (d.end) break;
-      const bool ok = F.wait_bar(qempty(qb), qph ^ 1u);
-      if (!__all_sync(0xffffffffu, ok)) break;
-      const int N = d.n_rows;
-      const int Npad = (N + 15) & ~15;
-      const uint32_t bits = p.srh_bits[F.list(d.s, d.g)];
-      uint8_t* qbuf = sQ + qb * 2 * qh;
-      const long long sbase = static_cast<long long>(d.s) * p.q_bs;
-      for (int idx = lane; idx < Npad * 16; idx += 32) {
-        const int r = idx >> 4;
-        const int ch = idx & 15;
-        uint8_t* dst = qbuf + (ch >> 3) * qh + r * 128 + (((ch & 7) ^ (r & 7)) << 4);
-        if (r < N) {
-          const int hi = r / W;
-          const int w = r - hi * W;
-          const int head = d.g * G + nth_bit(bits, hi);
-          cp_async16_hint(smem_u32(dst),
-                          p.q + sbase + static_cast<long long>(head) * p.q_hs +
-                              static_cast<long long>(w) * p.q_ws + ch * 8,
-                          qpol);
-        } else {
-          *reinterpret_cast<uint4*>(dst) = make_uint4(0u, 0u, 0u, 0u);
-        }
-      }
-      cp_async_wait_all();
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(qfull(qb));
-      if (++qb == nqb) {
-        qb = 0;
-        qph ^= 1u;
-      }
-    }
   } else if (warp >= kEpiWarp0 && warp < kEpiWarp0 + kEpiWarps) {
     // ------------------------------------------------------------ epilogue
     const int ew = warp - kEpiWarp0;
@@ -998,18 +1067,28 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
     int n2 = 0;       // pass-2 chunks so far (raw buffer parity)
     bool stop = false;
     // bounded barriers (a warp that stopped cannot hang the others)
-    auto wg_sync = [&]() -> bool {
-      __syncwarp();
-      if (lane == 0) mbar_arrive(wgbar(wg));
-      const bool ok = F.wait_bar(wgbar(wg), static_cast<uint32_t>(nsync) & 1u);
-      ++nsync;
-      return __all_sync(0xffffffffu, ok);
-    };
     auto epi_sync = [&]() -> bool {
       __syncwarp();
       if (lane == 0) mbar_arrive(epibar);
       const bool ok = F.wait_bar(epibar, static_cast<uint32_t>(nsync8) & 1u);
       ++nsync8;
+      return __all_sync(0xffffffffu, ok);
+    };
+    // the chunk's results are written: its claimer publishes it (fence, then
+    // the unit's counter) off the epilogue's path
+    auto publish = [&](int ci) -> bool {
+      const int k = ci % kPub;
+      bool ok = true;
+      if (ci >= kPub && lane == 0) ok = F.wait_bar(pubempty(k), static_cast<uint32_t>(ci / kPub - 1) & 1u);
+      __syncwarp();
+      if (lane == 0 && ok) mbar_arrive(pubfull(k));
+      return __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+    };
+    auto wg_sync = [&]() -> bool {
+      __syncwarp();
+      if (lane == 0) mbar_arrive(wgbar(wg));
+      const bool ok = F.wait_bar(wgbar(wg), static_cast<uint32_t>(nsync) & 1u);
+      ++nsync;
       return __all_sync(0xffffffffu, ok);
     };
     for (int ci = 0; !stop; ++ci) {
@@ -1126,9 +1205,8 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
           }
           part[q] = make_float2(m, z);
         }
-        __threadfence();
-        if (!wg_sync()) break;
-        if (tw == 0) atomicAdd(F.ticket(u), 1);
+        if (!wg_sync()) break;  // every row read (the next chunk reuses them)
+        if (!publish(ci)) break;
       } else {
         // ---------------------------------------- pass 2: raw scores
         // log2 D_q of every query row into this warp's row of sRef
@@ -1143,12 +1221,8 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
                      1.4426950408889634f;
           }
         } else {
-          bool okb = true;
-          if (lane == 0) okb = F.wait_counter(F.bias_state(u), 2);
-          if (!__shfl_sync(0xffffffffu, okb ? 1 : 0, 0)) {
-            stop = true;
-            break;
-          }
+          // published only after its claimer saw the unit's denominators
+          // merged (acquire), before the descriptor barrier
           const float* bias = p.bias + static_cast<long long>(u) * p.part_stride;
           for (int q = lane; q < N; q += 32) ref[q] = __ldcg(bias + q);
         }
@@ -1224,9 +1298,7 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
           for (int t = 0; t <= 2 * h; ++t) accp += cbuf[j - h + t - a];
           p.pooled[soff + j] = accp / fP;
         }
-        __threadfence();
-        __syncwarp();
-        if (lane == 0) atomicAdd(F.p2done(u), 1);
+        if (!publish(ci)) break;
       }
     }
   } else if (warp >= kCWarp0 && warp < kCWarp0 + kCThreads / 32) {
