@@ -147,7 +147,7 @@ struct GatherParams {
 // a call in two passes (softmax statistics, then normalised scores with K
 // re-read from L2), pools, selects and gathers, with work claimed from
 // counters in the workspace.
-constexpr int kChunkTiles = 8;          // K tiles per scoring chunk (references restart per chunk)
+constexpr int kChunkTiles = 16;         // K tiles per scoring chunk (references restart per chunk)
 constexpr int kChunkKeys = kChunkTiles * kTileTokens;
 constexpr int kFusedMaxSeqs = kMaxBatch;
 constexpr int kFusedMaxLists = 1024;    // (mask, group) SRH lists of one call

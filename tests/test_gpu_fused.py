@@ -2,10 +2,10 @@
 float64 oracle, through the C ABI (needs a GB300).
 
 Besides parity with the oracle (tolerances as in test_gpu_parity.py), the
-kernel's scores depend only on the unit itself: its exponent references
-restart on a fixed grid of 8 K tiles of every unit and each tile of that grid
-always goes to the same epilogue warpgroup, so a layer compressed alone and
-the same layer inside a larger call give identical bits.
+kernel's scores depend only on the unit itself: its softmax statistics
+restart on a fixed grid of 16-tile chunks of every unit and each tile of that
+grid always goes to the same epilogue warpgroup, so a layer compressed alone
+and the same layer inside a larger call give identical bits.
 """
 import numpy as np
 import pytest
@@ -18,7 +18,7 @@ from oracle import compare
 
 pytestmark = pytest.mark.gpu
 
-EXPO_RTOL = 2.0 ** -11 + 2e-5
+RTOL = 1e-4  # fp32 exponentials of fp32 logits, fp32 merged denominators
 
 
 def _bits(t):
@@ -84,10 +84,8 @@ def _check_block(blk, lay, cfg):
     if "raw" in blk:
         compare.check_layer(res, blk["raw"], blk["pooled"], blk["indices"], lay["cu_seqlens"],
                             cfg.window)
-        compare.check_scores("raw (fp16 table bound)", blk["raw"], res.raw, rtol=EXPO_RTOL,
-                             atol=1e-8)
-        compare.check_scores("pooled (fp16 table bound)", blk["pooled"], res.pooled,
-                             rtol=EXPO_RTOL, atol=1e-8)
+        compare.check_scores("raw", blk["raw"], res.raw, rtol=RTOL, atol=1e-8)
+        compare.check_scores("pooled", blk["pooled"], res.pooled, rtol=RTOL, atol=1e-8)
     else:
         for (s, g), unit in res.units.items():
             L = int(lay["cu_seqlens"][s + 1] - lay["cu_seqlens"][s])
@@ -146,8 +144,9 @@ def test_repeat_call_is_bit_identical(cuda_device):
 
 def test_full_32_layer_llama8b_32k_in_one_call(cuda_device):
     """The benchmark step itself: all 32 layers of the L=32K Llama-3.1-8B
-    workload in one call (256 units; more units than exponent-table slots, so
-    units wait for their slot's previous user).  The first and last layers
+    workload in one call (256 units of 16 chunks each, more units than CTAs,
+    so pass-2 chunks wait for merges of units spread over many CTAs).  The
+    first and last layers
     are checked against the oracle unit by unit."""
     dev = cuda_device
     cfg = wl.get("c2")
