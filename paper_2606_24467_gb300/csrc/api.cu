@@ -937,6 +937,7 @@ int run_fused(const ckv_problem* p, const Info& I, const SrhLists& S, const void
   P.head_stride_v16 = p->kv_head_stride / 8;
   P.indices = indices;
   P.raw = raw_user ? raw_user : reinterpret_cast<float*>(wb + FL.raw);
+  P.raw_scratch = raw_user ? 0 : 1;
   P.pooled = pooled_user ? pooled_user : reinterpret_cast<float*>(wb + FL.pooled);
   P.status = reinterpret_cast<int*>(wb);
   P.ctr = reinterpret_cast<int*>(wb + kFusedCtrOffset);

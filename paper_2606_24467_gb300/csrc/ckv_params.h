@@ -184,7 +184,8 @@ struct FusedParams {
   float c;                     // scale * log2(e)
   int window, pool_width, num_kv_heads, group_size, p_total, o_total, is_bf16;
   int n_units, n_chunks, batch;
-  int do_select;               // 0: scores only (no selection, no gather)
+  int do_select;
+  int raw_scratch;             // raw scores in the workspace: a unit's row may hold its candidates               // 0: scores only (no selection, no gather)
   int given_lse;               // 1: no first pass; denominators from `lse`
   int q_half_bytes;            // bytes of one 64-column half of a Q buffer
   int q_bufs;                  // Q buffers (2 or 3)

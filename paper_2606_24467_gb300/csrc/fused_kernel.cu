@@ -78,6 +78,7 @@ constexpr int kCWarp0 = 12;   // warps 12..19
 constexpr int kCThreads = 256;
 constexpr int kDescs = 4;     // chunk descriptors in flight (claimed ahead)
 constexpr int kNwg = 2;
+constexpr int kSelSamples = 1024;  // samples of a unit's pooled scores for the select threshold
 constexpr int kPub = 6;       // chunks written, not yet published (publish ring)       // epilogue warpgroups that take tiles (tile t of a chunk: t % 2)
 constexpr int kBarC = 3;      // named barrier of the worker warps
 constexpr float kShift = 7.0f;
@@ -102,15 +103,16 @@ struct ChunkDesc {
 
 // Shared memory of the worker warps (a merge or a selection at a time).
 struct SelShared {
-  int samp[256];
   uint32_t key[kFusedCandCap];
   int pos[kFusedCandCap];
   RadixShared rs;
   int wcnt[8], wbase[8];
+  int wcnt_ge[8];  // per-warp counts at the best threshold with at least k keys above
   int flag[4];
   uint32_t lo;
 };
 static_assert(sizeof(SelShared) <= kFusedCRegion, "select scratch");
+static_assert(kSelSamples <= kFusedCandCap, "samples live in the position array");
 static_assert(3 * kMaxQRows * 4 + 16 <= kFusedCRegion, "merge scratch");
 
 constexpr int kWposBytes = kMaxQRows * 4;
@@ -424,20 +426,32 @@ __device__ __noinline__ uint32_t grp_kth_largest(const uint32_t* keys, int count
     const int shf = hb + 1 - width;
     const uint32_t fm = (1u << width) - 1u;
     uint32_t* hh = sh.hist[pc & 3];
+    constexpr int kB = 8;  // keys per thread loaded before they are counted
 #pragma unroll 1
-    for (int i = 0; i < iters; ++i) {
-      const int j = (i << 8) + ct;
-      const uint32_t key = j < count ? key_at(j) : 0u;
-      const bool m = j < count && (key & pmask) == prefix;
-      const uint32_t act = __ballot_sync(0xffffffffu, m);
-      if (!act) continue;
-      const uint32_t bin = (key >> shf) & fm;
-      const int leader = __ffs(act) - 1;
-      const uint32_t lb = __shfl_sync(0xffffffffu, bin, leader);
-      if (__all_sync(0xffffffffu, !m || bin == lb)) {
-        if (lane == leader) atomicAdd(&hh[lb], static_cast<uint32_t>(__popc(act)));
-      } else if (m) {
-        atomicAdd(&hh[bin], 1u);
+    for (int i0 = 0; i0 < iters; i0 += kB) {
+      uint32_t kv[kB];
+#pragma unroll
+      for (int q = 0; q < kB; ++q) {
+        const int j = ((i0 + q) << 8) + ct;
+        kv[q] = j < count ? key_at(j) : 0u;
+      }
+#pragma unroll
+      for (int q = 0; q < kB; ++q) {
+        const int j = ((i0 + q) << 8) + ct;
+        const uint32_t key = kv[q];
+        const bool m = j < count && (key & pmask) == prefix;
+        const uint32_t act = __ballot_sync(0xffffffffu, m);
+        if (!act) continue;
+        const uint32_t bin = (key >> shf) & fm;
+        const int leader = __ffs(act) - 1;
+        const uint32_t lb = __shfl_sync(0xffffffffu, bin, leader);
+        if (__all_sync(0xffffffffu, !m || bin == lb)) {
+          if (lane == leader) atomicAdd(&hh[lb], static_cast<uint32_t>(__popc(act)));
+        } else if (m) {
+          // one add per distinct bin of the warp (no same-address serialisation)
+          const uint32_t same = __match_any_sync(act, bin);
+          if (lane == __ffs(same) - 1) atomicAdd(&hh[bin], static_cast<uint32_t>(__popc(same)));
+        }
       }
     }
     sh.hist[(pc + 2) & 3][ct] = 0u;
@@ -464,10 +478,12 @@ __device__ void emit_selected(int count, uint32_t tau, int need_eq, int32_t* out
   const int cw = ct >> 5;
   const int lane = ct & 31;
   int o = 0, eq_seen = 0;
+  uint32_t next = ct < count ? key_at(ct) : 0u;  // one block of keys loaded ahead
   for (int j0 = 0; j0 < count; j0 += kCThreads) {
     const int j = j0 + ct;
     const bool in = j < count;
-    const uint32_t key = in ? key_at(j) : 0u;
+    const uint32_t key = next;
+    if (j + kCThreads < count) next = key_at(j + kCThreads);
     const bool gt = in && key > tau;
     const bool eq = in && key == tau;
     const uint32_t mgt = __ballot_sync(0xffffffffu, gt);
@@ -603,36 +619,28 @@ __device__ __noinline__ void select_unit(const Fused& F, int u, uint8_t* creg, i
     return;
   }
   const uint32_t* keys = reinterpret_cast<const uint32_t*>(pooled);
-  const int ns = min(256, n);
-  sh.samp[ct] = ct < ns ? static_cast<int>(__ldcg(keys + static_cast<int>(
-                                                  (static_cast<long long>(ct) * n) / ns)))
-                        : -1;
+  // threshold lo: the rs-th largest of ns samples spread over the unit,
+  // chosen so that the keys >= lo are at least k and at most the shared
+  // candidate capacity; the samples sit in the (not yet used) position array
+  uint32_t* samp = reinterpret_cast<uint32_t*>(sh.pos);
+  const int ns = min(kSelSamples, n);
+  for (int i = ct; i < ns; i += kCThreads)
+    samp[i] = __ldcg(keys + static_cast<int>((static_cast<long long>(i) * n) / ns));
   radix_init_grp(sh.rs, ct);
   cbar();
+  int pc = 0, need_eq = 0;
   const float mu = static_cast<float>(k) * static_cast<float>(ns) / static_cast<float>(n);
   int rs = min(ns, static_cast<int>(ceilf(mu + 3.f * sqrtf(mu))) + 2);
-  uint32_t lo = 0;
-  int total = 0;
+  uint32_t lo = 0, lo_ge = 0;
+  int total = 0, tot_ge = -1;
   constexpr int kU = 8;  // loads in flight per lane
   const int seg = ((n + 8 * 32 * kU - 1) / (8 * 32 * kU)) * 32 * kU;  // positions per warp
   const int wlo = min(n, cw * seg);
   const int whi = min(n, wlo + seg);
   bool fast = false;
   for (int attempt = 0; attempt < 2; ++attempt) {
-    {  // the rs-th largest sample
-      const int v = sh.samp[ct];
-      const int4* s4 = reinterpret_cast<const int4*>(sh.samp);
-      int gt = 0, eq = 0;
-#pragma unroll 8
-      for (int j = 0; j < 64; ++j) {
-        const int4 xx = s4[j];
-        gt += (xx.x > v) + (xx.y > v) + (xx.z > v) + (xx.w > v);
-        eq += (xx.x == v) + (xx.y == v) + (xx.z == v) + (xx.w == v);
-      }
-      if (v >= 0 && gt < rs && rs <= gt + eq) sh.lo = static_cast<uint32_t>(v);
-    }
-    cbar();
-    lo = sh.lo;
+    // (same sample set every attempt: the radix's OR/AND of slot 0 stay valid)
+    lo = grp_kth_largest(samp, ns, 0u, 0xFFFFFFFFu, rs, sh.rs, 0, pc, &need_eq, ct, false);
     int wc = 0;
     for (int b0 = wlo; b0 < whi; b0 += 32 * kU) {
       uint32_t kv[kU];
@@ -649,20 +657,47 @@ __device__ __noinline__ void select_unit(const Fused& F, int u, uint8_t* creg, i
     cbar();
     total = 0;
     for (int w = 0; w < 8; ++w) total += sh.wcnt[w];
+    if (total >= k && (tot_ge < 0 || total < tot_ge)) {
+      lo_ge = lo;
+      tot_ge = total;
+      if (ct < 8) sh.wcnt_ge[ct] = sh.wcnt[ct];
+    }
     if (total >= k && total <= kFusedCandCap) {
       fast = true;
       break;
     }
-    if (total > kFusedCandCap || rs >= ns) break;
-    rs = min(ns, max(rs + 1, static_cast<int>(ceilf(0.5f * static_cast<float>(k + kFusedCandCap) *
-                                                    static_cast<float>(ns) /
-                                                    static_cast<float>(n)))));
-    cbar();  // every thread has read sh.lo and the counts
+    // aim at the middle of [k, capacity] from the density this attempt saw
+    const float per = static_cast<float>(max(total, 1)) / static_cast<float>(rs);
+    int want = static_cast<int>(ceilf(0.5f * static_cast<float>(k + kFusedCandCap) / per));
+    want = total < k ? max(want, rs + 1) : min(want, rs - 1);
+    if (want < 1 || want > ns || want == rs) break;
+    rs = want;
+    cbar();  // every thread has read the counts
   }
-  int pc = 0, need_eq = 0;
+  // the candidates' radix starts afresh
+  radix_init_grp(sh.rs, ct);
+  pc = 0;
+  need_eq = 0;
+  cbar();
+  // The candidates (keys >= lo) in position order: in shared memory when at
+  // most kFusedCandCap, else -- when the raw scores are workspace the select
+  // no longer reads (the chunk edges above were its last use) -- in the
+  // unit's raw-score row, keys in its first half and positions in its second.
+  uint32_t* ckey = sh.key;
+  int* cpos = sh.pos;
+  bool cglob = false;
+  if (!fast && p.raw_scratch && tot_ge >= k && tot_ge <= n / 2) {
+    lo = lo_ge;
+    total = tot_ge;
+    ckey = reinterpret_cast<uint32_t*>(p.raw + soff);
+    cpos = reinterpret_cast<int*>(ckey + n / 2);
+    cglob = true;
+    if (ct < 8) sh.wcnt[ct] = sh.wcnt_ge[ct];
+    cbar();
+    fast = true;
+  }
   uint32_t tau;
   if (fast) {
-    // candidates (keys >= lo) in position order
     int o = 0;
     for (int w = 0; w < cw; ++w) o += sh.wcnt[w];
     for (int b0 = wlo; b0 < whi; b0 += 32 * kU) {
@@ -679,21 +714,27 @@ __device__ __noinline__ void select_unit(const Fused& F, int u, uint8_t* creg, i
         const uint32_t mm = __ballot_sync(0xffffffffu, c);
         const int slot = o + __popc(mm & lanemask_lt(lane));
         if (c) {
-          sh.key[slot] = kv[q];
-          sh.pos[slot] = i;
+          ckey[slot] = kv[q];
+          cpos[slot] = i;
         }
         o += __popc(mm);
       }
     }
+    if (cglob) __threadfence_block();
     cbar();
     constexpr uint32_t kClamp = 0xFFFFu;
-    const uint32_t td = grp_kth_largest(sh.key, total, lo, kClamp, k, sh.rs, 0, pc, &need_eq, ct,
-                                        false);
+    const uint32_t td = grp_kth_largest(ckey, total, lo, kClamp, k, sh.rs, 0, pc, &need_eq, ct,
+                                        cglob);
     tau = lo + td;
     if (td == kClamp)
-      tau = grp_kth_largest(sh.key, total, 0u, 0xFFFFFFFFu, k, sh.rs, 1, pc, &need_eq, ct, false);
-    emit_selected(total, tau, need_eq, out, k, sh, ct, [&](int j) { return sh.key[j]; },
-                  [&](int j) { return sh.pos[j]; });
+      tau = grp_kth_largest(ckey, total, 0u, 0xFFFFFFFFu, k, sh.rs, 1, pc, &need_eq, ct, cglob);
+    if (cglob) {
+      emit_selected(total, tau, need_eq, out, k, sh, ct, [&](int j) { return __ldcg(ckey + j); },
+                    [&](int j) { return __ldcg(cpos + j); });
+    } else {
+      emit_selected(total, tau, need_eq, out, k, sh, ct, [&](int j) { return ckey[j]; },
+                    [&](int j) { return cpos[j]; });
+    }
   } else {
     tau = grp_kth_largest(keys, n, 0u, 0xFFFFFFFFu, k, sh.rs, 1, pc, &need_eq, ct, true);
     emit_selected(n, tau, need_eq, out, k, sh, ct, [&](int j) { return __ldcg(keys + j); },

@@ -179,11 +179,12 @@ static __device__ __noinline__ uint32_t cta_kth_largest(const uint32_t* keys, in
       const int leader = __ffs(act) - 1;
       const uint32_t lb = __shfl_sync(0xffffffffu, bin, leader);
       // one add per warp when its keys share the bin (dense scores), else
-      // one per key
+      // one per distinct bin of the warp
       if (__all_sync(0xffffffffu, !m || bin == lb)) {
         if (lane == leader) atomicAdd(&h[lb], static_cast<uint32_t>(__popc(act)));
       } else if (m) {
-        atomicAdd(&h[bin], 1u);
+        const uint32_t same = __match_any_sync(act, bin);
+        if (lane == __ffs(same) - 1) atomicAdd(&h[bin], static_cast<uint32_t>(__popc(same)));
       }
     }
     sh.hist[(pc + 2) & 3][tid] = 0u;  // one thread per bin (256 threads)

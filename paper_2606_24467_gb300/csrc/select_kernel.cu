@@ -238,13 +238,15 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
       const uint32_t bin = (key >> sh) & 255u;
       const uint32_t active = __ballot_sync(0xffffffffu, match);
       if (active) {
-        // one add per warp when its keys share the bin, else one per key
+        // one add per warp when its keys share the bin, else one per
+        // distinct bin of the warp
         const int leader = __ffs(active) - 1;
         const uint32_t lb = __shfl_sync(0xffffffffu, bin, leader);
         if (__all_sync(0xffffffffu, !match || bin == lb)) {
           if (lane == leader) atomicAdd(&h[lb], static_cast<uint32_t>(__popc(active)));
         } else if (match) {
-          atomicAdd(&h[bin], 1u);
+          const uint32_t same = __match_any_sync(active, bin);
+          if (lane == __ffs(same) - 1) atomicAdd(&h[bin], static_cast<uint32_t>(__popc(same)));
         }
       }
     }
