@@ -337,6 +337,17 @@ int compresskv_compress_layer_noalloc(const ckv_problem* p, const void* q_win, c
  * CKV_OK (or CKV_ERR_CUDA if the copy fails). */
 int compresskv_read_device_status(const void* workspace, void* stream, int32_t* status);
 
+/* Test hook for the failure path of the persistent per-group kernel
+ * (CKV_KERNEL_FUSED): the next call that launches it runs with every bounded
+ * wait limited to wait_ns (instead of 2 s), and its first CTA's claimer
+ * first waits for a counter that nothing sets -- before any copy or UMMA is
+ * issued -- so the wait runs out: the call stops every CTA, its device status
+ * reads CKV_ERR_DEVICE_TIMEOUT, its outputs are undefined and the context
+ * stays usable; compresskv_workspace_init makes the workspace usable again.
+ * wait_ns: 0 cancels a pending stall, else 100000 .. 2000000000 (else
+ * CKV_ERR_INVALID_ARG).  Process-wide, one-shot; not for production use. */
+int compresskv_debug_stall_next_fused_call(long long wait_ns);
+
 /* Error-aware layer budgets (Sec. 3.4: the offline per-layer eviction
  * errors, normalised as in Eq. 4, share the total budget after every layer
  * gets a minimum m, no layer above a maximum M; Sec. 4 uses m = 32 and

@@ -18,6 +18,7 @@ from .compresskv import (  # noqa: F401
     compress_layer_noalloc,
     compress_layers,
     compress_layers_lse,
+    debug_stall_next_fused_call,
     gather,
     head_budget_layout,
     load,

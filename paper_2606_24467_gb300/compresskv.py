@@ -48,6 +48,7 @@ EXPORTED = (
     "compresskv_compress_layers_lse",
     "compresskv_compress_layer_head_budgets",
     "compresskv_read_device_status",
+    "compresskv_debug_stall_next_fused_call",
     "compresskv_allocate_layer_budgets",
     "compresskv_status_string",
 )
@@ -115,6 +116,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         "compresskv_compress_layer_head_budgets": (c_int32, [pp, vp, vp, vp, vp, i32p, vp, i32p,
                                                               vp, vp, vp, vp, vp, c_size_t, vp]),
         "compresskv_read_device_status": (c_int32, [vp, vp, i32p]),
+        "compresskv_debug_stall_next_fused_call": (c_int32, [ctypes.c_longlong]),
         "compresskv_allocate_layer_budgets": (c_int32, [POINTER(ctypes.c_double), c_int32,
                                                         c_int64, c_int32, c_int32, i32p]),
         "compresskv_status_string": (ctypes.c_char_p, [c_int32]),
@@ -428,6 +430,13 @@ def compress_layer_head_budgets(problem: Problem, q_win, k, v, srh_mask, group_b
         _ptr(pooled), _ptr(ws), ws.numel(), _stream(stream)),
         "compresskv_compress_layer_head_budgets")
     return cu_out
+
+
+def debug_stall_next_fused_call(wait_ns: int) -> None:
+    """Test hook: the next persistent-kernel call stalls on purpose and stops
+    with CKV_ERR_DEVICE_TIMEOUT after `wait_ns` (see the header)."""
+    _check(load().compresskv_debug_stall_next_fused_call(ctypes.c_longlong(int(wait_ns))),
+           "compresskv_debug_stall_next_fused_call")
 
 
 def read_device_status(ws, stream=None) -> int:

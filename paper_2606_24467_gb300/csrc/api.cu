@@ -7,6 +7,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstring>
 #include <mutex>
@@ -18,6 +19,10 @@
 using namespace ckv;
 
 namespace {
+
+// Test hook: the wait limit of the next fused call that stalls on purpose
+// (0: none pending).
+std::atomic<long long> g_stall_next_ns{0};
 
 // Workspace header, zeroed by compresskv_workspace_init: the device status
 // word (256 B) and one ticket per scoring item (the scoring kernel's
@@ -938,6 +943,11 @@ int run_fused(const ckv_problem* p, const Info& I, const SrhLists& S, const void
   P.indices = indices;
   P.raw = raw_user ? raw_user : reinterpret_cast<float*>(wb + FL.raw);
   P.raw_scratch = raw_user ? 0 : 1;
+  {
+    const long long stall = g_stall_next_ns.exchange(0);
+    P.wait_ns = stall > 0 ? static_cast<unsigned long long>(stall) : kWaitTimeoutNs;
+    P.stall = stall > 0 ? 1 : 0;
+  }
   P.pooled = pooled_user ? pooled_user : reinterpret_cast<float*>(wb + FL.pooled);
   P.status = reinterpret_cast<int*>(wb);
   P.ctr = reinterpret_cast<int*>(wb + kFusedCtrOffset);
@@ -993,6 +1003,13 @@ int run_fused(const ckv_problem* p, const Info& I, const SrhLists& S, const void
 
 // ====================================================================== C ABI
 extern "C" {
+
+int compresskv_debug_stall_next_fused_call(long long wait_ns) {
+  if (wait_ns < 0 || (wait_ns > 0 && (wait_ns < 100000 || wait_ns > 2000000000ll)))
+    return CKV_ERR_INVALID_ARG;
+  g_stall_next_ns.store(wait_ns);
+  return CKV_OK;
+}
 
 size_t compresskv_workspace_size(const ckv_problem* p) {
   Info I;

@@ -185,7 +185,9 @@ struct FusedParams {
   int window, pool_width, num_kv_heads, group_size, p_total, o_total, is_bf16;
   int n_units, n_chunks, batch;
   int do_select;
-  int raw_scratch;             // raw scores in the workspace: a unit's row may hold its candidates               // 0: scores only (no selection, no gather)
+  int raw_scratch;             // raw scores in the workspace: a unit's row may hold its candidates
+  unsigned long long wait_ns;  // limit of every bounded wait of the call
+  int stall;                   // test hook: CTA 0's claimer first waits for a counter nothing sets               // 0: scores only (no selection, no gather)
   int given_lse;               // 1: no first pass; denominators from `lse`
   int q_half_bytes;            // bytes of one 64-column half of a Q buffer
   int q_bufs;                  // Q buffers (2 or 3)

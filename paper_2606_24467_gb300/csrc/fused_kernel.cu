@@ -49,7 +49,8 @@
 // when it is ready.  Every wait therefore depends only on
 // work claimed earlier by a running CTA that never waits on later work, so a
 // call completes whatever the number of CTAs resident at once; every wait
-// is bounded (kWaitTimeoutNs) and on expiry records CKV_ERR_DEVICE_TIMEOUT
+// is bounded (FusedParams::wait_ns, kWaitTimeoutNs unless a test shortens it)
+// and on expiry records CKV_ERR_DEVICE_TIMEOUT
 // and stops the call.
 // References restart at every chunk and tile t of a chunk always goes to
 // warpgroup t % nwg, so the scores depend only on the chunk grid (fixed per
@@ -91,7 +92,8 @@ constexpr int kCtrPass2 = 1;  // next pass-2 chunk
 constexpr int kCtrMerge = 2;  // next unit whose denominators to merge
 constexpr int kCtrSel = 3;    // next unit to select
 constexpr int kCtrExit = 4;   // CTAs finished
-constexpr int kCtrAbort = 5;  // set when any wait ran out
+constexpr int kCtrAbort = 5;
+constexpr int kCtrNever = 6;  // never set: the test hook's stall waits for it  // set when any wait ran out
 
 constexpr int kTaskEnd = 0;
 constexpr int kTaskMerge = 1;
@@ -179,7 +181,7 @@ struct Fused {
       __nanosleep(64);
       if (ld_acquire(ptr) >= target) return true;
       if (aborted() || *reinterpret_cast<volatile int*>(abort_cta)) return false;
-      if (globaltimer_ns() - t0 > kWaitTimeoutNs) {
+      if (globaltimer_ns() - t0 > p.wait_ns) {
         raise_abort();
         return false;
       }
@@ -188,7 +190,7 @@ struct Fused {
   // Bounded wait on one of this CTA's mbarriers; a timeout stops the call.
   __device__ bool wait_bar(uint32_t bar, uint32_t parity) const {
     if (mbar_test_wait(bar, parity)) return true;
-    const bool ok = mbar_wait_bounded(bar, parity, abort_cta, p.status);
+    const bool ok = mbar_wait_bounded(bar, parity, abort_cta, p.status, p.wait_ns);
     if (!ok && !aborted()) atomicExch(p.ctr + kCtrAbort, 1);
     return ok;
   }
@@ -245,7 +247,7 @@ struct Publisher {
   }
   __device__ bool still_waiting(uint64_t t0) const {
     if (F.aborted() || *reinterpret_cast<volatile int*>(F.abort_cta)) return false;
-    if (globaltimer_ns() - t0 > kWaitTimeoutNs) {
+    if (globaltimer_ns() - t0 > F.p.wait_ns) {
       F.raise_abort();
       return false;
     }
@@ -779,7 +781,7 @@ __device__ void claim_task(const Fused& F, int* task) {
     const uint64_t now = globaltimer_ns();
     if (t0 == 0) {
       t0 = now;
-    } else if (now - t0 > kWaitTimeoutNs) {
+    } else if (now - t0 > p.wait_ns) {
       F.raise_abort();
       break;
     }
@@ -911,6 +913,9 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
     if (lane == 0) {
       Publisher pb{F, pubfull(0), pubempty(0), {}, 0, 0};
       int pending = -1;  // pass-2 chunk claimed, not yet published
+      // test hook: a wait that cannot complete, before anything is issued;
+      // it runs out after p.wait_ns and stops the call
+      if (p.stall && blockIdx.x == 0) F.wait_counter(p.ctr + kCtrNever, 1);
       for (int c = 0;; ++c) {
         const int ds = c % kDescs;
         if (!pb.wait_bar(dempty(ds), ((c / kDescs) & 1) ^ 1)) break;

@@ -273,3 +273,12 @@ def test_binding_checks_lse_tensor():
                                     k, k, ws)
         assert e.value.code == B.CKV_ERR_INVALID_ARG
 
+
+
+def test_stall_hook_limits():
+    """The failure-path test hook takes 0 (cancel) or 0.1 ms .. 2 s."""
+    for bad in (-1, 99_999, 2_000_000_001):
+        with pytest.raises(ckv.CompressKVError):
+            ckv.debug_stall_next_fused_call(bad)
+    ckv.debug_stall_next_fused_call(1_000_000)
+    ckv.debug_stall_next_fused_call(0)  # cancelled: no later call stalls

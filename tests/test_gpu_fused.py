@@ -154,3 +154,35 @@ def test_full_32_layer_llama8b_32k_in_one_call(cuda_device):
     out, cu_out, cu = _run_call(layers, cfg, dev, scores=False)
     for l in (0, cfg.n_layers - 1):
         _check_block(_block(out, cu_out, cu, l, cfg.batch, cfg.window), layers[l], cfg)
+
+
+def test_bounded_wait_runs_out_and_the_workspace_recovers(cuda_device):
+    """The failure path of the persistent kernel: a wait that cannot complete
+    (the test hook's counter, before anything is issued) runs out after 2 ms;
+    the call returns, every CTA stops, the device status reads
+    CKV_ERR_DEVICE_TIMEOUT and, after workspace_init, the same call on the
+    same workspace is correct again."""
+    dev = cuda_device
+    cfg = wl.get("c2").scaled(seq_len=9000, n_layers=4)
+    layers = _layers(cfg)
+    q_all, k_all, v_all, cu, b_all, m_all = _pack(layers, dev)
+    prob = ckv.Problem(q_all, k_all, cu, cfg.window, cfg.pool_width)
+    out = ckv.LayerOutputs(prob, b_all, 128, k_all.dtype, dev, scores=True)
+    ws = ckv.workspace(prob, dev)
+
+    def call():
+        return ckv.compress_layers(prob, len(layers), q_all, k_all, v_all, m_all, b_all,
+                                   out.indices, out.k_out, out.v_out, ws, raw=out.raw,
+                                   pooled=out.pooled)
+
+    ckv.debug_stall_next_fused_call(2_000_000)
+    call()
+    torch.cuda.synchronize()
+    assert ckv.read_device_status(ws) == ckv.compresskv.CKV_ERR_DEVICE_TIMEOUT
+    ckv.compresskv._check(ckv.load().compresskv_workspace_init(ckv.compresskv._ptr(ws), ws.numel(),
+                                                               None), "workspace_init")
+    cu_out = call()
+    torch.cuda.synchronize()
+    assert ckv.read_device_status(ws) == 0
+    for l in (0, 3):
+        _check_block(_block(out, cu_out, cu, l, cfg.batch, cfg.window), layers[l], cfg)
