@@ -12,6 +12,8 @@ from .compresskv_oracle import (  # noqa: F401
     kept_count,
     kth_value,
     pool_avg,
+    pool_heads,
+    pool_max,
     raw_scores,
     select_top,
     srh_heads,

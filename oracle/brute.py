@@ -12,9 +12,11 @@ from __future__ import annotations
 import math
 
 
-def brute_unit(q_heads, k_unit, window, pool_width, budget, scale):
+def brute_unit(q_heads, k_unit, window, pool_width, budget, scale, pool_kind="avg"):
     """q_heads: list over SRH heads of W lists of d floats; k_unit: L lists of
-    d floats.  Returns (raw, pooled, indices) as Python lists."""
+    d floats.  pool_kind "avg" pools the heads' sum; "max" takes, per head,
+    the largest window-summed attention within the pooling window and sums
+    those over the heads.  Returns (raw, pooled, indices) as Python lists."""
     L = len(k_unit)
     W = window
     if budget < W:
@@ -24,7 +26,8 @@ def brute_unit(q_heads, k_unit, window, pool_width, budget, scale):
     n = L - W
     raw = [0.0] * n
     terms = [[] for _ in range(n)]
-    for head in q_heads:
+    head_terms = [[[] for _ in range(n)] for _ in q_heads]
+    for hi, head in enumerate(q_heads):
         for w in range(W):
             p = L - W + w
             logits = []
@@ -35,16 +38,29 @@ def brute_unit(q_heads, k_unit, window, pool_width, budget, scale):
             z = math.fsum(exps)
             for j in range(n):
                 terms[j].append(exps[j] / z)
+                head_terms[hi][j].append(exps[j] / z)
     for j in range(n):
         raw[j] = math.fsum(terms[j])
     r = (pool_width - 1) // 2
     pooled = []
-    for j in range(n):
-        acc = []
-        for t in range(-r, r + 1):
-            if 0 <= j + t < n:
-                acc.append(raw[j + t])
-        pooled.append(math.fsum(acc) / pool_width)
+    if pool_kind == "max":
+        head_raw = [[math.fsum(ht[j]) for j in range(n)] for ht in head_terms]
+        for j in range(n):
+            best = []
+            for hr in head_raw:
+                m = None
+                for t in range(-r, r + 1):
+                    if 0 <= j + t < n and (m is None or hr[j + t] > m):
+                        m = hr[j + t]
+                best.append(m)
+            pooled.append(math.fsum(best))
+    else:
+        for j in range(n):
+            acc = []
+            for t in range(-r, r + 1):
+                if 0 <= j + t < n:
+                    acc.append(raw[j + t])
+            pooled.append(math.fsum(acc) / pool_width)
     k = min(budget, L) - W
     ranked = sorted(range(n), key=lambda j: (-pooled[j], j))
     chosen = sorted(ranked[:k])

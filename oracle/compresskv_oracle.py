@@ -24,7 +24,9 @@ for every sequence ``s`` and GQA KV group ``g`` (a *unit*):
    window"; heads are combined by a sum, whose ranking equals the paper's
    average because ``|S|`` is fixed within a unit).
 4. pooled score: average pooling of width ``P`` (stride 1, ``r = (P-1)/2``
-   zeros of padding on each side, divisor ``P``) over the prefix scores.
+   zeros of padding on each side, divisor ``P``) over the prefix scores; or,
+   as an option, max pooling of each SRH head's window-summed attention
+   over ``[j - r, j + r]`` before the heads are summed (``pool_heads``).
 5. keep the ``k = min(B, L) - W`` prefix tokens with the largest pooled score
    (Sec. 3.3 "top N"; ties go to the lower position), plus the ``W`` window
    tokens, in ascending position order.
@@ -131,6 +133,36 @@ def pool_avg(raw: np.ndarray, pool_width: int) -> np.ndarray:
     return out
 
 
+def pool_max(raw: np.ndarray, pool_width: int) -> np.ndarray:
+    """Max pooling, stride 1, over ``[j - r, j + r]`` clipped to the prefix
+    (padding that never wins: scores are non-negative, so -inf and zero
+    padding agree); output has the input's length."""
+    if pool_width < 1 or pool_width % 2 == 0:
+        raise OracleError("pool width must be odd and >= 1")
+    raw = np.asarray(raw, np.float64)
+    n = raw.shape[0]
+    r = (pool_width - 1) // 2
+    out = np.zeros(n, dtype=np.float64)
+    for j in range(n):
+        out[j] = raw[max(0, j - r): min(n, j + r + 1)].max()
+    return out
+
+
+def pool_heads(attn_per_head: list[np.ndarray], n: int, pool_width: int, pool_kind: str) -> np.ndarray:
+    """Pooled score of a set of SRH heads (Sec. 3.3: pooling across the token
+    dimension, then the heads' vectors combined by a sum).  Average pooling
+    is linear, so it is applied to the head sum; max pooling is applied to
+    each head's window-summed attention before the sum."""
+    if pool_kind == "avg":
+        return pool_avg(raw_scores(attn_per_head, n), pool_width)
+    if pool_kind != "max":
+        raise OracleError("pool kind must be 'avg' or 'max'")
+    total = np.zeros(n, dtype=np.float64)
+    for A in attn_per_head:
+        total += pool_max(raw_scores([A], n), pool_width)
+    return total
+
+
 # ---------------------------------------------------------------------------
 # Step 5: top-k prefix selection (Sec. 3.3 "top N")
 # ---------------------------------------------------------------------------
@@ -176,7 +208,8 @@ class UnitResult:
 
 
 def compress_unit(q_heads: np.ndarray, k_unit: np.ndarray, window: int, pool_width: int,
-                  budget: int, scale: float, keep_attn: bool = False) -> UnitResult:
+                  budget: int, scale: float, keep_attn: bool = False,
+                  pool_kind: str = "avg") -> UnitResult:
     """Steps 2-5 for one unit.
 
     q_heads: ``[|S|, W, d]`` window queries of the unit's SRH heads.
@@ -194,7 +227,8 @@ def compress_unit(q_heads: np.ndarray, k_unit: np.ndarray, window: int, pool_wid
         raise OracleError("KV group without any SRH head")
     attn = [window_attention(q_heads[i], k_unit, scale) for i in range(q_heads.shape[0])]
     raw = raw_scores(attn, n)
-    pooled = pool_avg(raw, pool_width)
+    pooled = pool_avg(raw, pool_width) if pool_kind == "avg" else pool_heads(attn, n, pool_width,
+                                                                            pool_kind)
     k = kept - W
     sel = select_top(pooled, k)
     idx = np.concatenate([sel, np.arange(n, L, dtype=np.int64)])
@@ -262,7 +296,8 @@ def default_scale(head_dim: int) -> float:
 
 def compress_layer(q_win, k, v, cu_seqlens, srh_mask, budgets, window: int,
                    pool_width: int, scale: float | None = None,
-                   keep_attn: bool = False, selection: str = "group") -> LayerResult:
+                   keep_attn: bool = False, selection: str = "group",
+                   pool_kind: str = "avg") -> LayerResult:
     """Oracle of one layer's compression.
 
     q_win: ``[B, H_q, W, d]`` window queries (position ``L_s - W + w``).
@@ -270,6 +305,7 @@ def compress_layer(q_win, k, v, cu_seqlens, srh_mask, budgets, window: int,
            ``cu_seqlens[s] : cu_seqlens[s+1]``.
     srh_mask: ``[H_q]`` booleans; budgets: ``[B]`` ints (per sequence).
     selection: ``"group"`` or ``"layer"`` (see the module docstring).
+    pool_kind: ``"avg"`` or ``"max"`` (``pool_heads``).
     """
     if selection not in ("group", "layer"):
         raise OracleError("selection must be 'group' or 'layer'")
@@ -314,9 +350,9 @@ def compress_layer(q_win, k, v, cu_seqlens, srh_mask, budgets, window: int,
                     # then the heads' vectors are combined
                     attn = [window_attention(q64[s, h], ku, scale) for h in heads]
                     for A in attn:
-                        layer_pooled += pool_avg(raw_scores([A], n), pool_width)
+                        layer_pooled += pool_heads([A], n, pool_width, pool_kind)
                     g_raw = raw_scores(attn, n)
-                    g_pooled = pool_avg(g_raw, pool_width)
+                    g_pooled = pool_heads(attn, n, pool_width, pool_kind)
                 else:
                     attn, g_raw, g_pooled = [], np.zeros(n), np.zeros(n)
                 units[(s, g)] = UnitResult(heads, g_raw, g_pooled, 0, float("nan"),
@@ -347,7 +383,8 @@ def compress_layer(q_win, k, v, cu_seqlens, srh_mask, budgets, window: int,
                 raise OracleError(f"KV group {g} has no SRH head")
             qh = q64[s, heads] if heads else np.zeros((0, window, k.shape[2]))
             ku = k64[cu[s]:cu[s + 1], g]
-            res = compress_unit(qh, ku, window, pool_width, int(budgets[s]), scale, keep_attn)
+            res = compress_unit(qh, ku, window, pool_width, int(budgets[s]), scale, keep_attn,
+                                pool_kind)
             res.heads = heads
             units[(s, g)] = res
             raw[g, cu_prefix[s]:cu_prefix[s + 1]] = res.raw
