@@ -90,7 +90,19 @@ enum {
 #define CKV_STATIC_SCRATCH_BYTES (16u * 1024u * 1024u)
 
 enum { CKV_DTYPE_F16 = 0, CKV_DTYPE_BF16 = 1 };
-enum { CKV_POOL_AVG = 0 };
+/* Pooling across the token dimension (Sec. 3.3, width P of Sec. 4).  AVG:
+ * average pooling of the heads' summed window scores (divisor P, zero
+ * padding; linear, so the order of pooling and head sum does not matter).
+ * MAX: each SRH head's window-summed attention is max-pooled over
+ * [j - r, j + r] within the prefix, then the heads' pooled vectors are
+ * summed (pooling before the head sum, the paper's order).  MAX is taken by
+ * compresskv_compress_layer(s) and compresskv_compress_layer_noalloc (both
+ * selection scopes; the heads are scored one SRH head per group at a time,
+ * then pooled and selected; the workspace holds one more raw-score row per
+ * head of a group) and by compresskv_score (raw scores do not depend on it);
+ * compresskv_select (its input is already summed over the heads), the
+ * given-LSE and the head-budget calls return CKV_ERR_UNSUPPORTED for it. */
+enum { CKV_POOL_AVG = 0, CKV_POOL_MAX = 1 };
 /* Selection scope.  PER_GROUP: every KV group keeps the tokens its own SRH
  * heads rank highest, and a group without an SRH head is an error.
  * PER_LAYER (Sec. 3.3 read literally: all heads of a layer share one set of
@@ -130,9 +142,9 @@ typedef struct ckv_problem {
   int32_t num_kv_heads;     /* H_kv, 1..64 */
   int32_t head_dim;         /* d; 128 */
   int32_t window;           /* W >= 1, the observation window (Sec. 4) */
-  int32_t pool_width;       /* P, odd, 1..63, average pooling width (Sec. 4) */
+  int32_t pool_width;       /* P, odd, 1..63, pooling width (Sec. 4) */
   int32_t dtype;            /* CKV_DTYPE_F16 | CKV_DTYPE_BF16 for Q, K and V */
-  int32_t pool_kind;        /* CKV_POOL_AVG */
+  int32_t pool_kind;        /* CKV_POOL_AVG | CKV_POOL_MAX */
   float scale;              /* softmax scale; 0 selects 1/sqrt(head_dim) */
   int32_t selection;        /* CKV_SELECT_PER_GROUP or CKV_SELECT_PER_LAYER */
   const int32_t* cu_seqlens;/* host [batch+1] */

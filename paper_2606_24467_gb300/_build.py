@@ -18,6 +18,7 @@ INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB_PATH = os.path.join(OUT_DIR, "libcompresskv.so")
 SOURCES = ["api.cu", "fused_kernel.cu", "score_kernel.cu", "combine_kernel.cu", "select_kernel.cu",
+           "pool_kernel.cu",
            "gather_kernel.cu", "budget_alloc.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

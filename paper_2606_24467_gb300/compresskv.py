@@ -30,6 +30,7 @@ STATIC_SCRATCH_BYTES = 16 * 1024 * 1024
 CKV_DTYPE_F16 = 0
 CKV_DTYPE_BF16 = 1
 CKV_POOL_AVG = 0
+CKV_POOL_MAX = 1
 CKV_SELECT_PER_GROUP = 0
 CKV_SELECT_PER_LAYER = 1
 KERNEL_KINDS = {1: "score", 2: "combine", 3: "select", 4: "gather", 5: "fused"}
@@ -164,9 +165,10 @@ class Problem:
 
     def __init__(self, q_win: torch.Tensor, k: torch.Tensor, cu_seqlens, window: int,
                  pool_width: int, scale: float = 0.0, trace: "Trace | None" = None,
-                 selection: str = "group"):
+                 selection: str = "group", pool: str = "avg"):
         """``selection``: "group" (each KV group keeps its own SRH heads'
-        choice) or "layer" (one choice per sequence shared by every group)."""
+        choice) or "layer" (one choice per sequence shared by every group);
+        ``pool``: "avg" or "max" (each SRH head max-pooled, then summed)."""
         if k.dtype not in (torch.float16, torch.bfloat16) or q_win.dtype != k.dtype:
             raise CompressKVError(CKV_ERR_INVALID_ARG, "Q and K must share an f16/bf16 dtype")
         self._cu, cu_ptr = _i32(cu_seqlens)
@@ -179,7 +181,9 @@ class Problem:
         s.window = int(window)
         s.pool_width = int(pool_width)
         s.dtype = CKV_DTYPE_BF16 if k.dtype == torch.bfloat16 else CKV_DTYPE_F16
-        s.pool_kind = CKV_POOL_AVG
+        if pool not in ("avg", "max"):
+            raise CompressKVError(CKV_ERR_INVALID_ARG, "pool must be 'avg' or 'max'")
+        s.pool_kind = CKV_POOL_MAX if pool == "max" else CKV_POOL_AVG
         s.scale = float(scale)
         if selection not in ("group", "layer"):
             raise CompressKVError(CKV_ERR_INVALID_ARG, "selection must be 'group' or 'layer'")

@@ -109,6 +109,7 @@ struct Info {
   int B = 0, Hq = 0, Hkv = 0, G = 0, W = 0, P = 0;
   bool bf16 = false;
   bool layer = false;  // CKV_SELECT_PER_LAYER
+  bool pool_max = false;  // CKV_POOL_MAX
   float scale = 0.f;
   std::vector<int> cu, len, n, cu_prefix;
   long long T = 0, p_total = 0;
@@ -164,7 +165,7 @@ int validate(const ckv_problem* p, Info& I) {
   if (p->window < 1) return CKV_ERR_INVALID_ARG;
   if (p->pool_width < 1 || p->pool_width % 2 == 0 || p->pool_width > 63) return CKV_ERR_INVALID_ARG;
   if (p->dtype != CKV_DTYPE_F16 && p->dtype != CKV_DTYPE_BF16) return CKV_ERR_INVALID_ARG;
-  if (p->pool_kind != CKV_POOL_AVG) return CKV_ERR_UNSUPPORTED;
+  if (p->pool_kind != CKV_POOL_AVG && p->pool_kind != CKV_POOL_MAX) return CKV_ERR_INVALID_ARG;
   if (p->selection != CKV_SELECT_PER_GROUP && p->selection != CKV_SELECT_PER_LAYER)
     return CKV_ERR_INVALID_ARG;
   if (!(p->scale >= 0.f) || std::isinf(p->scale)) return CKV_ERR_INVALID_ARG;
@@ -182,6 +183,7 @@ int validate(const ckv_problem* p, Info& I) {
   I.P = p->pool_width;
   I.bf16 = p->dtype == CKV_DTYPE_BF16;
   I.layer = p->selection == CKV_SELECT_PER_LAYER;
+  I.pool_max = p->pool_kind == CKV_POOL_MAX;
   I.scale = p->scale > 0.f ? p->scale : 1.0f / std::sqrt(static_cast<float>(kHeadDim));
   I.cu.assign(p->cu_seqlens, p->cu_seqlens + I.B + 1);
   if (I.cu[0] != 0) return CKV_ERR_INVALID_ARG;
@@ -314,8 +316,17 @@ FusedLayout fused_layout(const Info& I) {
   return F;
 }
 
+// Max pooling: after both layouts, one raw-score row per SRH head slot (at
+// most G) of every group.
+size_t maxpool_slots_offset(const Info& I) {
+  return align256(std::max(workspace_layout(I).total, fused_layout(I).total));
+}
+
 size_t workspace_bytes(const Info& I) {
-  return std::max(workspace_layout(I).total, fused_layout(I).total);
+  const size_t base = std::max(workspace_layout(I).total, fused_layout(I).total);
+  if (!I.pool_max) return base;
+  return maxpool_slots_offset(I) +
+         align256(static_cast<size_t>(I.G) * I.Hkv * I.p_total * sizeof(float));
 }
 
 int carve(const Info& I, void* ws, size_t bytes, Workspace& out) {
@@ -1002,6 +1013,81 @@ int run_fused(const ckv_problem* p, const Info& I, const SrhLists& S, const void
 }  // namespace
 
 // ====================================================================== C ABI
+// compresskv_compress_layers under CKV_POOL_MAX: the raw scores of every
+// list's i-th SRH head (one head per group at a time, scored by the per-group
+// scoring path), then each head max-pooled and the heads summed, then the
+// selection from those pooled scores (per group or per layer) with the
+// gather.  Lists with fewer heads score their first head again in the later
+// rounds (a placeholder the pooling ignores), so every round is a valid
+// per-group problem.
+int run_maxpool_compress(const ckv_problem* p, const Info& I, const uint8_t* srh_masks,
+                         const void* q_win, const void* k, const void* v,
+                         const std::vector<int>& co, int32_t* indices, void* k_out, void* v_out,
+                         float* raw_scores, float* pooled_scores, const Workspace& ws,
+                         void* workspace, size_t workspace_bytes, cudaStream_t st) {
+  const int nl = I.n_masks * I.Hkv;
+  if (nl > kFusedMaxLists || I.G > 255) return CKV_ERR_UNSUPPORTED;
+  std::vector<std::vector<int>> heads(nl);
+  int rounds = 0;
+  for (int m = 0; m < I.n_masks; ++m)
+    for (int g = 0; g < I.Hkv; ++g) {
+      std::vector<int>& hl = heads[m * I.Hkv + g];
+      for (int i = 0; i < I.G; ++i)
+        if (srh_masks[static_cast<size_t>(m) * I.Hq + g * I.G + i]) hl.push_back(g * I.G + i);
+      rounds = std::max(rounds, static_cast<int>(hl.size()));
+    }
+  ckv_problem pg = *p;
+  pg.selection = CKV_SELECT_PER_GROUP;
+  pg.pool_kind = CKV_POOL_AVG;
+  Info Ig = I;
+  Ig.layer = false;
+  Ig.pool_max = false;
+  float* slots = reinterpret_cast<float*>(static_cast<char*>(workspace) + maxpool_slots_offset(I));
+  const long long slot_stride = static_cast<long long>(I.Hkv) * I.p_total;
+  std::vector<uint8_t> mask_i(static_cast<size_t>(I.n_masks) * I.Hq);
+  std::vector<int> co0(I.B + 1, 0);
+  int rc = CKV_OK;
+  for (int r = 0; r < rounds; ++r) {
+    std::fill(mask_i.begin(), mask_i.end(), 0);
+    for (int m = 0; m < I.n_masks; ++m)
+      for (int g = 0; g < I.Hkv; ++g) {
+        const std::vector<int>& hl = heads[m * I.Hkv + g];
+        const int h = hl.empty() ? g * I.G : hl[std::min(r, static_cast<int>(hl.size()) - 1)];
+        mask_i[static_cast<size_t>(m) * I.Hq + h] = 1;
+      }
+    SrhLists Si;
+    if ((rc = srh_lists(Ig, mask_i.data(), Si)) != CKV_OK) return rc;
+    float* raw_r = slots + r * slot_stride;
+    bool handled = false;
+    rc = run_fused(&pg, Ig, Si, q_win, k, nullptr, co0, nullptr, nullptr, nullptr, raw_r, nullptr,
+                   workspace, workspace_bytes, st, &handled, false);
+    if (!handled) rc = run_score(&pg, Ig, q_win, k, mask_i.data(), raw_r, ws.pooled, ws, st);
+    if (rc != CKV_OK) return rc;
+  }
+  static thread_local MaxPoolParams M;
+  std::memset(&M, 0, sizeof(M));
+  M.slots = slots;
+  M.slot_stride = slot_stride;
+  float* pooled = pooled_scores ? pooled_scores : ws.pooled;
+  M.pooled = pooled;
+  M.raw = raw_scores;
+  M.num_kv_heads = I.Hkv;
+  M.batch = I.B;
+  M.seqs_per_mask = I.spm;
+  M.pool_width = I.P;
+  M.p_total = static_cast<int>(I.p_total);
+  int max_n = 0;
+  for (int s = 0; s <= I.B; ++s) {
+    M.cu_prefix[s] = static_cast<int>(I.cu_prefix[s]);
+    if (s < I.B) max_n = std::max(max_n, I.n[s]);
+  }
+  for (int l = 0; l < nl; ++l) M.heads_of[l] = static_cast<uint8_t>(heads[l].size());
+  Tracer tr{p->trace, st};
+  if ((rc = traced(tr, CKV_KERNEL_COMBINE, [&] { return launch_maxpool(M, max_n, st); })) != CKV_OK)
+    return rc;
+  return run_select(p, I, nullptr, pooled, co, indices, nullptr, ws, st, k, v, k_out, v_out);
+}
+
 extern "C" {
 
 int compresskv_debug_stall_next_fused_call(long long wait_ns) {
@@ -1069,6 +1155,7 @@ int compresskv_select(const ckv_problem* p, const float* raw_scores, const int32
   Info I;
   int rc = validate(p, I);
   if (rc != CKV_OK) return rc;
+  if (I.pool_max) return CKV_ERR_UNSUPPORTED;  // needs the per-head scores
   std::vector<int> co;
   if ((rc = output_layout(I, budgets, co)) != CKV_OK) return rc;
   if (!cu_out) return CKV_ERR_INVALID_ARG;
@@ -1134,6 +1221,12 @@ int compresskv_compress_layers(const ckv_problem* p, int n_masks, const void* q_
   SrhLists S;
   if ((rc = srh_lists(I, srh_mask, S)) != CKV_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (I.pool_max) {
+    if ((rc = check_outputs(I, co, indices, k, v, k_out, v_out)) != CKV_OK) return rc;
+    std::copy(co.begin(), co.end(), cu_out);
+    return run_maxpool_compress(p, I, srh_mask, q_win, k, v, co, indices, k_out, v_out,
+                                raw_scores, pooled_scores, ws, workspace, workspace_bytes, st);
+  }
   if (!I.layer) {
     // per-group selection: one persistent kernel for every unit of the call
     bool handled = false;
@@ -1181,6 +1274,7 @@ int compresskv_compress_layers_lse(const ckv_problem* p, int n_masks, const void
   Info I;
   int rc = validate(p, I);
   if (rc != CKV_OK) return rc;
+  if (I.pool_max) return CKV_ERR_UNSUPPORTED;  // needs the per-head scores
   if (n_masks < 1 || I.B % n_masks != 0) return CKV_ERR_INVALID_ARG;
   if (n_masks > kMaxFusedMasks) return CKV_ERR_UNSUPPORTED;
   I.n_masks = n_masks;
@@ -1230,6 +1324,7 @@ int compresskv_compress_layer_head_budgets(const ckv_problem* p, const void* q_w
   Info I;
   int rc = validate(p, I);
   if (rc != CKV_OK) return rc;
+  if (I.pool_max) return CKV_ERR_UNSUPPORTED;  // needs the per-head scores
   if (I.layer) return CKV_ERR_INVALID_ARG;  // one shared selection has one budget
   if (!group_budgets || !cu_out) return CKV_ERR_INVALID_ARG;
   if (static_cast<long long>(I.B) * I.Hkv > kMaxBudgetUnits) return CKV_ERR_UNSUPPORTED;

@@ -214,6 +214,19 @@ static_assert(sizeof(CombineParams) <= 32764, "combine kernel parameters");
 static_assert(sizeof(SelectParams) <= 32764, "selection kernel parameters");
 static_assert(sizeof(FusedParams) <= 32764, "fused kernel parameters");
 
+// Max pooling of each SRH head's window scores, summed over the heads: head
+// slot i of list (mask m, group g) holds the raw scores of that list's i-th
+// SRH head (slots of a list beyond its head count are ignored).
+struct MaxPoolParams {
+  const float* slots;          // [n_slots][H_kv][p_total]
+  long long slot_stride;       // H_kv * p_total
+  float* pooled;               // [H_kv][p_total]
+  float* raw;                  // optional: the slots' raw scores summed
+  int num_kv_heads, batch, seqs_per_mask, pool_width, p_total;
+  int cu_prefix[kMaxBatch + 1];
+  uint8_t heads_of[kFusedMaxLists];  // SRH heads of list srh_group(s, g, ...)
+};
+
 // Host-side launchers (defined next to each kernel).
 cudaError_t launch_score(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s);
 cudaError_t launch_score_lse(const ScoreParams& p, int n_items, size_t smem, cudaStream_t s);
@@ -228,6 +241,7 @@ cudaError_t launch_select_sampled(const SelectParams& p, int n_units, size_t sme
 size_t select_sampled_smem_bytes(int slice);
 int select_sampled_max_cluster(int slice);  // 16 when the device takes such clusters, else 8
 cudaError_t launch_gather(const GatherParams& p, long long rows, cudaStream_t s);
+cudaError_t launch_maxpool(const MaxPoolParams& p, int max_n, cudaStream_t s);
 size_t score_smem_bytes(int q_half_bytes, int stages, int epi_warps);
 // Sets every scoring kernel's shared-memory limit: `bytes` for one CTA per
 // SM, half of it for the two-CTA form.

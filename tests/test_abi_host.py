@@ -71,7 +71,7 @@ def test_invalid_shapes_rejected():
                                ("window", 0, B.CKV_ERR_INVALID_ARG),
                                ("num_q_heads", 7, B.CKV_ERR_INVALID_ARG),
                                ("dtype", 5, B.CKV_ERR_INVALID_ARG),
-                               ("pool_kind", 1, B.CKV_ERR_UNSUPPORTED),
+                               ("pool_kind", 2, B.CKV_ERR_INVALID_ARG),
                                ("kv_token_stride", 100, B.CKV_ERR_INVALID_ARG)):
         old = getattr(s, field)
         setattr(s, field, value)
@@ -282,3 +282,27 @@ def test_stall_hook_limits():
             ckv.debug_stall_next_fused_call(bad)
     ckv.debug_stall_next_fused_call(1_000_000)
     ckv.debug_stall_next_fused_call(0)  # cancelled: no later call stalls
+
+
+def test_max_pooling_workspace_and_unsupported_calls():
+    """CKV_POOL_MAX: the workspace grows by one raw-score row per group head
+    slot (G rows per group); the calls that cannot pool per head refuse it
+    on the host."""
+    lib = ckv.load()
+    prob, q, k = _problem()
+    s = prob.struct
+    avg = lib.compresskv_workspace_size(prob.ref)
+    s.pool_kind = B.CKV_POOL_MAX
+    mx = lib.compresskv_workspace_size(prob.ref)
+    G = s.num_q_heads // s.num_kv_heads
+    p_total = sum(max(int(prob._cu[i + 1] - prob._cu[i]) - s.window, 0) for i in range(s.batch))
+    assert mx >= avg + G * s.num_kv_heads * p_total * 4
+    assert mx <= avg + 256 + (G * s.num_kv_heads * p_total * 4 + 255) // 256 * 256 + 256
+    vp = ctypes.c_void_p
+    ws = vp(_fake_dev_ptr())
+    bud, bp = B._i32([64, 64])
+    cu_out = (ctypes.c_int32 * 3)()
+    rc = lib.compresskv_select(prob.ref, vp(_fake_dev_ptr()), bp, vp(_fake_dev_ptr()), cu_out, None,
+                               ws, mx, None)
+    assert rc == B.CKV_ERR_UNSUPPORTED
+    s.pool_kind = B.CKV_POOL_AVG
