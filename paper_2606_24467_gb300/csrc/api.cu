@@ -912,10 +912,11 @@ int run_fused(const ckv_problem* p, const Info& I, const SrhLists& S, const void
   int rc = device_facts(&Fd);
   if (rc != CKV_OK) return rc;
   // three Q buffers when they fit beside a ring of at least four K tiles,
-  // else two beside at least two
+  // else two beside at least two; an even number of stages (each UMMA warp
+  // has half of them)
   int stages = 0, q_bufs = 0;
   for (int nq = 3; nq >= 2 && stages == 0; --nq) {
-    for (int st = 8; st >= (nq == 3 ? 4 : 2); --st) {
+    for (int st = 8; st >= (nq == 3 ? 4 : 2); st -= 2) {
       if (fused_smem_bytes(q_half, nq, st, row_stride, nwg) <=
           static_cast<size_t>(Fd->smem_optin)) {
         stages = st;

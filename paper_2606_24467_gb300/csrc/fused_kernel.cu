@@ -32,7 +32,9 @@
 //               up to kDescs ahead, in a descriptor ring;
 //   warp 0      loads each chunk's SRH query rows (one TMA box of W rows per
 //               head and 64-column half) into one of two or three Q buffers
-//               and streams its K tiles into a shared-memory ring, by TMA;
+//               and streams its K tiles, by TMA, into a shared-memory ring
+//               split in two sub-rings, one per UMMA warp (each consumes
+//               its own in order);
 //   warps 1, 2  UMMA issue (M = 128 keys, N = query rows), warp 1 for the
 //               tiles of warpgroup 0 and warp 2 for those of warpgroup 1
 //               (a UMMA of this shape holds the tensor core for a fixed 76
@@ -519,7 +521,7 @@ __device__ void emit_selected(int count, uint32_t tau, int need_eq, int32_t* out
 // Copy the K and V rows of out[0..count) (positions in the sequence) to the
 // compressed cache rows out0 .. out0 + count - 1 of group g.  Eight 16-byte
 // loads in flight per thread.
-__device__ __noinline__ void gather_rows(const FusedParams& p, int seq0, int g,
+__device__ __noinline__ void gather_rows(const FusedParams& p, int seq0, int L, int g,
                                          const int32_t* out, int out0, int count, int ct) {
   constexpr int kChunks = 2 * kHeadDim * 2 / 16;  // 16 K + 16 V chunks per token
   constexpr int kBatch = 8;
@@ -537,6 +539,10 @@ __device__ __noinline__ void gather_rows(const FusedParams& p, int seq0, int g,
         const int i = e / kChunks;
         const int ch = e - i * kChunks;
         const int tok = out[i];
+        if (tok < 0 || tok >= L) {  // never for a correct selection: record, skip
+          if (ch == 0) atomicCAS(p.status, 0, CKV_DEV_ERR_INDEX);
+          continue;
+        }
         is_v[k] = ch >= kChunks / 2;
         const int part = ch & (kChunks / 2 - 1);
         const long long src = static_cast<long long>(seq0 + tok) * p.tok_stride_v16 +
@@ -609,7 +615,7 @@ __device__ __noinline__ void select_unit(const Fused& F, int u, uint8_t* creg, i
     for (int i = ct; i < L; i += kCThreads) out[i] = i;
     __threadfence_block();
     cbar();
-    gather_rows(p, seq0, g, out, out0, L, ct);
+    gather_rows(p, seq0, L, g, out, out0, L, ct);
     return;
   }
   const int k = kept - W;  // 0 <= k < n
@@ -617,7 +623,7 @@ __device__ __noinline__ void select_unit(const Fused& F, int u, uint8_t* creg, i
   if (k == 0) {
     __threadfence_block();
     cbar();
-    gather_rows(p, seq0, g, out, out0, W, ct);
+    gather_rows(p, seq0, L, g, out, out0, W, ct);
     return;
   }
   const uint32_t* keys = reinterpret_cast<const uint32_t*>(pooled);
@@ -715,9 +721,11 @@ __device__ __noinline__ void select_unit(const Fused& F, int u, uint8_t* creg, i
         const bool c = i < whi && kv[q] >= lo;
         const uint32_t mm = __ballot_sync(0xffffffffu, c);
         const int slot = o + __popc(mm & lanemask_lt(lane));
-        if (c) {
+        if (c && slot < total) {
           ckey[slot] = kv[q];
           cpos[slot] = i;
+        } else if (c) {  // more keys above lo than counted: cannot happen; record
+          atomicCAS(p.status, 0, CKV_DEV_ERR_INDEX);
         }
         o += __popc(mm);
       }
@@ -744,7 +752,7 @@ __device__ __noinline__ void select_unit(const Fused& F, int u, uint8_t* creg, i
   }
   __threadfence_block();
   cbar();  // the indices written above are read back by the copy
-  gather_rows(p, seq0, g, out, out0, kept, ct);
+  gather_rows(p, seq0, L, g, out, out0, kept, ct);
 }
 
 // The workers' next task (one thread): the next unit to select once all its
@@ -954,9 +962,14 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
       const uint64_t pol1 = l2_policy_evict_last();
       const uint64_t pol2 = l2_policy_evict_first();
       const int G = p.group_size;
-      int gt = 0;  // K tiles issued
-      int st = 0;  // their ring stage and its phase
-      uint32_t sph = 0;
+      // Each UMMA warp has its own sub-ring of the K stages (warp w: stages
+      // w, w + 2, ...), consumed strictly in order: a warp that skipped the
+      // other warp's tiles could otherwise wait on a stage whose previous
+      // fill has not landed and mistake an older phase for its own.
+      const int nsw = nst >> 1;
+      int sw0 = 0, sw1 = 0;       // next slot of each sub-ring
+      uint32_t sp0 = 0, sp1 = 0;  // and its phase
+      uint32_t k_used = 0, k_phase = 0;  // per stage: filled, parity of its last fill
       int qb = 0;  // Q buffer of the next chunk and its phase
       uint32_t qph = 0;
       uint32_t q_issued = 0, q_phase = 0;  // per Q buffer: loads issued, phase of the last
@@ -990,7 +1003,10 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
         }
         bool stop = false;
         for (int t = d.t0; t < d.t1; ++t) {
-          if (!F.wait_bar(empty(st), sph ^ 1u)) {
+          const int w = (t - d.t0) & 1;  // the UMMA warp (and warpgroup) of the tile
+          const int st = w + 2 * (w ? sw1 : sw0);
+          const uint32_t ph = w ? sp1 : sp0;
+          if (!F.wait_bar(empty(st), ph ^ 1u)) {
             stop = true;
             break;
           }
@@ -999,21 +1015,38 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
           const int row = row0 + t * kTileTokens;
           tma_load_3d(dst, &p.tmap_k, full(st), 0, d.g, row, pol);
           tma_load_3d(dst + kHalfTileBytes, &p.tmap_k, full(st), 64, d.g, row, pol);
-          ++gt;
-          if (++st == nst) {
-            st = 0;
-            sph ^= 1u;
+          k_used |= 1u << st;
+          k_phase = (k_phase & ~(1u << st)) | (ph << st);
+          if (w) {
+            if (++sw1 == nsw) {
+              sw1 = 0;
+              sp1 ^= 1u;
+            }
+          } else if (++sw0 == nsw) {
+            sw0 = 0;
+            sp0 ^= 1u;
           }
         }
         if (stop) break;
       }
       if (*reinterpret_cast<volatile int*>(abort_cta)) {
         // let the copies already issued land before the CTA can exit
-        for (int i = max(0, gt - nst); i < gt; ++i)
-          wait_plain(full(i % nst), static_cast<uint32_t>(i / nst) & 1u, 100000000ull);
+        for (int i = 0; i < nst; ++i)
+          if ((k_used >> i) & 1u) wait_plain(full(i), (k_phase >> i) & 1u, 100000000ull);
         for (int b = 0; b < nqb; ++b)
           if ((q_issued >> b) & 1u) wait_plain(qfull(b), (q_phase >> b) & 1u, 100000000ull);
       }
+      // Tail: the UMMA warps release a stage (empty) and a Q buffer (qempty)
+      // with tcgen05.commit arrivals that nobody else waits for at the end;
+      // wait for the last ones, so that no asynchronous arrival can land in
+      // this CTA's shared memory after it exits (bounded: after an abort some
+      // never come).
+      const uint64_t tail_ns = *reinterpret_cast<volatile int*>(abort_cta) ? 100000000ull
+                                                                           : p.wait_ns;
+      for (int i = 0; i < nst; ++i)
+        if ((k_used >> i) & 1u) wait_plain(empty(i), (k_phase >> i) & 1u, tail_ns);
+      for (int b = 0; b < nqb; ++b)
+        if ((q_issued >> b) & 1u) wait_plain(qempty(b), (q_phase >> b) & 1u, tail_ns);
     }
     __syncwarp();
   } else if (warp == kMmaWarp || warp == kMmaWarp2) {
@@ -1023,7 +1056,8 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
       const uint64_t dk0 = smem_desc_sw128(smem_u32(sK));
       const int bpw = p.nbuf / kNwg;  // TMEM buffers per warpgroup (a power of two)
       const int lbpw = __ffs(bpw) - 1;
-      int st = 0;  // ring stage of the next K tile and its phase
+      const int nsw = nst >> 1;
+      int st = 0;  // next slot of this warp's K sub-ring (stages mw, mw + 2, ...) and its phase
       uint32_t sph = 0;
       int qb = 0;  // Q buffer of the next chunk and its phase
       uint32_t qph = 0;
@@ -1043,13 +1077,7 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
         const uint64_t dq0 = smem_desc_sw128(smem_u32(sQ + qb * 2 * qh));
         bool stop = false;
         for (int t = d.t0; t < d.t1; ++t) {
-          if (((t - d.t0) & 1) != mw) {  // the other warp's tile: only the ring advances
-            if (++st == nst) {
-              st = 0;
-              sph ^= 1u;
-            }
-            continue;
-          }
+          if (((t - d.t0) & 1) != mw) continue;  // the other warp's tile
           const int kk = kw++;
           const int b = mw + kNwg * (kk & (bpw - 1));
           const uint32_t use = static_cast<uint32_t>(kk >> lbpw) & 1u;
@@ -1057,24 +1085,25 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
             stop = true;
             break;
           }
-          if (!F.wait_bar(full(st), sph)) {
+          const int stp = mw + 2 * st;  // the stage
+          if (!F.wait_bar(full(stp), sph)) {
             stop = true;
             break;
           }
           tc_fence_after();
           const uint32_t dt = tbase + static_cast<uint32_t>(b * p.tstride);
-          const uint64_t dk = dk0 + static_cast<uint64_t>((st * kTileBytes) >> 4);
+          const uint64_t dk = dk0 + static_cast<uint64_t>((stp * kTileBytes) >> 4);
 #pragma unroll
           for (int k8 = 0; k8 < kHeadDim / 16; ++k8) {
             const uint32_t koff = (k8 >> 2) * kHalfTileBytes + (k8 & 3) * 32;
             const uint32_t qoff = (k8 >> 2) * qh + (k8 & 3) * 32;
             umma_f16(dt, dk + (koff >> 4), dq0 + (qoff >> 4), idesc, k8 > 0 ? 1u : 0u);
           }
-          umma_commit(empty(st));
+          umma_commit(empty(stp));
           umma_commit(tfull(b));
           last_b = b;
           last_use = use;
-          if (++st == nst) {
+          if (++st == nsw) {
             st = 0;
             sph ^= 1u;
           }
