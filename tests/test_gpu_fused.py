@@ -186,3 +186,34 @@ def test_bounded_wait_runs_out_and_the_workspace_recovers(cuda_device):
     assert ckv.read_device_status(ws) == 0
     for l in (0, 3):
         _check_block(_block(out, cu_out, cu, l, cfg.batch, cfg.window), layers[l], cfg)
+
+
+def test_ragged_odd_chunks_repeated_calls(cuda_device):
+    """A Qwen-shaped (7 query heads per group, 4 KV heads) ragged batch over
+    several layers, lengths chosen so that many units end in chunks of one or
+    an odd number of K tiles (the two UMMA warps then take unequal shares),
+    compressed repeatedly on one workspace: every call leaves a clean device
+    status and the same bits, and one layer matches the oracle."""
+    dev = cuda_device
+    lens = [2048 * 3 + 128, 2048 + 128 * 5, 128 * 3 + 40, 2048 * 2 + 1, 8000, 128 + 33]
+    cfg = wl.get("c4").scaled(seq_len=0, n_layers=5, batch=len(lens))
+    masks = wl.srh_masks(cfg)
+    budgets = wl.layer_budgets(cfg, lens)
+    layers = [wl.make_layer(cfg, l, lengths=lens, masks=masks, budgets=budgets)
+              for l in range(cfg.n_layers)]
+    q_all, k_all, v_all, cu, b_all, m_all = _pack(layers, dev)
+    prob = ckv.Problem(q_all, k_all, cu, cfg.window, cfg.pool_width)
+    out = ckv.LayerOutputs(prob, b_all, 128, k_all.dtype, dev, scores=False)
+    ws = ckv.workspace(prob, dev)
+    first = None
+    for _ in range(12):
+        cu_out = ckv.compress_layers(prob, len(layers), q_all, k_all, v_all, m_all, b_all,
+                                     out.indices, out.k_out, out.v_out, ws)
+        torch.cuda.synchronize()
+        assert ckv.read_device_status(ws) == 0
+        got = (out.indices.clone(), out.k_out.view(torch.int16).clone())
+        if first is None:
+            first = got
+        else:
+            assert torch.equal(first[0], got[0]) and torch.equal(first[1], got[1])
+    _check_block(_block(out, cu_out, cu, 2, cfg.batch, cfg.window), layers[2], cfg)
