@@ -80,7 +80,8 @@ enum {
   CKV_ERR_WORKSPACE = -5,       /* workspace null or smaller than compresskv_workspace_size */
   CKV_ERR_CUDA = -6,            /* a CUDA runtime call or kernel launch failed */
   CKV_ERR_DEVICE_TIMEOUT = -7,  /* a kernel's bounded wait ran out (device status only) */
-  CKV_ERR_DEVICE_INDEX = -8,    /* compresskv_gather got an index outside its sequence */
+  CKV_ERR_DEVICE_INDEX = -8,    /* an index outside its sequence: given to compresskv_gather, or
+                                   produced by a selection (a device self-check) */
   CKV_ERR_STATIC_SCRATCH = -9   /* problem needs more than CKV_STATIC_SCRATCH_BYTES of scratch */
 };
 

@@ -158,8 +158,11 @@ constexpr int kFusedCtrHead = 64;       // claim / exit / abort counters before 
 // second-pass contributions (one per epilogue warp and chunk) and the state
 // of its merged softmax denominators.
 constexpr size_t kFusedCtrBytes = static_cast<size_t>(kFusedCtrHead + 3 * kFusedMaxUnits) * 4;
-constexpr int kFusedCandCap = 4096;     // top-k candidates of one unit kept in shared memory
-constexpr int kFusedCRegion = 40 * 1024;  // shared memory of the merge / select warps
+// top-k candidates of one unit kept in shared memory (more go to the unit's
+// raw-score row); with it the merge / select region leaves room for two Q
+// buffers of 192 query rows (W = 64 with three SRH heads) and two K stages
+constexpr int kFusedCandCap = 3072;
+constexpr int kFusedCRegion = 32 * 1024;  // shared memory of the merge / select warps
 
 struct FusedParams {
   CUtensorMap tmap_k;          // 3-D map over K: (d, kv head, token)

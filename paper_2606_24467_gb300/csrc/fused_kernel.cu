@@ -80,9 +80,9 @@ constexpr int kEpiWarps = 8;
 constexpr int kCWarp0 = 12;   // warps 12..19
 constexpr int kCThreads = 256;
 constexpr int kDescs = 4;     // chunk descriptors in flight (claimed ahead)
-constexpr int kNwg = 2;
+constexpr int kNwg = 2;       // epilogue warpgroups that take tiles (tile t of a chunk: t % 2)
 constexpr int kSelSamples = 1024;  // samples of a unit's pooled scores for the select threshold
-constexpr int kPub = 6;       // chunks written, not yet published (publish ring)       // epilogue warpgroups that take tiles (tile t of a chunk: t % 2)
+constexpr int kPub = 6;       // chunks written, not yet published (publish ring)
 constexpr int kBarC = 3;      // named barrier of the worker warps
 constexpr float kShift = 7.0f;
 constexpr float kRaise = 64.0f;  // fp32 sums: exponents stay below 2^64 before R is raised
@@ -94,8 +94,8 @@ constexpr int kCtrPass2 = 1;  // next pass-2 chunk
 constexpr int kCtrMerge = 2;  // next unit whose denominators to merge
 constexpr int kCtrSel = 3;    // next unit to select
 constexpr int kCtrExit = 4;   // CTAs finished
-constexpr int kCtrAbort = 5;
-constexpr int kCtrNever = 6;  // never set: the test hook's stall waits for it  // set when any wait ran out
+constexpr int kCtrAbort = 5;  // set when any wait ran out
+constexpr int kCtrNever = 6;  // never set: the test hook's stall waits for it
 
 constexpr int kTaskEnd = 0;
 constexpr int kTaskMerge = 1;

@@ -217,3 +217,22 @@ def test_ragged_odd_chunks_repeated_calls(cuda_device):
         else:
             assert torch.equal(first[0], got[0]) and torch.equal(first[1], got[1])
     _check_block(_block(out, cu_out, cu, 2, cfg.batch, cfg.window), layers[2], cfg)
+
+
+def test_wide_groups_in_a_call_of_many_masks(cuda_device):
+    """Six layers of a Llama-70B-shaped problem (8 query heads per group,
+    W = 64) with three SRH heads in every group: 192 query rows per unit, the
+    most the persistent kernel's shared memory takes with two Q buffers and a
+    K stage per UMMA warp.  More masks than the separate path takes in one
+    call, so the call must run in the persistent kernel."""
+    dev = cuda_device
+    lens = [3000, 2048 + 77]
+    cfg = wl.get("c5").scaled(seq_len=0, n_layers=6, batch=len(lens), srh_per_group=(3, 3))
+    masks = wl.srh_masks(cfg)
+    assert int(np.asarray(masks).reshape(cfg.n_layers, cfg.num_kv_heads, -1).sum(-1).min()) == 3
+    budgets = wl.layer_budgets(cfg, lens)
+    layers = [wl.make_layer(cfg, l, lengths=lens, masks=masks, budgets=budgets)
+              for l in range(cfg.n_layers)]
+    out, cu_out, cu = _run_call(layers, cfg, dev)
+    for l in (0, 5):
+        _check_block(_block(out, cu_out, cu, l, cfg.batch, cfg.window), layers[l], cfg)
