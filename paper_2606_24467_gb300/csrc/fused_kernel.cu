@@ -520,41 +520,46 @@ __device__ void emit_selected(int count, uint32_t tau, int need_eq, int32_t* out
 
 // Copy the K and V rows of out[0..count) (positions in the sequence) to the
 // compressed cache rows out0 .. out0 + count - 1 of group g.  Eight 16-byte
-// loads in flight per thread.
+// loads in flight per thread: a batch's positions are loaded first, then its
+// rows, and a position outside the sequence (never, for a correct selection)
+// is skipped and recorded after the batch, so no load waits behind another.
 __device__ __noinline__ void gather_rows(const FusedParams& p, int seq0, int L, int g,
                                          const int32_t* out, int out0, int count, int ct) {
   constexpr int kChunks = 2 * kHeadDim * 2 / 16;  // 16 K + 16 V chunks per token
   constexpr int kBatch = 8;
   const int total = count * kChunks;
+  bool bad = false;
   for (int base = 0; base < total; base += kBatch * kCThreads) {
+    int tok[kBatch];
+#pragma unroll
+    for (int k = 0; k < kBatch; ++k) {
+      const int e = base + k * kCThreads + ct;
+      tok[k] = e < total ? out[e / kChunks] : 0;
+    }
     uint4 v[kBatch];
     long long dst[kBatch];
     bool is_v[kBatch];
 #pragma unroll
     for (int k = 0; k < kBatch; ++k) {
       const int e = base + k * kCThreads + ct;
-      dst[k] = -1;
-      is_v[k] = false;
-      if (e < total) {
-        const int i = e / kChunks;
-        const int ch = e - i * kChunks;
-        const int tok = out[i];
-        if (tok < 0 || tok >= L) {  // never for a correct selection: record, skip
-          if (ch == 0) atomicCAS(p.status, 0, CKV_DEV_ERR_INDEX);
-          continue;
-        }
-        is_v[k] = ch >= kChunks / 2;
-        const int part = ch & (kChunks / 2 - 1);
-        const long long src = static_cast<long long>(seq0 + tok) * p.tok_stride_v16 +
-                              static_cast<long long>(g) * p.head_stride_v16 + part;
-        v[k] = __ldg((is_v[k] ? p.v : p.k) + src);
-        dst[k] = (static_cast<long long>(out0 + i) * p.num_kv_heads + g) * (kHeadDim * 2 / 16) + part;
-      }
+      const int i = e / kChunks;
+      const int ch = e - i * kChunks;
+      const bool ok = e < total && tok[k] >= 0 && tok[k] < L;
+      bad |= e < total && !ok;
+      is_v[k] = ch >= kChunks / 2;
+      const int part = ch & (kChunks / 2 - 1);
+      const long long src = static_cast<long long>(seq0 + (ok ? tok[k] : 0)) * p.tok_stride_v16 +
+                            static_cast<long long>(g) * p.head_stride_v16 + part;
+      dst[k] = ok ? (static_cast<long long>(out0 + i) * p.num_kv_heads + g) * (kHeadDim * 2 / 16) +
+                        part
+                  : -1;
+      if (ok) v[k] = __ldg((is_v[k] ? p.v : p.k) + src);
     }
 #pragma unroll
     for (int k = 0; k < kBatch; ++k)
       if (dst[k] >= 0) (is_v[k] ? p.v_out : p.k_out)[dst[k]] = v[k];
   }
+  if (bad) atomicCAS(p.status, 0, CKV_DEV_ERR_INDEX);
 }
 
 // Pooled score of prefix key j from the raw scores (zeros outside [0, n)),
