@@ -85,7 +85,7 @@ constexpr int kSelSamples = 1024;  // samples of a unit's pooled scores for the 
 constexpr int kPub = 6;       // chunks written, not yet published (publish ring)
 constexpr int kBarC = 3;      // named barrier of the worker warps
 constexpr float kShift = 7.0f;
-constexpr float kRaise = 64.0f;  // fp32 sums: exponents stay below 2^64 before R is raised
+constexpr float kRaiseSum = 18446744073709551616.0f;  // 2^64: fp32 column sums stay below it before R is raised
 constexpr float kNegInf = -INFINITY;
 
 // counters (ints at p.ctr)
@@ -804,7 +804,7 @@ __device__ void claim_task(const Fused& F, int* task) {
   task[1] = 0;
 }
 
-// Pass 1, rare: an exponent of this 32-column group passed 2^kRaise (or the
+// Pass 1, rare: an exponent of this 32-column group passed 2^64 (or the
 // references are still -inf): raise every query's R to kShift below its
 // largest scaled logit among the warp's 32 keys, shrink the sums kept against
 // the old R, and return this group's column sums against the new R (column
@@ -1223,7 +1223,7 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
             float e[32];  // 2^(z c - R)
             if (first && !masked) {
               // the warp's first tile of the chunk: lane 0's scaled logit is
-              // the reference of each query row (any reference within 2^kRaise
+              // the reference of each query row (any reference within 2^64
               // of the largest keeps the fp32 sums exact enough)
 #pragma unroll
               for (int j = 0; j < 32; ++j) {
@@ -1257,9 +1257,9 @@ __global__ void __launch_bounds__(kFThreads, 1) fused_kernel(const __grid_consta
               }
             }
             float colsum = warp_transpose_sum32(e, lane);  // column c0 + lane
-            // an exponent above 2^kRaise shows in its column's sum (inf/NaN
+            // an exponent above 2^64 shows in its column's sum (inf/NaN
             // when above 2^128 or with the references still -inf)
-            if (__any_sync(0xffffffffu, !(colsum <= 18446744073709551616.0f)))
+            if (__any_sync(0xffffffffu, !(colsum <= kRaiseSum)))
               colsum = p1_raise_group(taddr + c0, rf, acc_s + c0, sWpos + c0, lim, edge, key, vis,
                                       c, lane);
             acc_s[c0 + lane] += colsum;
