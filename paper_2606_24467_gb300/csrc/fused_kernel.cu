@@ -79,7 +79,7 @@ constexpr int kEpiWarp0 = 4;  // warps 4..11: two warpgroups (TMEM lane quarter 
 constexpr int kEpiWarps = 8;
 constexpr int kCWarp0 = 12;   // warps 12..19
 constexpr int kCThreads = 256;
-constexpr int kDescs = 4;     // chunk descriptors in flight (claimed ahead)
+constexpr int kDescs = 2;     // chunk descriptors in flight (claimed ahead; 2 measured faster than 4)
 constexpr int kNwg = 2;       // epilogue warpgroups that take tiles (tile t of a chunk: t % 2)
 constexpr int kSelSamples = 1024;  // samples of a unit's pooled scores for the select threshold
 constexpr int kPub = 6;       // chunks written, not yet published (publish ring)

@@ -235,11 +235,12 @@ def _simulate(seed, stages, q_bufs, bufs_per_wg, sub_rings, n_chunks=30, pub=6, 
     raise AssertionError("no progress (spinning roles only)")
 
 
-@pytest.mark.parametrize("stages,q_bufs,bufs_per_wg", [(2, 2, 4), (4, 2, 4), (4, 3, 2), (8, 2, 1),
-                                                       (6, 3, 4)])
-def test_sub_rings_survive_random_interleavings(stages, q_bufs, bufs_per_wg):
+@pytest.mark.parametrize("stages,q_bufs,bufs_per_wg,descs", [(2, 2, 4, 2), (4, 2, 4, 2), (4, 3, 2, 2),
+                                                             (8, 2, 1, 2), (6, 3, 4, 2), (4, 2, 4, 4),
+                                                             (2, 3, 2, 4)])
+def test_sub_rings_survive_random_interleavings(stages, q_bufs, bufs_per_wg, descs):
     for seed in range(25):
-        assert _simulate(seed, stages, q_bufs, bufs_per_wg, sub_rings=True)
+        assert _simulate(seed, stages, q_bufs, bufs_per_wg, sub_rings=True, descs=descs)
 
 
 def test_shared_ring_with_two_issuers_is_caught():
