@@ -236,3 +236,27 @@ def test_wide_groups_in_a_call_of_many_masks(cuda_device):
     out, cu_out, cu = _run_call(layers, cfg, dev)
     for l in (0, 5):
         _check_block(_block(out, cu_out, cu, l, cfg.batch, cfg.window), layers[l], cfg)
+
+
+def test_groups_of_every_row_class_in_one_call(cuda_device):
+    """Groups of 64, 128 and 192 query rows (one to three SRH heads at W = 64)
+    in one call, whose largest group sets the kernel's shared-memory and TMEM
+    layout for all of them.  Every layer matches the oracle, and a layer
+    compressed alone gives the same bits as inside the call."""
+    dev = cuda_device
+    lens = [2500, 2048 + 300]
+    cfg = wl.get("c5").scaled(seq_len=0, n_layers=3, batch=len(lens), srh_per_group=(1, 3))
+    masks = wl.srh_masks(cfg)
+    rows = np.asarray(masks).reshape(cfg.n_layers, cfg.num_kv_heads, -1).sum(-1) * cfg.window
+    assert {64, 128, 192} <= set(rows.ravel().tolist())
+    budgets = wl.layer_budgets(cfg, lens)
+    layers = [wl.make_layer(cfg, l, lengths=lens, masks=masks, budgets=budgets)
+              for l in range(cfg.n_layers)]
+    big, cu_out, cu = _run_call(layers, cfg, dev)
+    for l in range(cfg.n_layers):
+        _check_block(_block(big, cu_out, cu, l, cfg.batch, cfg.window), layers[l], cfg)
+    alone, cu_out1, cu1 = _run_call([layers[1]], cfg, dev)
+    a = _block(alone, cu_out1, cu1, 0, cfg.batch, cfg.window)
+    b = _block(big, cu_out, cu, 1, cfg.batch, cfg.window)
+    for key in ("raw", "pooled", "indices", "k_out", "v_out", "cu_out"):
+        assert np.array_equal(a[key], b[key]), key
