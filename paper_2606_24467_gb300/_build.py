@@ -72,7 +72,7 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | N
         objs = list(ex.map(compile_one, SOURCES))
     libdir = _cuda_lib_dir(nvcc)
     tmp = LIB_PATH + ".tmp"
-    link = [nvcc, *ARCH, "-shared", "-cudart", "shared", "-o", tmp, *objs,
+    link = [nvcc, *ARCH, "-shared", "-cudart", "shared", "-o", tmp, *objs, "-ldl",
             "-Xlinker", f"-rpath={libdir}"]
     res = subprocess.run(link, capture_output=True, text=True)
     if res.returncode != 0:

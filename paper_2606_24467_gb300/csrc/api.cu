@@ -5,6 +5,7 @@
 // in compresskv_read_device_status).
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include <algorithm>
 #include <atomic>
@@ -15,6 +16,17 @@
 
 #include "ckv_params.h"
 #include "compresskv.h"
+
+namespace {
+// A named range around each entry point for profilers (NVTX; nothing happens
+// unless a profiling tool is attached to the process).
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+}  // namespace
 
 using namespace ckv;
 
@@ -1105,6 +1117,7 @@ size_t compresskv_workspace_size(const ckv_problem* p) {
 }
 
 int compresskv_workspace_init(void* workspace, size_t workspace_bytes, void* stream) {
+  NvtxRange nvtx_range(__func__);
   if (!workspace || workspace_bytes < kHeaderBytes) return CKV_ERR_WORKSPACE;
   return cudaMemsetAsync(workspace, 0, kHeaderBytes, static_cast<cudaStream_t>(stream)) ==
                  cudaSuccess
@@ -1129,6 +1142,7 @@ int compresskv_output_layout(const ckv_problem* p, const int32_t* budgets, int32
 int compresskv_score(const ckv_problem* p, const void* q_win, const void* k,
                      const uint8_t* srh_mask, float* raw_scores, void* workspace,
                      size_t workspace_bytes, void* stream) {
+  NvtxRange nvtx_range(__func__);
   Info I;
   int rc = validate(p, I);
   if (rc != CKV_OK) return rc;
@@ -1153,6 +1167,7 @@ int compresskv_score(const ckv_problem* p, const void* q_win, const void* k,
 int compresskv_select(const ckv_problem* p, const float* raw_scores, const int32_t* budgets,
                       int32_t* indices, int32_t* cu_out, float* pooled_scores, void* workspace,
                       size_t workspace_bytes, void* stream) {
+  NvtxRange nvtx_range(__func__);
   Info I;
   int rc = validate(p, I);
   if (rc != CKV_OK) return rc;
@@ -1173,6 +1188,7 @@ int compresskv_select(const ckv_problem* p, const float* raw_scores, const int32
 int compresskv_gather(const ckv_problem* p, const int32_t* indices, const int32_t* cu_out,
                       const void* k, const void* v, void* k_out, void* v_out, void* workspace,
                       void* stream) {
+  NvtxRange nvtx_range(__func__);
   Info I;
   int rc = validate(p, I);
   if (rc != CKV_OK) return rc;
@@ -1196,6 +1212,7 @@ int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const voi
                               int32_t* indices, int32_t* cu_out, void* k_out, void* v_out,
                               float* raw_scores, float* pooled_scores, void* workspace,
                               size_t workspace_bytes, void* stream) {
+  NvtxRange nvtx_range(__func__);
   return compresskv_compress_layers(p, 1, q_win, k, v, srh_mask, budgets, indices, cu_out, k_out,
                                     v_out, raw_scores, pooled_scores, workspace, workspace_bytes,
                                     stream);
@@ -1206,6 +1223,7 @@ int compresskv_compress_layers(const ckv_problem* p, int n_masks, const void* q_
                                const int32_t* budgets, int32_t* indices, int32_t* cu_out,
                                void* k_out, void* v_out, float* raw_scores, float* pooled_scores,
                                void* workspace, size_t workspace_bytes, void* stream) {
+  NvtxRange nvtx_range(__func__);
   Info I;
   int rc = validate(p, I);
   if (rc != CKV_OK) return rc;
@@ -1259,6 +1277,7 @@ int compresskv_compress_layer_lse(const ckv_problem* p, const void* q_win, const
                                   void* k_out, void* v_out, float* raw_scores,
                                   float* pooled_scores, void* workspace, size_t workspace_bytes,
                                   void* stream) {
+  NvtxRange nvtx_range(__func__);
   return compresskv_compress_layers_lse(p, 1, q_win, k, v, lse_win, lse_batch_stride,
                                         lse_head_stride, srh_mask, budgets, indices, cu_out,
                                         k_out, v_out, raw_scores, pooled_scores, workspace,
@@ -1272,6 +1291,7 @@ int compresskv_compress_layers_lse(const ckv_problem* p, int n_masks, const void
                                    int32_t* indices, int32_t* cu_out, void* k_out, void* v_out,
                                    float* raw_scores, float* pooled_scores, void* workspace,
                                    size_t workspace_bytes, void* stream) {
+  NvtxRange nvtx_range(__func__);
   Info I;
   int rc = validate(p, I);
   if (rc != CKV_OK) return rc;
@@ -1322,6 +1342,7 @@ int compresskv_compress_layer_head_budgets(const ckv_problem* p, const void* q_w
                                            float* raw_scores, float* pooled_scores,
                                            void* workspace, size_t workspace_bytes,
                                            void* stream) {
+  NvtxRange nvtx_range(__func__);
   Info I;
   int rc = validate(p, I);
   if (rc != CKV_OK) return rc;
@@ -1469,6 +1490,7 @@ extern "C" int compresskv_compress_layer_noalloc(
     const uint8_t* srh_mask, const int32_t* budgets, int32_t* indices, int32_t* cu_out,
     void* k_out, void* v_out, float* raw_scores, float* pooled_scores, int32_t* device_status,
     void* stream) {
+  NvtxRange nvtx_range(__func__);
   Info I;
   int rc = validate(p, I);
   if (rc != CKV_OK) return rc;
