@@ -260,3 +260,41 @@ def test_groups_of_every_row_class_in_one_call(cuda_device):
     b = _block(big, cu_out, cu, 1, cfg.batch, cfg.window)
     for key in ("raw", "pooled", "indices", "k_out", "v_out", "cu_out"):
         assert np.array_equal(a[key], b[key]), key
+
+
+def test_thirty_two_query_heads_per_group(cuda_device):
+    """The most query heads per KV group the persistent kernel takes (64
+    query / 2 KV heads), the smallest window (W = 16), one to four SRH heads
+    per group, fp16, pooling width 9: every layer against the oracle."""
+    dev = cuda_device
+    lens = [1500, 2100]
+    cfg = wl.get("c1").scaled(seq_len=0, n_layers=3, batch=len(lens), num_q_heads=64,
+                              num_kv_heads=2, window=16, pool_width=9, srh_per_group=(1, 4),
+                              budget_rule="dirichlet", budget_mean=120)
+    masks = wl.srh_masks(cfg)
+    budgets = wl.layer_budgets(cfg, lens)
+    layers = [wl.make_layer(cfg, l, lengths=lens, masks=masks, budgets=budgets)
+              for l in range(cfg.n_layers)]
+    out, cu_out, cu = _run_call(layers, cfg, dev)
+    for l in range(cfg.n_layers):
+        _check_block(_block(out, cu_out, cu, l, cfg.batch, cfg.window), layers[l], cfg)
+
+
+@pytest.mark.parametrize("window,pool_width,dtype", [(16, 1, "bf16"), (48, 3, "fp16"),
+                                                     (80, 5, "bf16")])
+def test_windows_and_pool_widths(cuda_device, window, pool_width, dtype):
+    """Windows whose query rows end in a partial 32-column group (W = 48, 80)
+    or fill one exactly (W = 16 x 2 heads), pooling widths 1, 3 and 5, fp16
+    and bf16, with one or two SRH heads per group (up to 160 rows)."""
+    dev = cuda_device
+    lens = [2048 * 2 + 77, 700]
+    cfg = wl.get("c2").scaled(seq_len=0, n_layers=2, batch=len(lens), window=window,
+                              pool_width=pool_width, dtype=dtype, srh_per_group=(1, 2),
+                              budget_mean=200)
+    masks = wl.srh_masks(cfg)
+    budgets = wl.layer_budgets(cfg, lens)
+    layers = [wl.make_layer(cfg, l, lengths=lens, masks=masks, budgets=budgets)
+              for l in range(cfg.n_layers)]
+    out, cu_out, cu = _run_call(layers, cfg, dev)
+    for l in range(cfg.n_layers):
+        _check_block(_block(out, cu_out, cu, l, cfg.batch, cfg.window), layers[l], cfg)
