@@ -240,15 +240,16 @@ int compresskv_compress_layer(const ckv_problem* p, const void* q_win, const voi
  * whose scores are complete.  It reads K twice per chunk of 16 tiles of 128
  * keys: a first pass sums each query row's exponentials (softmax statistics
  * of the chunk), and once every chunk of the unit is in and the row's
- * denominator merged, a second pass (K then mostly from L2) sums the
- * normalised probabilities of each key (Eq. 1-2) in fp32; no exponent table
+ * denominator merged, a second pass sums the normalised probabilities of
+ * each key (Eq. 1-2) in fp32 from K read again (for long calls mostly from
+ * DRAM: the step then moves about twice the bytes of K); no exponent table
  * is stored.  The chunk grid is fixed per unit and every chunk's statistics
  * restart, so the scores depend only on the unit itself: compressing a layer
  * alone or among others gives the same bits.  That kernel takes windows W
  * that are multiples of 16, query strides that are multiples of 8 elements,
- * at most 32 query heads per group and SRH lists whose query rows fit its
- * shared memory beside a ring of K tiles; other per-group problems use the
- * separate kernels.
+ * at most 32 query heads per group and SRH lists of at most 192 query rows
+ * (|S_g| W: two Q buffers of them beside a ring of two K tiles fill its
+ * shared memory); other per-group problems use the separate kernels.
  * n_masks: 1 <= n_masks, dividing batch (else CKV_ERR_INVALID_ARG); at most
  *   256 under CKV_SELECT_PER_GROUP and 4 under CKV_SELECT_PER_LAYER (or when
  *   the separate kernels run) (else CKV_ERR_UNSUPPORTED).
