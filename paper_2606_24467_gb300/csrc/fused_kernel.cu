@@ -17,8 +17,9 @@
 //           log2 D_q once every chunk of the unit is in;
 //   pass 2  raw_j = sum_q 2^(z_qj c - log2 D_q) over the unit's prefix keys
 //           j < n = L - W, straight from the logits in fp32; pass 2 of a
-//           chunk is published only once its unit's denominators are merged,
-//           so it follows pass 1 closely and finds K in L2;
+//           chunk is published only once its unit's denominators are merged
+//           (it reads K again: in long calls pass 1 runs too far ahead for
+//           L2 to keep it, so mostly from DRAM);
 // then pooled_j = (sum_{t=-h..h} raw_{j+t}) / P with zeros outside [0, n)
 // (inside a chunk by the epilogue from shared memory, within h of a chunk
 // edge by the select), the k = kept - W largest pooled scores (ties to the
@@ -122,6 +123,7 @@ static_assert(3 * kMaxQRows * 4 + 16 <= kFusedCRegion, "merge scratch");
 constexpr int kWposBytes = kMaxQRows * 4;
 constexpr int kChunkBufBytes = 2 * kChunkKeys * 4;  // raw scores of two pass-2 chunks
 constexpr int kBarBytes = 512;
+static_assert((51 + 2 * kPub) * 8 <= kBarBytes, "mbarriers (the publish ring's last) fit their block");
 constexpr int kMiscBytes = 256;  // TMEM address, abort flag, task
 constexpr int kFixedBytes = kWposBytes + kChunkBufBytes + kBarBytes + kMiscBytes +
                             kDescs * static_cast<int>(sizeof(ChunkDesc));
